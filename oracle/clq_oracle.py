@@ -1,0 +1,240 @@
+"""CPU oracle for the CLQ W4A4 orthogonal-based-smoothing (OBS) linear layer.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path may import or call this
+module: only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` use it.  It shares no code with the
+CUDA path and takes every input as a plain array.
+
+Each function restates one step of the method (arxiv 2509.24416) in the
+paper's order, in plain numpy, slowly and without blocking or fusion:
+
+* Sec. 3.3 "Data Preparing": batch mean S of the calibration activations.
+* Sec. 3.3 "Outlier Detection": per-channel absolute maximum of S as the
+  outlier score; the top 50% of channels are moved to the left side.
+* Sec. 3.3 "Orthogonal Smoothing" / "Overhead Analysis": G = S_swap H with H a
+  block-diagonal +-1 Hadamard matrix; G is absorbed into the weights before
+  quantization; the activations are rotated online; only the index vector s
+  of the column swap is stored.
+* Sec. 3.1, Eq. 1 with dynamic (per-input) activation bounds: uniform
+  quantization to n = 4 bits, read here in its symmetric form l = -r.
+* The INT4 x INT4 product, accumulated exactly in int64, then dequantized in
+  fp64 with the bias added.
+
+Readings of the paper that this file fixes (the paper leaves them open):
+
+1. Permutation direction.  The swap vector s holds, at position k, the index
+   of the original column placed there (Sec. 3.3), so X_p[:, k] = X[:, s[k]].
+2. Within-half order.  The paper needs no full descending order (Sec. 3.3);
+   we rank channels by score descending with ties to the lower index, take the
+   first floor(K/2) as the high set, and list the high set then the low set,
+   each in ascending channel index.
+3. Hadamard construction.  Sylvester, natural order:
+   H_b[i, j] = (-1)^popcount(i & j), entries +-1 (Sec. 3.3), b a power of two.
+   Blocks of size b tile the row; the 50/50 split need not fall on a block
+   boundary.
+4. Normalization.  H is kept unnormalized (exact +-1 arithmetic); since
+   H_b H_b^T = b I, the product of rotated operands is divided by b once in
+   the epilogue, which is exact (b is a power of two).
+5. Symmetric 4-bit grid.  Eq. 1 with l = -r and qmax = 2^(n-1) - 1 = 7:
+   r = max |row| (dynamic for activations, Sec. 3.1; optionally clipped for
+   weights), s = r / 7 in fp32, q = clamp(rint(v / s), -7, 7) with fp32
+   division and round-half-to-even (Eq. 1 says "nearest" and leaves ties
+   open).  A zero row gets s = 0 and all-zero codes.  Code -8 is unused.
+6. Precision.  The rotation is evaluated in fp64 and rounded once to fp32.
+   For fp16 inputs every partial sum of a block is a multiple of 2^-24 below
+   2^24 in magnitude, so the fp64 sums are exact and the fp32 result is the
+   correctly rounded exact rotation.  The batch mean for the outlier score is
+   taken in fp32 (sequential sum over the batch, then one division), the same
+   precision the GPU path uses, because it decides an integer permutation.
+7. Packing.  Byte j of a packed row holds code 2j in its low nibble and code
+   2j+1 in its high nibble, as 4-bit two's complement.
+"""
+
+import numpy as np
+
+QMAX = 7  # 2^(n-1) - 1 for n = 4 bits (symmetric reading of Eq. 1)
+
+
+# ---------------------------------------------------------------- Sec. 3.3 --
+def hadamard_sylvester(b):
+    """Sylvester Hadamard matrix of order b in natural order, int64 +-1.
+
+    H[i, j] = (-1)^popcount(i & j).  Sec. 3.3 ("Orthogonal Smoothing" and the
+    +-1 storage remark under "Overhead Analysis").
+    """
+    if b < 1 or (b & (b - 1)) != 0:
+        raise ValueError("Hadamard order must be a power of two")
+    idx = np.arange(b, dtype=np.int64)
+    anded = idx[:, None] & idx[None, :]
+    parity = np.zeros((b, b), dtype=np.int64)
+    bit = 1
+    while bit < b:
+        parity ^= (anded & bit) != 0
+        bit <<= 1
+    return np.where(parity == 1, -1, 1).astype(np.int64)
+
+
+def outlier_scores(calib):
+    """Outlier score per channel from calibration activations [B, T, K].
+
+    Sec. 3.3 "Data Preparing": S = mean of X over the batch axis (fp32,
+    summed over b in order, then divided by B).  "Outlier Detection": the
+    score of channel c is max over tokens of |S[:, c]|.
+    """
+    calib = np.asarray(calib, dtype=np.float32)
+    if calib.ndim != 3:
+        raise ValueError("calibration data must be [B, T, K]")
+    B = calib.shape[0]
+    total = np.zeros(calib.shape[1:], dtype=np.float32)
+    for bi in range(B):
+        total = total + calib[bi]
+    mean = total / np.float32(B)
+    return np.max(np.abs(mean), axis=0).astype(np.float32)
+
+
+def build_permutation(scores):
+    """Column-swap vector s from outlier scores (Sec. 3.3, reading 2).
+
+    Channels whose rank (score descending, ties to the lower index) is below
+    floor(K/2) form the high-peak set, placed on the left; the rest go right.
+    Each side lists its channels in ascending index.
+    """
+    scores = np.asarray(scores, dtype=np.float32)
+    K = scores.shape[0]
+    order = sorted(range(K), key=lambda c: (-float(scores[c]), c))
+    high = sorted(order[: K // 2])
+    low = sorted(order[K // 2:])
+    return np.array(high + low, dtype=np.int32)
+
+
+def rotate_fp64(X, perm, b):
+    """X_p H_blk in fp64: gather columns by s, then multiply every length-b
+    block of the row by H_b (Sec. 3.3, G = S H applied to the activation).
+
+    Rows are independent; any float input dtype is widened exactly to fp64.
+    """
+    X = np.asarray(X).astype(np.float64)
+    perm = np.asarray(perm, dtype=np.int64)
+    M, K = X.shape
+    if K % b != 0:
+        raise ValueError("K must be a multiple of the Hadamard block size")
+    Xp = X[:, perm]
+    H = hadamard_sylvester(b).astype(np.float64)
+    return (Xp.reshape(M, K // b, b) @ H).reshape(M, K)
+
+
+def rotate(X, perm, b):
+    """Rotated rows rounded once to fp32 (reading 6)."""
+    return rotate_fp64(X, perm, b).astype(np.float32)
+
+
+# ------------------------------------------------------------ Sec. 3.1 Eq.1 --
+def quantize_symmetric(V, clip=None):
+    """Per-row symmetric INT4 quantization of fp32 rows (Eq. 1, reading 5).
+
+    Returns (codes int8 [R, K] in [-7, 7], scales fp32 [R]).  ``clip`` (one
+    fp32 bound per row, > 0) replaces the row's absolute maximum by
+    min(absmax, clip); values beyond it saturate at +-7.
+    """
+    V = np.asarray(V, dtype=np.float32)
+    amax = np.max(np.abs(V), axis=1).astype(np.float32)
+    if clip is not None:
+        amax = np.minimum(amax, np.asarray(clip, dtype=np.float32))
+    scale = (amax / np.float32(QMAX)).astype(np.float32)
+    codes = np.zeros(V.shape, dtype=np.int8)
+    nz = scale > 0
+    if np.any(nz):
+        ratio = (V[nz] / scale[nz][:, None]).astype(np.float32)
+        codes[nz] = np.clip(np.rint(ratio), -QMAX, QMAX).astype(np.int8)
+    scale = np.where(nz, scale, np.float32(0)).astype(np.float32)
+    return codes, scale
+
+
+def pack_int4(codes):
+    """Two codes per byte, code 2j in the low nibble (reading 7)."""
+    codes = np.asarray(codes, dtype=np.int8)
+    if codes.shape[1] % 2:
+        raise ValueError("row length must be even to pack")
+    lo = codes[:, 0::2].astype(np.int16) & 0xF
+    hi = codes[:, 1::2].astype(np.int16) & 0xF
+    return (lo | (hi << 4)).astype(np.uint8)
+
+
+def unpack_int4(packed):
+    """Inverse of pack_int4: sign-extend each nibble."""
+    packed = np.asarray(packed, dtype=np.uint8).astype(np.int16)
+    lo = packed & 0xF
+    hi = (packed >> 4) & 0xF
+    lo = np.where(lo >= 8, lo - 16, lo)
+    hi = np.where(hi >= 8, hi - 16, hi)
+    out = np.empty((packed.shape[0], packed.shape[1] * 2), dtype=np.int8)
+    out[:, 0::2] = lo
+    out[:, 1::2] = hi
+    return out
+
+
+def rotate_quant_act(X, perm, b):
+    """Online activation path: gather by s, block Hadamard, dynamic per-token
+    scale, codes, pack (Sec. 3.1 dynamic quantization + Sec. 3.3).
+
+    Returns (Xq uint8 [M, K/2], s_x fp32 [M], x_rot fp32 [M, K], codes int8).
+    """
+    x_rot = rotate(X, perm, b)
+    codes, s_x = quantize_symmetric(x_rot)
+    return pack_int4(codes), s_x, x_rot, codes
+
+
+def prepare_weights(W, perm, b, clip=None):
+    """Offline weight path: absorb G into W (W~ = W_p H_blk, Sec. 3.3
+    "Overhead Analysis"), then per-output-channel symmetric INT4.
+
+    W is [N, K] as in nn.Linear.  Returns (Wq uint8 [N, K/2], s_w fp32 [N],
+    w_rot fp32 [N, K], codes int8).
+    """
+    w_rot = rotate(W, perm, b)
+    codes, s_w = quantize_symmetric(w_rot, clip)
+    return pack_int4(codes), s_w, w_rot, codes
+
+
+# ------------------------------------------------------------ INT4 product --
+def int_gemm(qx, qw):
+    """acc[i, n] = sum_k qx[i, k] * qw[n, k], exact in int64."""
+    acc = np.asarray(qx, dtype=np.int64) @ np.asarray(qw, dtype=np.int64).T
+    if acc.size and np.max(np.abs(acc)) >= 2 ** 31:
+        raise OverflowError("accumulator exceeds int32")
+    return acc
+
+
+def dequant_epilogue(acc, s_x, s_w, b, bias=None):
+    """y = acc * s_x[i] * s_w[n] / b + bias[n] in fp64 (reading 4)."""
+    y = (np.asarray(acc, dtype=np.float64)
+         * np.asarray(s_x, dtype=np.float64)[:, None]
+         * np.asarray(s_w, dtype=np.float64)[None, :] / float(b))
+    if bias is not None:
+        y = y + np.asarray(bias).astype(np.float64)[None, :]
+    return y
+
+
+def w4a4_linear(Xq, s_x, Wq, s_w, b, bias=None):
+    """Packed INT4 x INT4 product with the dequant + bias epilogue.
+
+    Returns (y fp64 [M, N], acc int64 [M, N]).
+    """
+    acc = int_gemm(unpack_int4(Xq), unpack_int4(Wq))
+    return dequant_epilogue(acc, s_x, s_w, b, bias), acc
+
+
+def fused_linear(X, perm, b, Wq, s_w, bias=None):
+    """Rotate-quant of X followed by the W4A4 product (same arithmetic as the
+    two separate steps; the fusion is a GPU scheduling choice only)."""
+    Xq, s_x, _, _ = rotate_quant_act(X, perm, b)
+    y, _ = w4a4_linear(Xq, s_x, Wq, s_w, b, bias)
+    return y
+
+
+def linear_fp64(X, W, bias=None):
+    """Unquantized X W^T + bias in fp64, for reporting quantization error."""
+    y = np.asarray(X).astype(np.float64) @ np.asarray(W).astype(np.float64).T
+    if bias is not None:
+        y = y + np.asarray(bias).astype(np.float64)[None, :]
+    return y

@@ -1,0 +1,363 @@
+"""Pins for the CPU oracle: what the paper and the mathematics fix, checked
+against the oracle without using the oracle to check itself.
+
+* a hand-derived worked example (tests/golden/obs_worked_example.json);
+* H_b H_b^T = b I exactly and agreement with scipy's Sylvester matrix;
+* rotation invariance (X P H)(W P H)^T / b = X W^T (Sec. 3.3, G G^T = I);
+* one-hot rows, linearity, a dense block-diagonal product;
+* b = 1 with the identity swap reduces to textbook per-token / per-channel
+  symmetric INT4, checked against an independent scalar loop;
+* code range, abs-max hit, quantize-dequantize error bound (Eq. 1);
+* brute-force integer GEMM on tiny shapes;
+* planted mistakes in the oracle that the pins must catch.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+import scipy.linalg
+
+import oracle
+from oracle import clq_oracle as orc
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden",
+                      "obs_worked_example.json")
+
+
+def _golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+def golden_mismatches(mod):
+    """Run the worked example through module ``mod``; list what differs."""
+    g = _golden()
+    bad = []
+    X = np.array(g["X"], dtype=np.float32)
+    W = np.array(g["W"], dtype=np.float32)
+    perm = np.array(g["perm"], dtype=np.int32)
+    b = g["b"]
+    if not np.array_equal(mod.hadamard_sylvester(4), np.array(g["H4"])):
+        bad.append("H4")
+    Xq, s_x, x_rot, xc = mod.rotate_quant_act(X, perm, b)
+    if not np.array_equal(x_rot, np.array(g["x_rot"], dtype=np.float32)):
+        bad.append("x_rot")
+    if not np.array_equal(s_x, np.array(g["s_x"], dtype=np.float32)):
+        bad.append("s_x")
+    if not np.array_equal(xc, np.array(g["x_codes"])):
+        bad.append("x_codes")
+    if not np.array_equal(Xq, np.array(g["Xq"], dtype=np.uint8)):
+        bad.append("Xq")
+    Wq, s_w, w_rot, wc = mod.prepare_weights(W, perm, b)
+    if not np.array_equal(w_rot, np.array(g["w_rot"], dtype=np.float32)):
+        bad.append("w_rot")
+    if not np.array_equal(wc, np.array(g["w_codes"])):
+        bad.append("w_codes")
+    if not np.array_equal(Wq, np.array(g["Wq"], dtype=np.uint8)):
+        bad.append("Wq")
+    bias = np.array(g["bias"], dtype=np.float32)
+    y, acc = mod.w4a4_linear(Xq, s_x, Wq, s_w, b, bias)
+    if not np.array_equal(acc, np.array(g["acc"])):
+        bad.append("acc")
+    if not np.array_equal(y, np.array(g["y"])):
+        bad.append("y")
+    sc = g["scores_case"]
+    if not np.array_equal(mod.build_permutation(sc["scores"]), sc["perm"]):
+        bad.append("perm")
+    st = g["scores_tie_case"]
+    if not np.array_equal(mod.build_permutation(st["scores"]), st["perm"]):
+        bad.append("perm_tie")
+    cc = g["calib_case"]
+    if not np.array_equal(mod.outlier_scores(np.array(cc["calib"])),
+                          np.array(cc["scores"], dtype=np.float32)):
+        bad.append("scores")
+    return bad
+
+
+def test_golden_worked_example():
+    assert golden_mismatches(orc) == []
+
+
+@pytest.mark.parametrize("b", [1, 2, 4, 8, 16, 32, 64, 128, 256])
+def test_hadamard_orthogonal_and_sylvester(b):
+    H = orc.hadamard_sylvester(b)
+    assert set(np.unique(H)) <= {-1, 1}
+    assert np.array_equal(H @ H.T, b * np.eye(b, dtype=np.int64))
+    # scipy builds the same Sylvester matrix by repeated Kronecker doubling.
+    assert np.array_equal(H, scipy.linalg.hadamard(b))
+
+
+def _perm(K, seed):
+    return np.random.default_rng(seed).permutation(K).astype(np.int32)
+
+
+@pytest.mark.parametrize("b", [1, 2, 32, 64, 128, 256])
+def test_rotation_invariance(b):
+    rng = np.random.default_rng(10 + b)
+    M, N, K = 5, 7, 512
+    X = rng.standard_normal((M, K))
+    W = rng.standard_normal((N, K))
+    perm = _perm(K, b)
+    lhs = orc.rotate_fp64(X, perm, b) @ orc.rotate_fp64(W, perm, b).T / b
+    rhs = X @ W.T
+    assert np.max(np.abs(lhs - rhs)) <= 1e-12 * np.max(np.abs(rhs))
+
+
+@pytest.mark.parametrize("b", [4, 64])
+def test_one_hot_row_gives_hadamard_row(b):
+    K = 256
+    perm = _perm(K, 3)
+    inv = np.argsort(perm)
+    H = scipy.linalg.hadamard(b)
+    for c in [0, 17, 255]:
+        x = np.zeros((1, K))
+        x[0, c] = 1.0
+        r = orc.rotate_fp64(x, perm, b)[0]
+        pos = inv[c]
+        blk, off = divmod(pos, b)
+        expect = np.zeros(K)
+        expect[blk * b:(blk + 1) * b] = H[off]
+        assert np.array_equal(r, expect)
+
+
+def test_rotation_linear_and_dense_blockdiag():
+    rng = np.random.default_rng(5)
+    K, b = 128, 32
+    perm = _perm(K, 9)
+    X = rng.standard_normal((3, K))
+    Y = rng.standard_normal((3, K))
+    r = orc.rotate_fp64(2.0 * X - 0.5 * Y, perm, b)
+    assert np.allclose(r, 2.0 * orc.rotate_fp64(X, perm, b)
+                       - 0.5 * orc.rotate_fp64(Y, perm, b), atol=1e-12)
+    P = np.zeros((K, K))
+    P[perm, np.arange(K)] = 1.0          # (X P)[:, j] = X[:, perm[j]]
+    G = P @ scipy.linalg.block_diag(*([scipy.linalg.hadamard(b)] * (K // b)))
+    assert np.allclose(orc.rotate_fp64(X, perm, b), X @ G, atol=1e-12)
+
+
+def _naive_symmetric_codes(row):
+    """Textbook per-row symmetric 4-bit quantizer written as a scalar loop."""
+    amax = np.float32(0)
+    for v in row:
+        if abs(v) > amax:
+            amax = np.float32(abs(v))
+    s = np.float32(amax / np.float32(7))
+    codes = []
+    for v in row:
+        if s == 0:
+            codes.append(0)
+            continue
+        ratio = float(np.float32(np.float32(v) / s))
+        q = round(ratio)                   # Python rounds ties to even
+        codes.append(max(-7, min(7, q)))
+    return codes, s
+
+
+def test_b1_identity_is_textbook_quantization():
+    rng = np.random.default_rng(21)
+    X = (rng.standard_normal((6, 64)) * 3).astype(np.float16)
+    X[2, :] = 0
+    perm = np.arange(64, dtype=np.int32)
+    _, s_x, x_rot, codes = orc.rotate_quant_act(X, perm, 1)
+    assert np.array_equal(x_rot, X.astype(np.float32))
+    for i in range(X.shape[0]):
+        c, s = _naive_symmetric_codes(X[i].astype(np.float32))
+        assert codes[i].tolist() == c
+        assert s_x[i] == s
+
+
+def test_codes_range_absmax_and_error_bound():
+    rng = np.random.default_rng(4)
+    X = (rng.standard_normal((32, 256)) * rng.uniform(0.1, 50, (32, 1)))
+    X = X.astype(np.float16)
+    perm = _perm(256, 1)
+    _, s_x, x_rot, codes = orc.rotate_quant_act(X, perm, 64)
+    assert codes.min() >= -7 and codes.max() <= 7
+    for i in range(32):
+        j = np.argmax(np.abs(x_rot[i]))
+        assert abs(int(codes[i, j])) == 7
+    err = np.abs(x_rot.astype(np.float64)
+                 - codes.astype(np.float64) * s_x[:, None].astype(np.float64))
+    # half a step, plus fp32 rounding of the ratio
+    assert np.all(err <= s_x[:, None] * (0.5 + 1e-5))
+
+
+def test_clip_saturates():
+    rng = np.random.default_rng(8)
+    V = rng.standard_normal((4, 64)).astype(np.float32)
+    amax = np.max(np.abs(V), axis=1)
+    clip = (amax * 0.5).astype(np.float32)
+    codes, s = orc.quantize_symmetric(V, clip)
+    assert np.array_equal(s, (clip / np.float32(7)).astype(np.float32))
+    big = np.abs(V) > clip[:, None] * (7.5 / 7.0) * 1.0001
+    assert np.all(np.abs(codes[big]) == 7)
+
+
+def test_int_gemm_bruteforce():
+    rng = np.random.default_rng(2)
+    for (M, N, K) in [(1, 1, 2), (3, 5, 8), (17, 9, 64)]:
+        qx = rng.integers(-7, 8, (M, K))
+        qw = rng.integers(-7, 8, (N, K))
+        acc = orc.int_gemm(qx, qw)
+        for i in range(M):
+            for n in range(N):
+                s = 0
+                for k in range(K):
+                    s += int(qx[i, k]) * int(qw[n, k])
+                assert acc[i, n] == s
+
+
+def test_accumulator_extreme_is_exact():
+    K = 12288
+    qx = np.full((2, K), 7, dtype=np.int8)
+    qw = np.full((2, K), 7, dtype=np.int8)
+    qw[1] = -7
+    acc = orc.int_gemm(qx, qw)
+    assert acc[0, 0] == 49 * K and acc[0, 1] == -49 * K
+
+
+def test_pack_nibble_order_and_roundtrip():
+    codes = np.array([[3, -2, -7, 7, 0, -1]], dtype=np.int8)
+    packed = orc.pack_int4(codes)
+    assert packed.tolist() == [[0xE3, 0x79, 0xF0]]
+    allc = np.array([list(range(-8, 8)) * 2], dtype=np.int8)
+    assert np.array_equal(orc.unpack_int4(orc.pack_int4(allc)), allc)
+
+
+def test_outlier_scores_properties():
+    rng = np.random.default_rng(6)
+    cal = rng.standard_normal((4, 32, 16)).astype(np.float32)
+    s = orc.outlier_scores(cal)
+    # token order does not matter; scaling one channel by 4 (exact) scales it
+    assert np.array_equal(orc.outlier_scores(cal[:, ::-1, :]), s)
+    cal2 = cal.copy()
+    cal2[:, :, 3] *= 4
+    s2 = orc.outlier_scores(cal2)
+    assert s2[3] == 4 * s[3] and np.array_equal(np.delete(s2, 3),
+                                                 np.delete(s, 3))
+    # brute force on the definition
+    for c in range(16):
+        best = 0.0
+        for t in range(32):
+            m = np.float32(0)
+            for bi in range(4):
+                m = np.float32(m + cal[bi, t, c])
+            best = max(best, abs(float(np.float32(m / np.float32(4)))))
+        assert s[c] == np.float32(best)
+
+
+def test_build_permutation_properties():
+    rng = np.random.default_rng(7)
+    scores = rng.uniform(0, 1, 1152).astype(np.float32)
+    scores[rng.choice(1152, 12, replace=False)] *= 50
+    perm = orc.build_permutation(scores)
+    assert sorted(perm.tolist()) == list(range(1152))
+    left, right = perm[:576], perm[576:]
+    assert scores[left].min() >= scores[right].max()
+    assert np.all(np.diff(left) > 0) and np.all(np.diff(right) > 0)
+
+
+def test_token_permutation_equivariance():
+    rng = np.random.default_rng(11)
+    X = (rng.standard_normal((24, 128)) * 4).astype(np.float16)
+    W = (rng.standard_normal((16, 128)) * 0.02).astype(np.float16)
+    perm = _perm(128, 2)
+    Wq, s_w, _, _ = orc.prepare_weights(W, perm, 32)
+    pi = rng.permutation(24)
+    y = orc.fused_linear(X, perm, 32, Wq, s_w)
+    y_pi = orc.fused_linear(X[pi], perm, 32, Wq, s_w)
+    assert np.array_equal(y_pi, y[pi])
+
+
+def test_obs_reduces_quantization_error():
+    """Informational echo of the paper's OBS ablation (Sec. 4.2): on
+    activations with a few large-outlier channels the rotated W4A4 output is
+    closer to the fp64 product than plain per-token INT4.  (On this synthetic
+    distribution the reduction is about 30%, not the 90% the paper reports
+    for its trained models, so only the direction is asserted.)"""
+    rng = np.random.default_rng(12)
+    K, M, N = 1152, 128, 256
+    X = rng.standard_normal((M, K)).astype(np.float32)
+    ch = rng.choice(K, 8, replace=False)
+    X[:, ch] *= 40
+    X = X.astype(np.float16)
+    W = (rng.standard_normal((N, K)) * 0.02).astype(np.float16)
+    ref = orc.linear_fp64(X, W)
+    ident = np.arange(K, dtype=np.int32)
+
+    def err(perm, b):
+        Wq, s_w, _, _ = orc.prepare_weights(W, perm, b)
+        y = orc.fused_linear(X, perm, b, Wq, s_w)
+        return np.linalg.norm(y - ref) / np.linalg.norm(ref)
+
+    cal = X.astype(np.float32)[None]
+    perm = orc.build_permutation(orc.outlier_scores(cal))
+    e_plain, e_obs = err(ident, 1), err(perm, 64)
+    assert e_obs < 0.8 * e_plain
+
+
+# ----------------------------------------------------- planted mistakes ----
+def _rotate_scatter(X, perm, b):
+    # wrong direction: X_p[:, perm[k]] = X[:, k]
+    X = np.asarray(X).astype(np.float64)
+    Xp = np.empty_like(X)
+    Xp[:, np.asarray(perm)] = X
+    H = orc.hadamard_sylvester(b).astype(np.float64)
+    M, K = X.shape
+    return (Xp.reshape(M, K // b, b) @ H).reshape(M, K)
+
+
+def _hadamard_sequency(b):
+    # right matrix family, wrong row order (Walsh / sequency order)
+    H = scipy.linalg.hadamard(b)
+    return H[np.argsort([np.count_nonzero(np.diff(r)) for r in H])]
+
+
+def _quantize_half_away(V, clip=None):
+    V = np.asarray(V, dtype=np.float32)
+    amax = np.max(np.abs(V), axis=1).astype(np.float32)
+    s = (amax / np.float32(7)).astype(np.float32)
+    r = V / np.where(s > 0, s, 1)[:, None]
+    q = np.sign(r) * np.floor(np.abs(r) + 0.5)
+    return np.clip(q, -7, 7).astype(np.int8), s
+
+
+def _pack_swapped(codes):
+    codes = np.asarray(codes, dtype=np.int8)
+    lo = codes[:, 1::2].astype(np.int16) & 0xF
+    hi = codes[:, 0::2].astype(np.int16) & 0xF
+    return (lo | (hi << 4)).astype(np.uint8)
+
+
+def _epilogue_no_b(acc, s_x, s_w, b, bias=None):
+    y = acc * s_x[:, None].astype(np.float64) * s_w[None, :]
+    return y + (0 if bias is None else bias[None, :].astype(np.float64))
+
+
+def _perm_descending(scores):
+    return np.argsort(-np.asarray(scores), kind="stable").astype(np.int32)
+
+
+def _scores_no_mean(calib):
+    return np.max(np.max(np.abs(np.asarray(calib, np.float32)), axis=0),
+                  axis=0)
+
+
+@pytest.mark.parametrize("name,fn", [
+    ("rotate_fp64", _rotate_scatter),
+    ("hadamard_sylvester", _hadamard_sequency),
+    ("quantize_symmetric", _quantize_half_away),
+    ("pack_int4", _pack_swapped),
+    ("dequant_epilogue", _epilogue_no_b),
+    ("build_permutation", _perm_descending),
+    ("outlier_scores", _scores_no_mean),
+])
+def test_planted_mistake_is_caught(monkeypatch, name, fn):
+    assert golden_mismatches(orc) == []
+    monkeypatch.setattr(orc, name, fn)
+    assert golden_mismatches(orc) != [], name
+
+
+def test_package_reexports():
+    assert oracle.QMAX == 7 and oracle.hadamard_sylvester is not None
