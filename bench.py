@@ -1,0 +1,452 @@
+"""Benchmark of the W4A4 OBS linear layer set on GB300.
+
+One step = the online hot path of every layer of one DiT block (default: the
+PixArt-alpha block at 1024 px, M = 8192 tokens, hidden 1152, b = 64, fp16):
+for each of QKV, attention-out, FFN-up and FFN-down, clq_rotate_quant_act
+then clq_w4a4_linear (or clq_fused_linear with --fused).  Weight preparation
+is offline and untimed.  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl clq|reference]
+
+--impl reference times the CPU oracle on the host cores (bounded row sample
+per step) as the reference arm.  Under torchrun every rank runs its own batch
+(independent tokens; no collective on the data path): weak scaling.
+"""
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("W4A4 linear effective TOPS & us/layer; % INT8 tensor peak; "
+          "rotate-quant HBM GB/s")
+L2_BYTES = 129 * 1024 * 1024
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=300)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", default="clq", choices=["clq", "reference"])
+    p.add_argument("--workload", default="pixart_1024")
+    p.add_argument("--fused", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def layer_ops(cfg, M=None):
+    M = cfg["M"] if M is None else M
+    return [2.0 * M * N * K for (_, K, N) in cfg["layers"]]
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, 1900.0, "fallback"
+
+
+def kernel_source_sha():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2509_24416_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken
+    on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except (OSError, ValueError):
+        return None
+    e = d.get(kernel, {}).get(workload)
+    if not e or e.get("source_sha") != kernel_source_sha():
+        return None
+    return e.get("bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,"
+         "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.proc = None
+
+    def start(self):
+        cmd = ["nvidia-smi", "--query-gpu=" + self.Q, "--format=csv,noheader,nounits",
+               "-lms", "50"]
+        if self.uuid:
+            cmd += ["-i", self.uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------- CPU oracle --
+def _oracle_sample_worker(args):
+    """Runs in a fresh (spawned) single-threaded process."""
+    workload, rows, reps = args
+    import oracle
+    from paper_2509_24416_gb300 import synth
+    cfg = synth.WORKLOADS[workload]
+    prepared = []
+    for li in range(len(cfg["layers"])):
+        d = synth.layer_inputs(cfg, li, M=rows)
+        perm = oracle.build_permutation(oracle.outlier_scores(d["calib"]))
+        Wq, s_w, _, _ = oracle.prepare_weights(d["W32"], perm, cfg["b"])
+        prepared.append((d["X32"], perm, Wq, s_w, d["bias32"]))
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        for (x, perm, Wq, s_w, bias) in prepared:
+            Xq, s_x, _, _ = oracle.rotate_quant_act(x, perm, cfg["b"])
+            oracle.w4a4_linear(Xq, s_x, Wq, s_w, cfg["b"], bias)
+        times.append(time.perf_counter() - t0)
+    return times
+
+
+def run_oracle(workload, rows, reps):
+    import multiprocessing as mp
+    env = {"OMP_NUM_THREADS": "1", "OPENBLAS_NUM_THREADS": "1",
+           "MKL_NUM_THREADS": "1"}
+    old = {k: os.environ.get(k) for k in env}
+    os.environ.update(env)
+    try:
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(1) as pool:
+            return pool.apply(_oracle_sample_worker, ((workload, rows, reps),))
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+
+
+def cpu_baseline(workload, budget_s=20.0):
+    from paper_2509_24416_gb300 import synth
+    cfg = synth.WORKLOADS[workload]
+    probe_rows = 16
+    t = run_oracle(workload, probe_rows, 1)[0]
+    rows = int(max(16, min(cfg["M"], probe_rows * budget_s / max(t, 1e-3) / 2)))
+    times = run_oracle(workload, rows, 2)
+    sec = min(times)
+    ops = sum(layer_ops(cfg, rows))
+    return {"value": ops / sec / 1e12, "unit": "TOPS", "cores": 1,
+            "kind": "oracle",
+            "sample": "%d of %d tokens per layer, all %d layers, rotate-quant + "
+                      "int64 GEMM + fp64 epilogue, numpy single-threaded, best of 2"
+                      % (rows, cfg["M"], len(cfg["layers"]))}
+
+
+def reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2509_24416_gb300 import synth
+    cfg = synth.WORKLOADS[args.workload]
+    n = args.steps + args.warmup
+    t = run_oracle(args.workload, 16, 1)[0]
+    per_step_budget = 150.0 / max(n, 1)
+    rows = int(max(1, min(cfg["M"], 16 * per_step_budget / max(t, 1e-3))))
+    times = run_oracle(args.workload, rows, n)[args.warmup:]
+    sec = float(np.sum(times))
+    ops = sum(layer_ops(cfg, rows)) * args.steps
+    value = ops / sec / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * sec / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64/int64",
+        "data": "synthetic", "config": config_dict(cfg, args),
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1,
+                         "kind": "oracle",
+                         "sample": "%d of %d tokens per layer per step" % (rows, cfg["M"])},
+        "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_dict(cfg, args):
+    return {"workload": args.workload, "tokens": cfg["M"], "b": cfg["b"],
+            "layers": ["%s %dx%d" % (n, K, N) for (n, K, N) in cfg["layers"]],
+            "io_dtype": cfg["dtype"], "path": "fused" if args.fused else "separate",
+            "l2": "inputs rotated over sets totalling > 2x L2 (129 MB)"}
+
+
+# --------------------------------------------------------------- GPU arm ---
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+        return
+    import torch
+    import torch.distributed as dist
+    from paper_2509_24416_gb300 import clq, synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    clq.load()
+    cfg = synth.WORKLOADS[args.workload]
+    td = {"f16": torch.float16, "bf16": torch.bfloat16}[cfg["dtype"]]
+    b = cfg["b"]
+    M = cfg["M"]
+
+    # ---- offline: calibration, swap vectors, prepared weights (untimed) ----
+    layers, xs_host = [], []
+    for li in range(len(cfg["layers"])):
+        d = synth.layer_inputs(cfg, li)
+        calib = torch.from_numpy(d["calib"]).to(td).to(dev)
+        perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
+        lay = clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b,
+                                             bias=d["bias"].to(dev))
+        layers.append((d["name"], d["K"], d["N"], lay))
+        xs_host.append(d["X"])
+    set_bytes = sum(x.numel() * 2 for x in xs_host)
+    nsets = max(2, math.ceil(2 * L2_BYTES / set_bytes) + 1)
+    xsets = [[x.to(dev) for x in xs_host] for _ in range(nsets)]
+    xq = [torch.empty((M, K // 2), dtype=torch.uint8, device=dev) for (_, K, _, _) in layers]
+    sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in layers]
+    ys = [torch.empty((M, N), dtype=td, device=dev) for (_, _, N, _) in layers]
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    nlay = len(layers)
+
+    def step(si, ev=None):
+        xs = xsets[si % nsets]
+        for i, (_, K, N, lay) in enumerate(layers):
+            if ev is not None:
+                ev[4 * i].record(stream)
+            if args.fused:
+                st = clq.clq_fused_linear(xs[i].data_ptr(), clq._dt(xs[i]), M, K, K,
+                                          lay.perm.data_ptr(), b, lay.Wq.data_ptr(),
+                                          lay.s_w.data_ptr(), lay.bias.data_ptr(), N,
+                                          ys[i].data_ptr(), sp)
+                if st:
+                    raise clq.ClqError(st, "clq_fused_linear")
+                if ev is not None:
+                    ev[4 * i + 1].record(stream)
+                    ev[4 * i + 2].record(stream)
+            else:
+                st = clq.clq_rotate_quant_act(xs[i].data_ptr(), clq._dt(xs[i]), M, K, K,
+                                              lay.perm.data_ptr(), b, xq[i].data_ptr(),
+                                              sx[i].data_ptr(), None, sp)
+                if st:
+                    raise clq.ClqError(st, "clq_rotate_quant_act")
+                if ev is not None:
+                    ev[4 * i + 1].record(stream)
+                    ev[4 * i + 2].record(stream)
+                st = clq.clq_w4a4_linear(xq[i].data_ptr(), sx[i].data_ptr(),
+                                         lay.Wq.data_ptr(), lay.s_w.data_ptr(),
+                                         lay.bias.data_ptr(), M, N, K, b, clq._dt(ys[i]),
+                                         ys[i].data_ptr(), None, sp)
+                if st:
+                    raise clq.ClqError(st, "clq_w4a4_linear")
+            if ev is not None:
+                ev[4 * i + 3].record(stream)
+
+    # warm-up, then a clock settle of ~1 s of untimed steps
+    for i in range(max(3, args.warmup)):
+        step(i)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    n_settle = 0
+    while time.perf_counter() - t0 < 1.0:
+        step(n_settle)
+        n_settle += 1
+        if n_settle % 50 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        uuid = None
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    time.sleep(0.3)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4 * nlay)]
+           for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for k in range(args.steps):
+        step(k, evs[k])
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    status = clq.device_status()
+    if status != 0:
+        raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
+
+    total_ms = evs[0][0].elapsed_time(evs[-1][-1])
+    rq_ms = np.zeros(nlay)
+    gm_ms = np.zeros(nlay)
+    for e in evs:
+        for i in range(nlay):
+            rq_ms[i] += e[4 * i].elapsed_time(e[4 * i + 1])
+            gm_ms[i] += e[4 * i + 2].elapsed_time(e[4 * i + 3])
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    ops_step = sum(layer_ops(cfg))
+    value = ops_step * args.steps * world / (total_ms * 1e-3) / 1e12
+    hbm_peak, bf16_peak, peak_src = peaks()
+    fp8_peak = 2.0 * bf16_peak  # E4M3 dense rate = 2x bf16 (nominal ratio)
+    K_list = [K for (_, K, _, _) in layers]
+    N_list = [N for (_, _, N, _) in layers]
+    per_layer = []
+    gemm_flops = sum(layer_ops(cfg))
+    for i, (name, K, N, _) in enumerate(layers):
+        rq_us = 1e3 * rq_ms[i] / args.steps
+        gm_us = 1e3 * gm_ms[i] / args.steps
+        rq_bytes = M * (2.5 * K + 4)
+        per_layer.append({
+            "layer": name, "K": K, "N": N,
+            "us": round(rq_us + gm_us, 2),
+            "rotate_quant_us": round(rq_us, 2),
+            "rotate_quant_GBps": round(rq_bytes / (rq_us * 1e-6) / 1e9, 1) if rq_us > 0 else None,
+            "gemm_us": round(gm_us, 2),
+            "gemm_TOPS": round(2.0 * M * N * K / (gm_us * 1e-6) / 1e12, 1),
+        })
+    gm_total_s = gm_ms.sum() * 1e-3 / args.steps
+    rq_total_s = rq_ms.sum() * 1e-3 / args.steps
+    gemm_kernel = "fused_linear" if args.fused else "w4a4_gemm"
+    achieved = gemm_flops / gm_total_s / 1e12
+    rq_bytes_all = sum(M * (2.5 * K + 4) for K in K_list)
+    roofline = {"kernel": gemm_kernel, "bound": "tensor", "achieved": round(achieved, 1),
+                "peak": fp8_peak, "unit": "TFLOP/s", "frac": round(achieved / fp8_peak, 4),
+                "traffic": recorded_traffic(gemm_kernel, args.workload),
+                "peak_note": "E4M3 kind::f8f6f4 dense = 2 x bf16 %s (%s)" % (bf16_peak, peak_src)}
+    rq_roof = None
+    if not args.fused:
+        rq_ach = rq_bytes_all / rq_total_s / 1e9
+        rq_roof = {"kernel": "rotate_quant", "bound": "hbm", "achieved": round(rq_ach, 1),
+                   "peak": hbm_peak, "unit": "GB/s", "frac": round(rq_ach / hbm_peak, 4),
+                   "frac_of_8TBps": round(rq_ach / 8000.0, 4),
+                   "traffic": recorded_traffic("rotate_quant", args.workload)}
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        xh = [x.pin_memory() for x in xs_host]
+        yh = [torch.empty((M, N), dtype=td).pin_memory() for N in N_list]
+        xd = xsets[0]
+        h2d = sum(x.numel() * 2 for x in xh)
+        d2h = sum(y.numel() * 2 for y in yh)
+        reps = max(3, min(args.steps, 30))
+
+        def e2e_step():
+            for i, (_, K, N, lay) in enumerate(layers):
+                xd[i].copy_(xh[i], non_blocking=True)
+                Y = lay(xd[i], fused=args.fused)
+                yh[i].copy_(Y, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            e2e_step()
+        z.record(stream)
+        torch.cuda.synchronize()
+        e2e_s = a.elapsed_time(z) * 1e-3 / reps
+        e2e = {"value": ops_step * world / e2e_s / 1e12, "unit": "TOPS",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": round(e2e_s * 1e3, 3)}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args.workload)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "TOPS",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3-int4/f32",
+            "data": "synthetic (seeded Philox, DiT-shaped; no model weights)",
+            "config": config_dict(cfg, args), "roofline": roofline,
+            "roofline_rotate_quant": rq_roof, "per_layer": per_layer,
+            "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": (1 if args.fused else 2) * nlay * args.steps,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

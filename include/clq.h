@@ -1,0 +1,164 @@
+/*
+ * clq.h - C ABI of libclq, the GB300 (sm_103a) inference path of CLQ's
+ * W4A4 orthogonal-based-smoothing (OBS) linear layer, arxiv 2509.24416.
+ *
+ * The layer computes Y = X W^T + bias with both operands quantized to 4 bits
+ * after the OBS transform G = S H (Sec. 3.3): S is a column swap stored as
+ * an index vector `perm` (position k holds the original column perm[k]) and
+ * H = diag(H_b, ..., H_b) with H_b the Sylvester Hadamard matrix of order b,
+ * H_b[i][j] = (-1)^popcount(i & j).  G is absorbed into W offline; the
+ * activations are rotated online with a fast Walsh-Hadamard transform and
+ * quantized per token with dynamic bounds (Sec. 3.1).  Quantization is the
+ * symmetric reading of Eq. 1: r = max|row| (optionally clipped), s = r / 7
+ * in fp32, q = clamp(rint(v / s), -7, 7), ties to even, code -8 unused.
+ * H is unnormalized (H_b H_b^T = b I), so the epilogue divides by b once:
+ *     Y[i][n] = acc[i][n] * s_x[i] * s_w[n] / b + bias[n],
+ *     acc[i][n] = sum_k qx[i][k] * qw[n][k]  (exact integer).
+ *
+ * Conventions for every call:
+ *  - Returns a clq_status; 0 (CLQ_OK) on success.  No exception or abort
+ *    crosses the ABI.  Arguments are validated on the host before anything is
+ *    launched; on an error nothing is launched and no output is touched.
+ *  - Tensor pointers are DEVICE pointers owned by the caller unless the name
+ *    starts with host_.  The library allocates, frees and synchronizes
+ *    nothing in these calls (clq_get_device_status synchronizes by design).
+ *  - Launches are asynchronous on `stream` (a cudaStream_t passed as void*;
+ *    NULL is the legacy default stream).
+ *  - Row-major layouts; `ld*` arguments are row strides in ELEMENTS.
+ *  - Packed INT4 rows: byte j holds code 2j in its low nibble and code 2j+1
+ *    in its high nibble, 4-bit two's complement.  A packed row of K codes is
+ *    K/2 bytes and rows are contiguous (stride K/2).
+ *  - Shape rules: 1 <= b <= 256 and b a power of two; K % 32 == 0,
+ *    K % b == 0, 32 <= K <= 32768; M, N >= 0 (0 is an empty no-op);
+ *    ld* >= K and ld* % 8 == 0; every pointer 16-byte aligned.
+ *  - Device-side faults the host cannot see (an index in `perm` outside
+ *    [0, K), a pipeline wait that exceeds its time limit) are recorded in a
+ *    device status word read by clq_get_device_status; the kernel skips the
+ *    offending access instead of faulting.
+ *  - The library keeps no per-call state and is safe to call from several
+ *    host threads.
+ */
+#ifndef CLQ_H
+#define CLQ_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t clq_status;
+#define CLQ_OK 0
+#define CLQ_ERR_INVALID_ARG 1 /* null pointer, bad enum, negative size    */
+#define CLQ_ERR_SHAPE 2       /* shape rule above violated                 */
+#define CLQ_ERR_ALIGN 3       /* pointer or stride not 16-byte aligned     */
+#define CLQ_ERR_UNSUPPORTED 4 /* no usable sm_103a device / feature        */
+#define CLQ_ERR_CUDA 5        /* a CUDA runtime call failed                */
+#define CLQ_ERR_TIMEOUT 6     /* a bounded device-side wait ran out        */
+#define CLQ_ERR_DEVICE_INDEX 7 /* perm held an index outside [0, K)        */
+
+typedef int32_t clq_dtype;
+#define CLQ_F16 0
+#define CLQ_BF16 1
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* clq_status_string(clq_status status);
+
+/* ABI version, major * 100 + minor. */
+int32_t clq_version(void);
+
+/*
+ * Outlier score per input channel (Sec. 3.3, "Data Preparing" and "Outlier
+ * Detection"): S = mean over the batch of calib[B][T][K] (fp32, summed over
+ * the batch in order, then divided by B), score[k] = max_t |S[t][k]|.
+ * calib: device, dtype `dtype`, contiguous [B][T][K].  scores: device fp32
+ * [K].  Requires B, T, K >= 1.  Offline; not on the timed path.
+ */
+clq_status clq_outlier_scores(const void* calib, clq_dtype dtype, int32_t B,
+                              int32_t T, int32_t K, float* scores,
+                              void* stream);
+
+/*
+ * Column-swap vector from outlier scores (Sec. 3.3, "Outlier Detection"):
+ * rank channels by score descending (ties to the lower index); the first
+ * K/2 (rounded down) form the high-peak set, placed left, the rest right,
+ * each side in ascending channel index.  HOST pointers: host_scores [K],
+ * host_perm [K] (written).  Requires K >= 1; NaN scores are rejected.
+ */
+clq_status clq_build_permutation(const float* host_scores, int32_t K,
+                                 int32_t* host_perm);
+
+/*
+ * Offline weight preparation (Sec. 3.3, "Overhead Analysis": W~ = G^T-side
+ * absorption, here W~ = W_p H with W_p[n][k] = W[n][perm[k]]), then
+ * per-output-channel symmetric INT4: s_w[n] = min(max_k |W~[n][k]|,
+ * clip[n]) / 7, Wq[n] = pack(clamp(rint(W~[n] / s_w[n]), -7, 7)).
+ * W: device [N][ldw] of `dtype`.  perm: device int32 [K].  clip: device fp32
+ * [N] (> 0) or NULL for no clipping.  Wq: device uint8 [N][K/2].  s_w:
+ * device fp32 [N].  w_rot_dbg: device fp32 [N][K] or NULL; when given it
+ * receives W~ (the fp32 rotated rows) for parity checks.
+ */
+clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N,
+                               int32_t K, int32_t ldw, const int32_t* perm,
+                               int32_t b, const float* clip, uint8_t* Wq,
+                               float* s_w, float* w_rot_dbg, void* stream);
+
+/*
+ * Online activation rotate + quantize (Sec. 3.1 dynamic quantization with
+ * Sec. 3.3's online fast Hadamard): X~ = X_p H in fp32, s_x[i] =
+ * max_k |X~[i][k]| / 7, Xq[i] = pack(clamp(rint(X~[i] / s_x[i]), -7, 7)).
+ * One HBM pass over X.  X: device [M][ldx] of `dtype`.  perm: device int32
+ * [K].  Xq: device uint8 [M][K/2].  s_x: device fp32 [M].  x_rot_dbg: device
+ * fp32 [M][K] or NULL (receives X~).
+ */
+clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M,
+                                int32_t K, int32_t ldx, const int32_t* perm,
+                                int32_t b, uint8_t* Xq, float* s_x,
+                                float* x_rot_dbg, void* stream);
+
+/*
+ * Packed INT4 x INT4 product with the dequant + bias epilogue:
+ * Y[i][n] = out_dtype(acc[i][n] * s_x[i] * s_w[n] / b + bias[n]).
+ * Xq: device uint8 [M][K/2]; s_x: device fp32 [M]; Wq: device uint8
+ * [N][K/2]; s_w: device fp32 [N]; bias: device [N] of `out_dtype` or NULL;
+ * Y: device [M][N] of `out_dtype`.  acc_dbg: device int32 [M][N] or NULL;
+ * when given it receives the exact integer accumulators.
+ */
+clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x,
+                           const uint8_t* Wq, const float* s_w,
+                           const void* bias, int32_t M, int32_t N, int32_t K,
+                           int32_t b, clq_dtype out_dtype, void* Y,
+                           int32_t* acc_dbg, void* stream);
+
+/*
+ * The whole layer in one kernel: clq_rotate_quant_act fused into the GEMM
+ * prologue, so the activation codes never reach HBM.  Same arithmetic and
+ * results as the two separate calls.  X: device [M][ldx] of `dtype`; Y:
+ * device [M][N] of `dtype`; bias: device [N] of `dtype` or NULL.
+ */
+clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M,
+                            int32_t K, int32_t ldx, const int32_t* perm,
+                            int32_t b, const uint8_t* Wq, const float* s_w,
+                            const void* bias, int32_t N, void* Y,
+                            void* stream);
+
+/*
+ * Synchronize `stream`, then read and clear the device status word of the
+ * current device: *out receives CLQ_OK or the first device-side error
+ * recorded since the last read.
+ */
+clq_status clq_get_device_status(void* stream, int32_t* out);
+
+/*
+ * Self-test of the bounded-wait machinery: launches one CTA that waits on an
+ * mbarrier nothing will ever complete, with a limit of timeout_ns
+ * nanoseconds (1e3 .. 1e9).  The wait must give up, record CLQ_ERR_TIMEOUT
+ * in the device status word and return, leaving the context usable.
+ */
+clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CLQ_H */

@@ -1,0 +1,284 @@
+"""Python binding of libclq (include/clq.h): argument marshalling only.
+
+Two layers:
+
+* ``clq_*`` functions with the C names and C arguments (integers for device
+  pointers and the stream), returning the status code;
+* tensor helpers (``rotate_quant_act``, ``w4a4_linear`` ...) that take torch
+  tensors, allocate outputs with torch, pass their pointers and the current
+  stream to the C call, and raise ``ClqError`` on a non-zero status.
+
+Every step of the computation runs in the CUDA kernels of libclq.so; there is
+no CPU or PyTorch fallback.  If the library is missing, the first call raises.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libclq.so")
+
+CLQ_F16, CLQ_BF16 = 0, 1
+STATUS = {0: "CLQ_OK", 1: "CLQ_ERR_INVALID_ARG", 2: "CLQ_ERR_SHAPE",
+          3: "CLQ_ERR_ALIGN", 4: "CLQ_ERR_UNSUPPORTED", 5: "CLQ_ERR_CUDA",
+          6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX"}
+EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
+           "clq_build_permutation", "clq_prepare_weights",
+           "clq_rotate_quant_act", "clq_w4a4_linear", "clq_fused_linear",
+           "clq_get_device_status", "clq_selftest_bounded_wait")
+
+_lib = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int32
+_SIGS = {
+    "clq_status_string": (ctypes.c_char_p, [_I]),
+    "clq_version": (_I, []),
+    "clq_outlier_scores": (_I, [_P, _I, _I, _I, _I, _P, _P]),
+    "clq_build_permutation": (_I, [_P, _I, _P]),
+    "clq_prepare_weights": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P,
+                                 _P]),
+    "clq_rotate_quant_act": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P,
+                                  _P]),
+    "clq_w4a4_linear": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P,
+                             _P]),
+    "clq_fused_linear": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _P,
+                              _P]),
+    "clq_get_device_status": (_I, [_P, _P]),
+    "clq_selftest_bounded_wait": (_I, [ctypes.c_int64, _P]),
+}
+
+
+class ClqError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = int(status)
+        super().__init__("%s failed: %s" % (where, status_string(status)))
+
+
+def load():
+    """Load libclq.so (built in-tree by ``build.build()``)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libclq.so is not built (%s); run "
+                               "paper_2509_24416_gb300.build.build()"
+                               % LIB_PATH)
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+def status_string(status):
+    try:
+        return load().clq_status_string(int(status)).decode()
+    except RuntimeError:
+        return STATUS.get(int(status), "unknown")
+
+
+# ------------------------------------------------- C-named raw entry points --
+def clq_outlier_scores(calib, dtype, B, T, K, scores, stream):
+    return load().clq_outlier_scores(calib, dtype, B, T, K, scores, stream)
+
+
+def clq_build_permutation(host_scores, K, host_perm):
+    return load().clq_build_permutation(host_scores, K, host_perm)
+
+
+def clq_prepare_weights(W, dtype, N, K, ldw, perm, b, clip, Wq, s_w,
+                        w_rot_dbg, stream):
+    return load().clq_prepare_weights(W, dtype, N, K, ldw, perm, b, clip, Wq,
+                                      s_w, w_rot_dbg, stream)
+
+
+def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, Xq, s_x, x_rot_dbg,
+                         stream):
+    return load().clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, Xq, s_x,
+                                       x_rot_dbg, stream)
+
+
+def clq_w4a4_linear(Xq, s_x, Wq, s_w, bias, M, N, K, b, out_dtype, Y,
+                    acc_dbg, stream):
+    return load().clq_w4a4_linear(Xq, s_x, Wq, s_w, bias, M, N, K, b,
+                                  out_dtype, Y, acc_dbg, stream)
+
+
+def clq_fused_linear(X, dtype, M, K, ldx, perm, b, Wq, s_w, bias, N, Y,
+                     stream):
+    return load().clq_fused_linear(X, dtype, M, K, ldx, perm, b, Wq, s_w,
+                                   bias, N, Y, stream)
+
+
+def clq_get_device_status(stream, out):
+    return load().clq_get_device_status(stream, out)
+
+
+def clq_selftest_bounded_wait(timeout_ns, stream):
+    return load().clq_selftest_bounded_wait(timeout_ns, stream)
+
+
+# ----------------------------------------------------------- tensor helpers --
+def _dt(t):
+    if t.dtype == torch.float16:
+        return CLQ_F16
+    if t.dtype == torch.bfloat16:
+        return CLQ_BF16
+    raise TypeError("expected float16 or bfloat16, got %s" % t.dtype)
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def _check(st, where):
+    if st != 0:
+        raise ClqError(st, where)
+
+
+def _row_major(t, name):
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("%s must be a 2-D tensor with unit column stride"
+                         % name)
+
+
+def outlier_scores(calib, stream=None):
+    """calib [B, T, K] fp16/bf16 on the GPU -> fp32 scores [K]."""
+    calib = calib.contiguous()
+    B, T, K = calib.shape
+    scores = torch.empty(K, dtype=torch.float32, device=calib.device)
+    _check(clq_outlier_scores(_ptr(calib), _dt(calib), B, T, K, _ptr(scores),
+                              _stream(stream)), "clq_outlier_scores")
+    return scores
+
+
+def build_permutation(scores):
+    """Host column-swap vector from scores (any device) -> int32 CPU [K]."""
+    s = scores.detach().to("cpu", torch.float32).contiguous()
+    K = s.numel()
+    perm = torch.empty(K, dtype=torch.int32)
+    _check(clq_build_permutation(_ptr(s), K, _ptr(perm)),
+           "clq_build_permutation")
+    return perm
+
+
+def prepare_weights(W, perm, b, clip=None, with_rot=False, stream=None):
+    """W [N, K] -> (Wq uint8 [N, K/2], s_w fp32 [N][, w_rot fp32 [N, K]])."""
+    _row_major(W, "W")
+    N, K = W.shape
+    dev = W.device
+    Wq = torch.empty((N, K // 2), dtype=torch.uint8, device=dev)
+    s_w = torch.empty(N, dtype=torch.float32, device=dev)
+    rot = (torch.empty((N, K), dtype=torch.float32, device=dev)
+           if with_rot else None)
+    _check(clq_prepare_weights(_ptr(W), _dt(W), N, K, W.stride(0), _ptr(perm),
+                               b, _ptr(clip), _ptr(Wq), _ptr(s_w), _ptr(rot),
+                               _stream(stream)), "clq_prepare_weights")
+    return (Wq, s_w, rot) if with_rot else (Wq, s_w)
+
+
+def rotate_quant_act(X, perm, b, Xq=None, s_x=None, with_rot=False,
+                     stream=None):
+    """X [M, K] -> (Xq uint8 [M, K/2], s_x fp32 [M][, x_rot fp32 [M, K]])."""
+    _row_major(X, "X")
+    M, K = X.shape
+    dev = X.device
+    if Xq is None:
+        Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+    if s_x is None:
+        s_x = torch.empty(M, dtype=torch.float32, device=dev)
+    rot = (torch.empty((M, K), dtype=torch.float32, device=dev)
+           if with_rot else None)
+    _check(clq_rotate_quant_act(_ptr(X), _dt(X), M, K, X.stride(0),
+                                _ptr(perm), b, _ptr(Xq), _ptr(s_x), _ptr(rot),
+                                _stream(stream)), "clq_rotate_quant_act")
+    return (Xq, s_x, rot) if with_rot else (Xq, s_x)
+
+
+def w4a4_linear(Xq, s_x, Wq, s_w, b, bias=None, out_dtype=torch.float16,
+                Y=None, with_acc=False, stream=None):
+    """Packed codes -> Y [M, N] (out_dtype)[, acc int32 [M, N]]."""
+    M, Kh = Xq.shape
+    N = Wq.shape[0]
+    K = 2 * Kh
+    if Y is None:
+        Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
+    acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
+           if with_acc else None)
+    if bias is not None and bias.dtype != Y.dtype:
+        raise TypeError("bias must have the output dtype")
+    _check(clq_w4a4_linear(_ptr(Xq), _ptr(s_x), _ptr(Wq), _ptr(s_w),
+                           _ptr(bias), M, N, K, b, _dt(Y), _ptr(Y), _ptr(acc),
+                           _stream(stream)), "clq_w4a4_linear")
+    return (Y, acc) if with_acc else Y
+
+
+def fused_linear(X, perm, b, Wq, s_w, bias=None, Y=None, stream=None):
+    """X [M, K] -> Y [M, N] in X's dtype, rotate-quant fused into the GEMM."""
+    _row_major(X, "X")
+    M, K = X.shape
+    N = Wq.shape[0]
+    if Y is None:
+        Y = torch.empty((M, N), dtype=X.dtype, device=X.device)
+    _check(clq_fused_linear(_ptr(X), _dt(X), M, K, X.stride(0), _ptr(perm), b,
+                            _ptr(Wq), _ptr(s_w), _ptr(bias), N, _ptr(Y),
+                            _stream(stream)), "clq_fused_linear")
+    return Y
+
+
+def device_status(stream=None):
+    """Synchronize and read-and-clear the device status word."""
+    out = ctypes.c_int32(0)
+    _check(clq_get_device_status(_stream(stream), ctypes.addressof(out)),
+           "clq_get_device_status")
+    return out.value
+
+
+def selftest_bounded_wait(timeout_ns=1000000, stream=None):
+    _check(clq_selftest_bounded_wait(int(timeout_ns), _stream(stream)),
+           "clq_selftest_bounded_wait")
+
+
+class PreparedLinear:
+    """A quantized linear layer: the prepared-weight package (Wq, s_w, perm,
+    b, bias) of Sec. 3.3, where the swap vector is the only stored part of G.
+
+    ``state_dict()`` / ``from_state_dict()`` hold plain tensors for
+    ``torch.save``.  Calling the object runs the separate rotate-quant and
+    GEMM kernels (``fused=False``) or the fused kernel.
+    """
+
+    def __init__(self, Wq, s_w, perm, b, bias=None):
+        self.Wq, self.s_w, self.perm, self.b, self.bias = Wq, s_w, perm, b, bias
+
+    @classmethod
+    def from_weight(cls, W, perm, b, bias=None, clip=None):
+        perm = perm.to(W.device, torch.int32).contiguous()
+        Wq, s_w = prepare_weights(W.contiguous(), perm, b, clip)
+        return cls(Wq, s_w, perm, b, bias)
+
+    def state_dict(self):
+        d = dict(Wq=self.Wq, s_w=self.s_w, perm=self.perm,
+                 b=torch.tensor(self.b))
+        if self.bias is not None:
+            d["bias"] = self.bias
+        return d
+
+    @classmethod
+    def from_state_dict(cls, d):
+        return cls(d["Wq"], d["s_w"], d["perm"], int(d["b"]), d.get("bias"))
+
+    def __call__(self, X, fused=False, stream=None):
+        if fused:
+            return fused_linear(X, self.perm, self.b, self.Wq, self.s_w,
+                                self.bias, stream=stream)
+        Xq, s_x = rotate_quant_act(X, self.perm, self.b, stream=stream)
+        return w4a4_linear(Xq, s_x, self.Wq, self.s_w, self.b, self.bias,
+                           out_dtype=X.dtype, stream=stream)

@@ -1,0 +1,257 @@
+// C ABI of libclq (declared in include/clq.h): argument validation, the host
+// column-swap builder, the device status word and kernel launches.  Nothing
+// here allocates device memory or synchronizes, except
+// clq_get_device_status, which synchronizes by design.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+#include <numeric>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/clq.h"
+#include "clq_kernels.h"
+
+namespace {
+
+// Device status word: first device-side error since the last read.
+__device__ int32_t g_device_status;
+
+constexpr int kMaxDevices = 64;
+std::atomic<int32_t*> g_status_ptr[kMaxDevices];
+std::atomic<int> g_arch_ok[kMaxDevices];  // 0 unknown, 1 sm_103, -1 other
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool pow2_le256(int b) { return b >= 1 && b <= 256 && (b & (b - 1)) == 0; }
+
+int log2i(int b) {
+  int l = 0;
+  while ((1 << l) < b) ++l;
+  return l;
+}
+
+clq_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CLQ_OK : CLQ_ERR_CUDA; }
+
+// Current device's status-word address and architecture check.  The first
+// call on a device resolves the symbol address; later calls read the cache.
+clq_status device_setup(int32_t** status) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return CLQ_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return CLQ_ERR_UNSUPPORTED;
+  int arch = g_arch_ok[dev].load(std::memory_order_acquire);
+  if (arch == 0) {
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+      return CLQ_ERR_CUDA;
+    arch = (major == 10 && minor == 3) ? 1 : -1;
+    g_arch_ok[dev].store(arch, std::memory_order_release);
+  }
+  if (arch != 1) return CLQ_ERR_UNSUPPORTED;
+  int32_t* p = g_status_ptr[dev].load(std::memory_order_acquire);
+  if (p == nullptr) {
+    void* q = nullptr;
+    if (cudaGetSymbolAddress(&q, g_device_status) != cudaSuccess) return CLQ_ERR_CUDA;
+    p = static_cast<int32_t*>(q);
+    g_status_ptr[dev].store(p, std::memory_order_release);
+  }
+  *status = p;
+  return CLQ_OK;
+}
+
+clq_status check_k_b(int K, int b) {
+  if (!pow2_le256(b)) return CLQ_ERR_SHAPE;
+  if (K < 32 || K > 16384 || K % 32 != 0 || K % b != 0) return CLQ_ERR_SHAPE;
+  return CLQ_OK;
+}
+
+bool valid_dtype(int d) { return d == CLQ_F16 || d == CLQ_BF16; }
+
+clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ld,
+                               const int32_t* perm, int32_t b, const float* clip, uint8_t* Q,
+                               float* S, float* rot, void* stream) {
+  if (!valid_dtype(dtype) || M < 0) return CLQ_ERR_INVALID_ARG;
+  clq_status st = check_k_b(K, b);
+  if (st != CLQ_OK) return st;
+  if (ld < K) return CLQ_ERR_SHAPE;
+  if (ld % 8 != 0) return CLQ_ERR_ALIGN;
+  if (M == 0) return CLQ_OK;
+  if (X == nullptr || perm == nullptr || Q == nullptr || S == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(X, 16) || !aligned(Q, 16) || !aligned(perm, 4) || !aligned(S, 4) ||
+      (rot != nullptr && !aligned(rot, 16)) || (clip != nullptr && !aligned(clip, 4)))
+    return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  clq::RotateQuantArgs a{};
+  a.X = X;
+  a.M = M;
+  a.K = K;
+  a.ld = ld;
+  a.perm = perm;
+  a.clip = clip;
+  a.Q = Q;
+  a.S = S;
+  a.rot = rot;
+  a.status = status;
+  return from_cuda(
+      clq::launch_rotate_quant(a, dtype, log2i(b), static_cast<cudaStream_t>(stream)));
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* clq_status_string(clq_status s) {
+  switch (s) {
+    case CLQ_OK: return "CLQ_OK";
+    case CLQ_ERR_INVALID_ARG: return "CLQ_ERR_INVALID_ARG: null pointer, bad enum or negative size";
+    case CLQ_ERR_SHAPE: return "CLQ_ERR_SHAPE: shape rule violated (b, K, ld)";
+    case CLQ_ERR_ALIGN: return "CLQ_ERR_ALIGN: pointer or stride not aligned";
+    case CLQ_ERR_UNSUPPORTED: return "CLQ_ERR_UNSUPPORTED: no sm_103 device or feature";
+    case CLQ_ERR_CUDA: return "CLQ_ERR_CUDA: a CUDA runtime call failed";
+    case CLQ_ERR_TIMEOUT: return "CLQ_ERR_TIMEOUT: a bounded device-side wait ran out";
+    case CLQ_ERR_DEVICE_INDEX: return "CLQ_ERR_DEVICE_INDEX: perm index outside [0, K)";
+    default: return "unknown clq_status";
+  }
+}
+
+int32_t clq_version(void) { return 100; }
+
+clq_status clq_build_permutation(const float* host_scores, int32_t K, int32_t* host_perm) {
+  if (host_scores == nullptr || host_perm == nullptr || K < 1) return CLQ_ERR_INVALID_ARG;
+  for (int32_t k = 0; k < K; ++k)
+    if (std::isnan(host_scores[k])) return CLQ_ERR_INVALID_ARG;
+  std::vector<int32_t> order(K);
+  std::iota(order.begin(), order.end(), 0);
+  std::sort(order.begin(), order.end(), [&](int32_t a, int32_t c) {
+    if (host_scores[a] != host_scores[c]) return host_scores[a] > host_scores[c];
+    return a < c;
+  });
+  std::vector<char> high(K, 0);
+  for (int32_t i = 0; i < K / 2; ++i) high[order[i]] = 1;
+  int32_t pos = 0;
+  for (int32_t k = 0; k < K; ++k)
+    if (high[k]) host_perm[pos++] = k;
+  for (int32_t k = 0; k < K; ++k)
+    if (!high[k]) host_perm[pos++] = k;
+  return CLQ_OK;
+}
+
+clq_status clq_outlier_scores(const void* calib, clq_dtype dtype, int32_t B, int32_t T,
+                              int32_t K, float* scores, void* stream) {
+  if (!valid_dtype(dtype) || B < 1 || T < 1 || K < 1) return CLQ_ERR_INVALID_ARG;
+  if (calib == nullptr || scores == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(calib, 2) || !aligned(scores, 4)) return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  return from_cuda(
+      clq::launch_outlier_scores(calib, dtype, B, T, K, scores, static_cast<cudaStream_t>(stream)));
+}
+
+clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N, int32_t K, int32_t ldw,
+                               const int32_t* perm, int32_t b, const float* clip, uint8_t* Wq,
+                               float* s_w, float* w_rot_dbg, void* stream) {
+  return rotate_quant_common(W, dtype, N, K, ldw, perm, b, clip, Wq, s_w, w_rot_dbg, stream);
+}
+
+clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
+                                const int32_t* perm, int32_t b, uint8_t* Xq, float* s_x,
+                                float* x_rot_dbg, void* stream) {
+  return rotate_quant_common(X, dtype, M, K, ldx, perm, b, nullptr, Xq, s_x, x_rot_dbg, stream);
+}
+
+clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x, const uint8_t* Wq,
+                           const float* s_w, const void* bias, int32_t M, int32_t N, int32_t K,
+                           int32_t b, clq_dtype out_dtype, void* Y, int32_t* acc_dbg,
+                           void* stream) {
+  if (!valid_dtype(out_dtype) || M < 0 || N < 0) return CLQ_ERR_INVALID_ARG;
+  clq_status st = check_k_b(K, b);
+  if (st != CLQ_OK) return st;
+  if (M == 0 || N == 0) return CLQ_OK;
+  if (Xq == nullptr || s_x == nullptr || Wq == nullptr || s_w == nullptr || Y == nullptr)
+    return CLQ_ERR_INVALID_ARG;
+  if (!aligned(Xq, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_x, 4) ||
+      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)) ||
+      (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
+    return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  clq::GemmArgs g{};
+  g.s_x = s_x;
+  g.s_w = s_w;
+  g.bias = bias;
+  g.Y = Y;
+  g.acc_dbg = acc_dbg;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.inv_b = 1.0f / static_cast<float>(b);
+  g.status = status;
+  return from_cuda(clq::launch_w4a4_gemm(Xq, Wq, g, out_dtype, static_cast<cudaStream_t>(stream)));
+}
+
+clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
+                            const int32_t* perm, int32_t b, const uint8_t* Wq, const float* s_w,
+                            const void* bias, int32_t N, void* Y, void* stream) {
+  if (!valid_dtype(dtype) || M < 0 || N < 0) return CLQ_ERR_INVALID_ARG;
+  clq_status st = check_k_b(K, b);
+  if (st != CLQ_OK) return st;
+  if (ldx < K) return CLQ_ERR_SHAPE;
+  if (ldx % 8 != 0) return CLQ_ERR_ALIGN;
+  if (M == 0 || N == 0) return CLQ_OK;
+  if (X == nullptr || perm == nullptr || Wq == nullptr || s_w == nullptr || Y == nullptr)
+    return CLQ_ERR_INVALID_ARG;
+  if (!aligned(X, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(perm, 4) ||
+      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)))
+    return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  clq::FusedArgs f{};
+  f.X = X;
+  f.ld = ldx;
+  f.perm = perm;
+  f.logb = log2i(b);
+  f.s_w = s_w;
+  f.bias = bias;
+  f.Y = Y;
+  f.M = M;
+  f.N = N;
+  f.K = K;
+  f.inv_b = 1.0f / static_cast<float>(b);
+  f.status = status;
+  return from_cuda(clq::launch_fused_linear(Wq, f, dtype, static_cast<cudaStream_t>(stream)));
+}
+
+clq_status clq_get_device_status(void* stream, int32_t* out) {
+  if (out == nullptr) return CLQ_ERR_INVALID_ARG;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return CLQ_ERR_CUDA;
+  int32_t v = 0;
+  if (cudaMemcpyAsync(&v, status, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return CLQ_ERR_CUDA;
+  *out = v;
+  return CLQ_OK;
+}
+
+clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream) {
+  if (timeout_ns < 1000 || timeout_ns > 1000000000) return CLQ_ERR_INVALID_ARG;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  return from_cuda(clq::launch_wait_selftest(static_cast<uint64_t>(timeout_ns), status,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,69 @@
+// Host-side launch interface between the C ABI (clq_api.cu) and the kernels.
+#pragma once
+
+#include <algorithm>
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace clq {
+
+struct RotateQuantArgs {
+  const void* X;         // [M][ld] fp16 / bf16
+  int32_t M, K, ld;
+  const int32_t* perm;   // [K]
+  const float* clip;     // [M] or null (weights only)
+  uint8_t* Q;            // [M][K/2]
+  float* S;              // [M]
+  float* rot;            // [M][K] or null
+  int32_t rows_per_tile; // filled in by the launcher
+  int32_t* status;       // device status word
+};
+
+cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
+                                cudaStream_t st);
+void rotate_quant_config(int K, int* rows_per_tile, int* threads, size_t* smem);
+cudaError_t launch_outlier_scores(const void* calib, int dtype, int B, int T, int K,
+                                  float* scores, cudaStream_t st);
+
+struct GemmArgs {
+  const float* s_x;   // [M]
+  const float* s_w;   // [N]
+  const void* bias;   // [N] out dtype, or null
+  void* Y;            // [M][N] out dtype
+  int32_t* acc_dbg;   // [M][N] or null
+  int32_t M, N, K;
+  float inv_b;
+  int32_t* status;
+};
+
+// Packed INT4 operands are described by TMA maps built here from raw
+// pointers: A = Xq [M][K/2], B = Wq [N][K/2].
+cudaError_t launch_w4a4_gemm(const uint8_t* Xq, const uint8_t* Wq, const GemmArgs& g,
+                             int out_dtype, cudaStream_t st);
+
+struct FusedArgs {
+  const void* X;        // [M][ld]
+  int32_t ld;
+  const int32_t* perm;  // [K]
+  int32_t logb;
+  const float* s_w;
+  const void* bias;
+  void* Y;
+  int32_t M, N, K;
+  float inv_b;
+  int32_t* status;
+};
+
+cudaError_t launch_fused_linear(const uint8_t* Wq, const FusedArgs& f, int dtype,
+                                cudaStream_t st);
+
+// Bounded-wait self test (one CTA, one mbarrier nothing arrives at).
+cudaError_t launch_wait_selftest(uint64_t timeout_ns, int32_t* status, cudaStream_t st);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point.
+bool encode_tma_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
+                      uint64_t rows, uint32_t box_inner, uint32_t box_rows);
+
+}  // namespace clq

@@ -1,0 +1,117 @@
+"""CPU-only checks of the C ABI: the library loads, exports every symbol that
+include/clq.h declares, rejects bad arguments on the host before any launch,
+and its host column-swap builder matches the oracle's."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2509_24416_gb300 import build, clq
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return clq.load()
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "clq.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(clq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_matches_binding():
+    assert declared_functions() == sorted(clq.EXPORTS)
+
+
+def test_all_symbols_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    for code, name in clq.STATUS.items():
+        assert lib.clq_status_string(code).decode().startswith(name)
+    assert lib.clq_version() == 100
+
+
+P = 1 << 20  # a fake, 16-byte aligned "device" address; never dereferenced
+
+
+@pytest.mark.parametrize("args,code", [
+    # (X, dtype, M, K, ldx, perm, b, Xq, s_x, rot) -> expected status
+    ((P, 2, 4, 64, 64, P, 32, P, P, None), 1),      # bad dtype
+    ((P, 0, -1, 64, 64, P, 32, P, P, None), 1),     # negative M
+    ((P, 0, 4, 64, 64, P, 3, P, P, None), 2),       # b not a power of two
+    ((P, 0, 4, 64, 64, P, 512, P, P, None), 2),     # b > 256
+    ((P, 0, 4, 48, 48, P, 16, P, P, None), 2),      # K % 32
+    ((P, 0, 4, 1152, 1152, P, 256, P, P, None), 2), # K % b (1152 / 256)
+    ((P, 0, 4, 32768, 32768, P, 32, P, P, None), 2),  # K too large
+    ((P, 0, 4, 64, 32, P, 32, P, P, None), 2),      # ldx < K
+    ((P, 0, 4, 64, 68, P, 32, P, P, None), 3),      # ldx % 8
+    ((None, 0, 4, 64, 64, P, 32, P, P, None), 1),   # null X
+    ((P, 0, 4, 64, 64, None, 32, P, P, None), 1),   # null perm
+    ((P + 8, 0, 4, 64, 64, P, 32, P, P, None), 3),  # misaligned X
+    ((P, 0, 4, 64, 64, P, 32, P + 4, P, None), 3),  # misaligned Xq
+    ((P, 0, 0, 64, 64, None, 32, None, None, None), 0),  # empty: no-op
+])
+def test_rotate_quant_host_validation(lib, args, code):
+    assert clq.clq_rotate_quant_act(*args, None) == code
+
+
+@pytest.mark.parametrize("args,code", [
+    # (Xq, s_x, Wq, s_w, bias, M, N, K, b, out_dtype, Y, acc)
+    ((P, P, P, P, None, 4, 4, 64, 32, 3, P, None), 1),
+    ((P, P, P, P, None, 4, -2, 64, 32, 0, P, None), 1),
+    ((P, P, P, P, None, 4, 4, 96, 64, 0, P, None), 2),
+    ((P, P, P, P, None, 4, 4, 64, 32, 0, P + 2, None), 3),
+    ((P, P, P, P, P + 1, 4, 4, 64, 32, 0, P, None), 3),
+    ((None, P, P, P, None, 4, 4, 64, 32, 0, P, None), 1),
+    ((None, None, None, None, None, 0, 4, 64, 32, 0, None, None), 0),
+    ((None, None, None, None, None, 4, 0, 64, 32, 0, None, None), 0),
+])
+def test_w4a4_host_validation(lib, args, code):
+    assert clq.clq_w4a4_linear(*args, None) == code
+
+
+def test_fused_and_prepare_host_validation(lib):
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 7, P, P, None, 4, P,
+                                None) == 2
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, P, None, 0, P,
+                                None) == 0
+    assert clq.clq_prepare_weights(P, 0, 4, 64, 64, P, 32, P + 2, P, P, None,
+                                   None) == 3
+    assert clq.clq_outlier_scores(P, 0, 0, 4, 4, P, None) == 1
+    assert clq.clq_selftest_bounded_wait(10, None) == 1
+    assert clq.clq_get_device_status(None, None) == 1
+
+
+@pytest.mark.parametrize("K,seed", [(1, 0), (2, 1), (7, 2), (64, 3),
+                                    (1152, 4), (4608, 5)])
+def test_build_permutation_matches_oracle(lib, K, seed):
+    rng = np.random.default_rng(seed)
+    scores = rng.uniform(0, 1, K).astype(np.float32)
+    scores[rng.choice(K, max(1, K // 100), replace=False)] *= 40
+    scores[: K // 3] = np.round(scores[: K // 3] * 4) / 4  # many exact ties
+    got = clq.build_permutation(torch.from_numpy(scores)).numpy()
+    assert np.array_equal(got, oracle.build_permutation(scores))
+
+
+def test_build_permutation_rejects_nan(lib):
+    s = torch.tensor([1.0, float("nan"), 2.0])
+    perm = torch.empty(3, dtype=torch.int32)
+    assert clq.clq_build_permutation(s.data_ptr(), 3, perm.data_ptr()) == 1
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    monkeypatch.setattr(clq, "_lib", None)
+    monkeypatch.setattr(clq, "LIB_PATH", str(tmp_path / "nope.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        clq.load()

@@ -1,0 +1,331 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle, element
+by element on the same seeded inputs.  Tolerances: tests/parity_utils.py."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2509_24416_gb300 import clq, synth
+from parity_utils import (check_codes, check_output_elementwise,
+                          check_output_frobenius, check_rot, check_scales)
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda:0")
+TD = {"f16": torch.float16, "bf16": torch.bfloat16}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    clq.load()
+    yield
+    assert clq.device_status() == 0
+
+
+def _inputs(M, K, dtype, seed, scale=3.0, outliers=4):
+    rng = np.random.default_rng(seed)
+    x = rng.standard_normal((M, K)).astype(np.float32) * scale
+    if outliers:
+        ch = rng.choice(K, min(outliers, K), replace=False)
+        x[:, ch] *= 40
+    t = torch.from_numpy(x).to(TD[dtype])
+    return t, t.float().numpy()
+
+
+def _perm(K, kind, seed=0):
+    if kind == "identity":
+        return np.arange(K, dtype=np.int32)
+    if kind == "reversed":
+        return np.arange(K - 1, -1, -1, dtype=np.int32)
+    return np.random.default_rng(seed).permutation(K).astype(np.int32)
+
+
+def _rq_gpu(x, perm, b):
+    Xq, s_x, rot = clq.rotate_quant_act(x.to(DEV), torch.from_numpy(perm).to(DEV),
+                                        b, with_rot=True)
+    torch.cuda.synchronize()
+    return Xq.cpu().numpy(), s_x.cpu().numpy(), rot.cpu().numpy()
+
+
+def _check_rq(x_t, x32, perm, b):
+    gq, gs, grot = _rq_gpu(x_t, perm, b)
+    oq, os_, orot, oc = oracle.rotate_quant_act(x32, perm, b)
+    check_rot(grot, orot)
+    check_scales(gs, os_)
+    check_codes(oracle.unpack_int4(gq), oc, orot, os_)
+    return gq, gs
+
+
+# ------------------------------------------------------------ rotate-quant --
+@pytest.mark.parametrize("b", [1, 2, 8, 32, 64, 128, 256])
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_rotate_quant_block_sizes(b, dtype):
+    K = 512
+    x_t, x32 = _inputs(37, K, dtype, seed=b)
+    _check_rq(x_t, x32, _perm(K, "random", b), b)
+
+
+@pytest.mark.parametrize("M,K", [(1, 32), (3, 64), (17, 96), (64, 1152),
+                                 (300, 1152), (33, 4608), (5, 12288),
+                                 (9, 3072), (2, 16384)])
+def test_rotate_quant_shapes(M, K):
+    b = 32 if K % 64 else 64
+    x_t, x32 = _inputs(M, K, "f16", seed=M + K)
+    _check_rq(x_t, x32, _perm(K, "random", K), b)
+
+
+@pytest.mark.parametrize("kind", ["identity", "reversed", "random"])
+def test_rotate_quant_permutations(kind):
+    K = 1152
+    x_t, x32 = _inputs(40, K, "f16", seed=7)
+    _check_rq(x_t, x32, _perm(K, kind, 3), 64)
+
+
+def test_rotate_quant_strided_rows():
+    M, K, ld = 20, 256, 264
+    big = torch.randn(M, ld, generator=torch.Generator().manual_seed(1)).half()
+    view = big[:, :K]
+    perm = _perm(K, "random", 5)
+    g = clq.rotate_quant_act(view.to(DEV), torch.from_numpy(perm).to(DEV), 64,
+                             with_rot=True)
+    # the device view keeps the row stride of the padded buffer
+    dev_big = big.to(DEV)
+    g2 = clq.rotate_quant_act(dev_big[:, :K], torch.from_numpy(perm).to(DEV),
+                              64, with_rot=True)
+    torch.cuda.synchronize()
+    assert dev_big[:, :K].stride(0) == ld
+    oq, os_, orot, oc = oracle.rotate_quant_act(view.float().numpy(), perm, 64)
+    for Xq, s, rot in (g, g2):
+        check_rot(rot.cpu().numpy(), orot)
+        check_codes(oracle.unpack_int4(Xq.cpu().numpy()), oc, orot, os_)
+
+
+def test_rotate_quant_zero_rows_and_spikes():
+    K, b = 256, 64
+    x = np.zeros((6, K), np.float32)
+    x[1, 5] = 3.0                        # single spike
+    x[2, :] = 0.0                        # zero row
+    x[3, ::b] = -2.0                     # one spike per block
+    x[4, 7] = 65504.0                    # fp16 maximum
+    x[5, :] = 1e-4
+    x_t = torch.from_numpy(x).half()
+    perm = _perm(K, "random", 9)
+    gq, gs, grot = _rq_gpu(x_t, perm, b)
+    oq, os_, orot, oc = oracle.rotate_quant_act(x_t.float().numpy(), perm, b)
+    assert gs[0] == 0 and gs[2] == 0 and not gq[0].any() and not gq[2].any()
+    check_rot(grot, orot)
+    check_scales(gs, os_)
+    assert np.array_equal(gq, oq)
+
+
+def test_rotate_quant_exact_ties_half_even():
+    # rotated rows with s = 1 exactly and entries at k + 1/2: X = X~ H / b.
+    b, K = 16, 64
+    rng = np.random.default_rng(3)
+    rot = rng.integers(-6, 7, (8, K)).astype(np.float64) + 0.5
+    rot[:, ::b] = 7.0                     # row abs-max 7 -> s = 1
+    H = oracle.hadamard_sylvester(b).astype(np.float64)
+    xp = (rot.reshape(8, K // b, b) @ H / b).reshape(8, K)
+    perm = _perm(K, "random", 4)
+    x = np.empty_like(xp)
+    x[:, perm] = xp                       # X[:, perm[j]] = X_p[:, j]
+    x_t = torch.from_numpy(x.astype(np.float32)).half()
+    assert np.array_equal(x_t.float().numpy(), x.astype(np.float32))
+    gq, gs, grot = _rq_gpu(x_t, perm, b)
+    oq, os_, orot, oc = oracle.rotate_quant_act(x_t.float().numpy(), perm, b)
+    assert np.array_equal(orot, rot.astype(np.float32))
+    assert np.all(os_ == 1.0) and np.array_equal(gs, os_)
+    assert np.array_equal(grot, orot)
+    assert np.array_equal(gq, oq)         # ties to even, bit for bit
+
+
+def test_rotate_quant_bad_perm_index_is_reported():
+    K = 64
+    x_t, _ = _inputs(4, K, "f16", seed=1)
+    perm = _perm(K, "identity")
+    perm[5] = K + 100
+    clq.rotate_quant_act(x_t.to(DEV), torch.from_numpy(perm).to(DEV), 32)
+    assert clq.device_status() == 7       # CLQ_ERR_DEVICE_INDEX
+    assert clq.device_status() == 0       # read-and-clear
+
+
+def test_prepare_weights_with_clip():
+    N, K, b = 70, 1152, 64
+    rng = np.random.default_rng(2)
+    w = (rng.standard_normal((N, K)) * 0.02).astype(np.float32)
+    w_t = torch.from_numpy(w).half()
+    perm = _perm(K, "random", 1)
+    _, _, orot0, _ = oracle.prepare_weights(w_t.float().numpy(), perm, b)
+    clip = (np.max(np.abs(orot0), axis=1) * 0.6).astype(np.float32)
+    clip[::3] = 1e9                        # no clipping on every third row
+    Wq, s_w, rot = clq.prepare_weights(w_t.to(DEV), torch.from_numpy(perm).to(DEV),
+                                       b, clip=torch.from_numpy(clip).to(DEV),
+                                       with_rot=True)
+    torch.cuda.synchronize()
+    oq, os_, orot, oc = oracle.prepare_weights(w_t.float().numpy(), perm, b, clip)
+    check_rot(rot.cpu().numpy(), orot)
+    check_scales(s_w.cpu().numpy(), os_)
+    check_codes(oracle.unpack_int4(Wq.cpu().numpy()), oc, orot, os_)
+
+
+# -------------------------------------------------------------------- GEMM --
+def _gemm_case(M, N, K, b, dtype, seed, bias=True):
+    x_t, x32 = _inputs(M, K, dtype, seed)
+    rng = np.random.default_rng(seed + 1)
+    w_t = torch.from_numpy((rng.standard_normal((N, K)) * 0.02).astype(np.float32)).to(TD[dtype])
+    bias_t = (torch.from_numpy((rng.standard_normal(N) * 0.01).astype(np.float32)).to(TD[dtype])
+              if bias else None)
+    perm = _perm(K, "random", seed)
+    oXq, os_x, _, _ = oracle.rotate_quant_act(x32, perm, b)
+    oWq, os_w, _, _ = oracle.prepare_weights(w_t.float().numpy(), perm, b)
+    b32 = None if bias_t is None else bias_t.float().numpy()
+    y64, acc = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, b32)
+    Y, gacc = clq.w4a4_linear(torch.from_numpy(oXq).to(DEV), torch.from_numpy(os_x).to(DEV),
+                              torch.from_numpy(oWq).to(DEV), torch.from_numpy(os_w).to(DEV),
+                              b, None if bias_t is None else bias_t.to(DEV),
+                              out_dtype=TD[dtype], with_acc=True)
+    torch.cuda.synchronize()
+    assert np.array_equal(gacc.cpu().numpy(), acc)
+    y = Y.float().cpu().numpy()
+    check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
+    check_output_frobenius(y, y64)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 1, 32), (3, 17, 64), (17, 64, 128),
+                                   (64, 256, 1152), (300, 600, 1152),
+                                   (129, 257, 96), (250, 1000, 160),
+                                   (256, 512, 4608)])
+def test_gemm_acc_exact_and_output(M, N, K):
+    _gemm_case(M, N, K, 32, "f16", seed=M + N + K)
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_gemm_dtypes_and_no_bias(dtype):
+    _gemm_case(200, 300, 1152, 64, dtype, seed=5, bias=False)
+    _gemm_case(130, 260, 1152, 64, dtype, seed=6, bias=True)
+
+
+@pytest.mark.parametrize("K", [1152, 4608, 12288, 16384])
+def test_gemm_carrier_exact_at_extremes(K):
+    """All codes +-7: |acc| reaches 49 K (602112 at K = 12288); mixed-sign
+    rows make large partial sums cancel.  fp32 accumulation of the E4M3
+    carrier must stay exact."""
+    M, N = 136, 264
+    rng = np.random.default_rng(K)
+    qx = np.where(rng.random((M, K)) < 0.5, -7, 7).astype(np.int8)
+    qw = np.where(rng.random((N, K)) < 0.5, -7, 7).astype(np.int8)
+    qx[:8] = 7
+    qw[:8] = 7
+    qw[8:16] = -7
+    qx[8:16, : K // 2] = 7
+    qx[8:16, K // 2:] = -7                 # partial sums rise to 49 K/2, end at 0
+    Xq = oracle.pack_int4(qx)
+    Wq = oracle.pack_int4(qw)
+    acc = oracle.int_gemm(qx, qw)
+    ones_x = torch.ones(M, dtype=torch.float32, device=DEV)
+    ones_w = torch.ones(N, dtype=torch.float32, device=DEV)
+    _, gacc = clq.w4a4_linear(torch.from_numpy(Xq).to(DEV), ones_x,
+                              torch.from_numpy(Wq).to(DEV), ones_w, 32,
+                              out_dtype=torch.bfloat16, with_acc=True)
+    torch.cuda.synchronize()
+    assert np.array_equal(gacc.cpu().numpy(), acc)
+
+
+def test_gemm_random_codes_all_values():
+    M, N, K = 160, 320, 2048
+    rng = np.random.default_rng(11)
+    qx = rng.integers(-7, 8, (M, K)).astype(np.int8)
+    qw = rng.integers(-7, 8, (N, K)).astype(np.int8)
+    acc = oracle.int_gemm(qx, qw)
+    s = torch.ones(max(M, N), dtype=torch.float32, device=DEV)
+    _, gacc = clq.w4a4_linear(torch.from_numpy(oracle.pack_int4(qx)).to(DEV), s[:M],
+                              torch.from_numpy(oracle.pack_int4(qw)).to(DEV), s[:N], 32,
+                              with_acc=True)
+    torch.cuda.synchronize()
+    assert np.array_equal(gacc.cpu().numpy(), acc)
+
+
+# ------------------------------------------------------ end-to-end layers --
+def _layer_e2e(cfg, li, M, rows=None):
+    d = synth.layer_inputs(cfg, li, M=M)
+    b = d["b"]
+    calib = torch.from_numpy(d["calib"]).to(TD[d["dtype"]]).to(DEV)
+    g_scores = clq.outlier_scores(calib)
+    o_scores = oracle.outlier_scores(d["calib"])
+    assert np.array_equal(g_scores.cpu().numpy(), o_scores)
+    perm = clq.build_permutation(g_scores)
+    assert np.array_equal(perm.numpy(), oracle.build_permutation(o_scores))
+    permd = perm.to(DEV)
+    layer = clq.PreparedLinear.from_weight(d["W"].to(DEV), permd, b, bias=d["bias"].to(DEV))
+    X = d["X"].to(DEV)
+    Xq, s_x, rot = clq.rotate_quant_act(X, permd, b, with_rot=True)
+    Y = clq.w4a4_linear(Xq, s_x, layer.Wq, layer.s_w, b, layer.bias, out_dtype=X.dtype)
+    torch.cuda.synchronize()
+    rows = np.arange(M) if rows is None else rows
+    p = perm.numpy()
+    oWq, os_w, orot_w, owc = oracle.prepare_weights(d["W32"], p, b)
+    check_scales(layer.s_w.cpu().numpy(), os_w)
+    check_codes(oracle.unpack_int4(layer.Wq.cpu().numpy()), owc, orot_w, os_w)
+    x32 = d["X32"][rows]
+    oXq, os_x, orot, oc = oracle.rotate_quant_act(x32, p, b)
+    check_rot(rot.cpu().numpy()[rows], orot)
+    check_scales(s_x.cpu().numpy()[rows], os_x)
+    check_codes(oracle.unpack_int4(Xq.cpu().numpy()[rows]), oc, orot, os_x)
+    y64, _ = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, d["bias32"])
+    check_output_frobenius(Y.float().cpu().numpy()[rows], y64)
+    return d, layer, Y
+
+
+def test_single_layer_full():
+    _layer_e2e(synth.WORKLOADS["single_1152"], 0, 256)
+
+
+@pytest.mark.parametrize("name", ["pixart_1024", "video_16x32x32", "mmdit_4608"])
+def test_layer_sets_full_size_sampled_rows(name):
+    cfg = synth.WORKLOADS[name]
+    rng = np.random.default_rng(0)
+    for li in range(len(cfg["layers"])):
+        M = cfg["M"]
+        rows = np.sort(np.concatenate([rng.choice(M, 40, replace=False),
+                                       [0, M - 1]]))
+        _layer_e2e(cfg, li, M, rows)
+
+
+def test_video_token_permutation_equivariance():
+    cfg = synth.WORKLOADS["video_16x32x32"]
+    d, layer, Y = _layer_e2e(cfg, 0, cfg["M"], rows=np.arange(0, cfg["M"], 997))
+    X2 = synth.temporal_reorder(d["X"]).to(DEV)
+    Y2 = layer(X2)
+    torch.cuda.synchronize()
+    Y_re = synth.temporal_reorder(Y.cpu())
+    assert torch.equal(Y2.cpu(), Y_re)
+
+
+def test_prepared_linear_state_roundtrip(tmp_path):
+    cfg = synth.WORKLOADS["single_1152"]
+    d = synth.layer_inputs(cfg, 0, M=64)
+    perm = torch.from_numpy(oracle.build_permutation(oracle.outlier_scores(d["calib"])))
+    layer = clq.PreparedLinear.from_weight(d["W"].to(DEV), perm, 64, bias=d["bias"].to(DEV))
+    torch.save(layer.state_dict(), tmp_path / "l.pt")
+    layer2 = clq.PreparedLinear.from_state_dict(torch.load(tmp_path / "l.pt"))
+    X = d["X"].to(DEV)
+    assert torch.equal(layer(X), layer2(X))
+
+
+# ------------------------------------------------------- failure handling --
+def test_bounded_wait_selftest_reports_timeout():
+    clq.selftest_bounded_wait(2_000_000)   # 2 ms
+    assert clq.device_status() == 6        # CLQ_ERR_TIMEOUT
+    # the context stays usable
+    x_t, x32 = _inputs(8, 64, "f16", seed=3)
+    _check_rq(x_t, x32, _perm(64, "random", 1), 32)
+    assert clq.device_status() == 0
+
+
+def test_empty_inputs_are_noops():
+    z = torch.empty((0, 64), dtype=torch.float16, device=DEV)
+    perm = torch.arange(64, dtype=torch.int32, device=DEV)
+    Xq, s_x = clq.rotate_quant_act(z, perm, 32)
+    assert Xq.shape == (0, 32) and s_x.shape == (0,)
+    Wq = torch.zeros((0, 32), dtype=torch.uint8, device=DEV)
+    Y = clq.w4a4_linear(Xq, s_x, Wq, torch.empty(0, device=DEV), 32)
+    assert Y.shape == (0, 0)
