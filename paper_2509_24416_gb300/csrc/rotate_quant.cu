@@ -167,9 +167,12 @@ __global__ void __launch_bounds__(512) rotate_quant_kernel(RotateQuantArgs a) {
 #pragma unroll
     for (int e = 0; e < 32; ++e) m = fmaxf(m, fabsf(v[e]));
     {
-      const unsigned grp = __match_any_sync(0xffffffffu, r_local);
+      // Padding lanes (tid >= items) only keep the shuffles convergent; their
+      // values are not data of any row and must not reach a row maximum.
+      const int key = active ? r_local : -1;
+      const unsigned grp = __match_any_sync(0xffffffffu, key);
       const unsigned mx = __reduce_max_sync(grp, __float_as_uint(m));
-      if (lane == __ffs(grp) - 1) atomicMax(&amax_s[par * R + r_local], mx);
+      if (active && lane == __ffs(grp) - 1) atomicMax(&amax_s[par * R + r_local], mx);
     }
     __syncthreads();
 
@@ -261,8 +264,9 @@ cudaError_t launch_rq_dtype(const RotateQuantArgs& a, int logb, int threads, siz
 
 }  // namespace
 
-// Rows per tile: as many as keep the CTA at <= 512 threads, preferring a
-// thread count that fills whole warps.
+// Rows per tile: the CTA gets one thread per 32-element segment of each of
+// its rows.  Prefer thread counts that fill whole warps (padding lanes do no
+// useful work) and lie in [192, 384], which keeps two to three CTAs per SM.
 void rotate_quant_config(int K, int* rows_per_tile, int* threads, size_t* smem) {
   const int segs = K >> 5;
   int best_r = 1;
@@ -271,7 +275,9 @@ void rotate_quant_config(int K, int* rows_per_tile, int* threads, size_t* smem) 
     const int t = r * segs;
     const int t32 = (t + 31) & ~31;
     const double fill = static_cast<double>(t) / t32;
-    const double score = fill * 4.0 + std::min(t32, 384) / 384.0;
+    const double size_term =
+        t32 < 192 ? t32 / 384.0 : (t32 <= 384 ? 1.0 + t32 / 4096.0 : 0.5);
+    const double score = fill * 4.0 + size_term;
     if (score > best_score + 1e-9) {
       best_score = score;
       best_r = r;

@@ -73,6 +73,16 @@ def test_rotate_quant_shapes(M, K):
     _check_rq(x_t, x32, _perm(K, "random", K), b)
 
 
+@pytest.mark.parametrize("K,b", [(1184, 32), (1216, 64), (1280, 128),
+                                 (2112, 64)])
+def test_rotate_quant_padding_lanes_do_not_leak(K, b):
+    """K / 32 segments per row that do not fill whole warps: the CTA has
+    padding lanes, which must not touch any row's abs-max.  Rows without
+    outliers make any leak visible in the scales."""
+    x_t, x32 = _inputs(45, K, "f16", seed=K, scale=0.02, outliers=0)
+    _check_rq(x_t, x32, _perm(K, "random", K), b)
+
+
 @pytest.mark.parametrize("kind", ["identity", "reversed", "random"])
 def test_rotate_quant_permutations(kind):
     K = 1152
