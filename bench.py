@@ -46,6 +46,12 @@ def parse():
     p.add_argument("--fused", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--layer", default=None,
+                   help="time only this layer of the workload (profiling)")
+    p.add_argument("--tokens", type=int, default=None,
+                   help="override the token count M (profiling)")
+    p.add_argument("--settle", type=float, default=1.0,
+                   help="seconds of untimed steps before timing")
     return p.parse_args()
 
 
@@ -226,7 +232,8 @@ def reference_arm(args):
 
 
 def config_dict(cfg, args):
-    return {"workload": args.workload, "tokens": cfg["M"], "b": cfg["b"],
+    return {"workload": args.workload + ("" if args.layer is None else ":" + args.layer),
+            "tokens": cfg["M"], "b": cfg["b"],
             "layers": ["%s %dx%d" % (n, K, N) for (n, K, N) in cfg["layers"]],
             "io_dtype": cfg["dtype"], "path": "fused" if args.fused else "separate",
             "l2": "inputs rotated over sets totalling > 2x L2 (129 MB)"}
@@ -250,15 +257,23 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     clq.load()
-    cfg = synth.WORKLOADS[args.workload]
+    cfg = dict(synth.WORKLOADS[args.workload])
+    if args.layer is not None:
+        cfg["layers"] = tuple(l for l in cfg["layers"] if l[0] == args.layer)
+        if not cfg["layers"]:
+            raise SystemExit("no layer %r in %s" % (args.layer, args.workload))
+    if args.tokens is not None:
+        cfg["M"] = int(args.tokens)
     td = {"f16": torch.float16, "bf16": torch.bfloat16}[cfg["dtype"]]
     b = cfg["b"]
     M = cfg["M"]
 
     # ---- offline: calibration, swap vectors, prepared weights (untimed) ----
     layers, xs_host = [], []
-    for li in range(len(cfg["layers"])):
-        d = synth.layer_inputs(cfg, li)
+    all_names = [l[0] for l in synth.WORKLOADS[args.workload]["layers"]]
+    for lname, _, _ in cfg["layers"]:
+        li = all_names.index(lname)
+        d = synth.layer_inputs(dict(synth.WORKLOADS[args.workload], M=cfg["M"]), li)
         calib = torch.from_numpy(d["calib"]).to(td).to(dev)
         perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
         lay = clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b,
@@ -271,6 +286,7 @@ def main():
     xq = [torch.empty((M, K // 2), dtype=torch.uint8, device=dev) for (_, K, _, _) in layers]
     sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in layers]
     ys = [torch.empty((M, N), dtype=td, device=dev) for (_, _, N, _) in layers]
+    wss = [clq.fused_workspace(M, K, dev) for (_, K, _, _) in layers]
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
     nlay = len(layers)
@@ -282,9 +298,10 @@ def main():
                 ev[4 * i].record(stream)
             if args.fused:
                 st = clq.clq_fused_linear(xs[i].data_ptr(), clq._dt(xs[i]), M, K, K,
-                                          lay.perm.data_ptr(), b, lay.Wq.data_ptr(),
-                                          lay.s_w.data_ptr(), lay.bias.data_ptr(), N,
-                                          ys[i].data_ptr(), sp)
+                                          lay.perm.data_ptr(), b, lay.We.data_ptr(),
+                                          clq.CLQ_W_E4M3, lay.s_w.data_ptr(),
+                                          lay.bias.data_ptr(), N, ys[i].data_ptr(),
+                                          wss[i].data_ptr(), wss[i].numel(), sp)
                 if st:
                     raise clq.ClqError(st, "clq_fused_linear")
                 if ev is not None:
@@ -300,9 +317,9 @@ def main():
                     ev[4 * i + 1].record(stream)
                     ev[4 * i + 2].record(stream)
                 st = clq.clq_w4a4_linear(xq[i].data_ptr(), sx[i].data_ptr(),
-                                         lay.Wq.data_ptr(), lay.s_w.data_ptr(),
-                                         lay.bias.data_ptr(), M, N, K, b, clq._dt(ys[i]),
-                                         ys[i].data_ptr(), None, sp)
+                                         lay.We.data_ptr(), clq.CLQ_W_E4M3,
+                                         lay.s_w.data_ptr(), lay.bias.data_ptr(), M, N, K, b,
+                                         clq._dt(ys[i]), ys[i].data_ptr(), None, sp)
                 if st:
                     raise clq.ClqError(st, "clq_w4a4_linear")
             if ev is not None:
@@ -314,7 +331,7 @@ def main():
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     n_settle = 0
-    while time.perf_counter() - t0 < 1.0:
+    while time.perf_counter() - t0 < args.settle:
         step(n_settle)
         n_settle += 1
         if n_settle % 50 == 0:
@@ -409,7 +426,7 @@ def main():
         def e2e_step():
             for i, (_, K, N, lay) in enumerate(layers):
                 xd[i].copy_(xh[i], non_blocking=True)
-                Y = lay(xd[i], fused=args.fused)
+                Y = lay(xd[i], fused=args.fused, workspace=wss[i])
                 yh[i].copy_(Y, non_blocking=True)
 
         for _ in range(2):

@@ -29,8 +29,9 @@
  *    in its high nibble, 4-bit two's complement.  A packed row of K codes is
  *    K/2 bytes and rows are contiguous (stride K/2).
  *  - Shape rules: 1 <= b <= 256 and b a power of two; K % 32 == 0,
- *    K % b == 0, 32 <= K <= 32768; M, N >= 0 (0 is an empty no-op);
- *    ld* >= K and ld* % 8 == 0; every pointer 16-byte aligned.
+ *    K % b == 0, 32 <= K <= 16384; M, N >= 0 (0 is an empty no-op);
+ *    ld* >= K and ld* % 8 == 0.  Matrices and code arrays are 16-byte
+ *    aligned; vectors (perm, scales, clip) 4-byte and bias 2-byte aligned.
  *  - Device-side faults the host cannot see (an index in `perm` outside
  *    [0, K), a pipeline wait that exceeds its time limit) are recorded in a
  *    device status word read by clq_get_device_status; the kernel skips the
@@ -41,6 +42,7 @@
 #ifndef CLQ_H
 #define CLQ_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -60,6 +62,12 @@ typedef int32_t clq_status;
 typedef int32_t clq_dtype;
 #define CLQ_F16 0
 #define CLQ_BF16 1
+
+/* Layout of the prepared weight codes handed to the GEMM calls. */
+typedef int32_t clq_wformat;
+#define CLQ_W_INT4_PACKED 0 /* [N][K/2] bytes, two codes per byte (storage)   */
+#define CLQ_W_E4M3 1        /* [N][K] bytes, each code as its exact E4M3      */
+                            /* value (execution layout, clq_expand_weights)   */
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char* clq_status_string(clq_status status);
@@ -117,29 +125,57 @@ clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M,
                                 float* x_rot_dbg, void* stream);
 
 /*
- * Packed INT4 x INT4 product with the dequant + bias epilogue:
- * Y[i][n] = out_dtype(acc[i][n] * s_x[i] * s_w[n] / b + bias[n]).
- * Xq: device uint8 [M][K/2]; s_x: device fp32 [M]; Wq: device uint8
- * [N][K/2]; s_w: device fp32 [N]; bias: device [N] of `out_dtype` or NULL;
- * Y: device [M][N] of `out_dtype`.  acc_dbg: device int32 [M][N] or NULL;
- * when given it receives the exact integer accumulators.
+ * Execution layout of prepared weights: every packed INT4 code of Wq
+ * [N][K/2] becomes one byte of We [N][K] holding the code's exact E4M3
+ * encoding (every integer in [-7, 7] is an E4M3 value).  The codes are
+ * unchanged; only the container widens to 8 bits, so the GEMM can load
+ * weight tiles with TMA straight into the tensor-core operand layout instead
+ * of expanding nibbles in every CTA.  Offline, once per layer.  Wq: device
+ * [N][K/2]; We: device [N][K].  Requires N >= 0, K % 32 == 0, K <= 16384.
  */
-clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x,
-                           const uint8_t* Wq, const float* s_w,
-                           const void* bias, int32_t M, int32_t N, int32_t K,
-                           int32_t b, clq_dtype out_dtype, void* Y,
-                           int32_t* acc_dbg, void* stream);
+clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K,
+                              uint8_t* We, void* stream);
 
 /*
- * The whole layer in one kernel: clq_rotate_quant_act fused into the GEMM
- * prologue, so the activation codes never reach HBM.  Same arithmetic and
- * results as the two separate calls.  X: device [M][ldx] of `dtype`; Y:
- * device [M][N] of `dtype`; bias: device [N] of `dtype` or NULL.
+ * INT4 x INT4 product with the dequant + bias epilogue:
+ * Y[i][n] = out_dtype(acc[i][n] * s_x[i] * s_w[n] / b + bias[n]).
+ * Xq: device uint8 [M][K/2] packed activation codes; s_x: device fp32 [M];
+ * W: device weight codes in layout `w_format` (CLQ_W_INT4_PACKED: [N][K/2],
+ * CLQ_W_E4M3: [N][K]); s_w: device fp32 [N]; bias: device [N] of
+ * `out_dtype` or NULL; Y: device [M][N] of `out_dtype`.  acc_dbg: device
+ * int32 [M][N] or NULL; when given it receives the exact integer
+ * accumulators.  Both weight layouts give identical results.
+ */
+clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x,
+                           const uint8_t* W, clq_wformat w_format,
+                           const float* s_w, const void* bias, int32_t M,
+                           int32_t N, int32_t K, int32_t b,
+                           clq_dtype out_dtype, void* Y, int32_t* acc_dbg,
+                           void* stream);
+
+/*
+ * Bytes of device workspace clq_fused_linear needs for M tokens of K
+ * channels (activation codes, scales and per-tile readiness counters).
+ */
+size_t clq_fused_linear_workspace_size(int32_t M, int32_t K);
+
+/*
+ * The whole layer in one persistent kernel: every CTA first rotates and
+ * quantizes its share of token rows into `workspace` (which stays in L2 for
+ * the layer sizes of the paper's models), then runs GEMM tiles, each of which
+ * starts as soon as the rows of its token block are published.  Same
+ * arithmetic and results as clq_rotate_quant_act followed by
+ * clq_w4a4_linear.  X: device [M][ldx] of `dtype`; Y: device [M][N] of
+ * `dtype`; bias: device [N] of `dtype` or NULL; W / w_format as for
+ * clq_w4a4_linear; workspace: device, 256-byte aligned, at least
+ * clq_fused_linear_workspace_size(M, K) bytes, owned by the caller and
+ * overwritten by the call.
  */
 clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M,
                             int32_t K, int32_t ldx, const int32_t* perm,
-                            int32_t b, const uint8_t* Wq, const float* s_w,
-                            const void* bias, int32_t N, void* Y,
+                            int32_t b, const uint8_t* W, clq_wformat w_format,
+                            const float* s_w, const void* bias, int32_t N,
+                            void* Y, void* workspace, size_t workspace_bytes,
                             void* stream);
 
 /*

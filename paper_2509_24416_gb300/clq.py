@@ -20,17 +20,20 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libclq.so")
 
 CLQ_F16, CLQ_BF16 = 0, 1
+CLQ_W_INT4_PACKED, CLQ_W_E4M3 = 0, 1
 STATUS = {0: "CLQ_OK", 1: "CLQ_ERR_INVALID_ARG", 2: "CLQ_ERR_SHAPE",
           3: "CLQ_ERR_ALIGN", 4: "CLQ_ERR_UNSUPPORTED", 5: "CLQ_ERR_CUDA",
           6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX"}
 EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_build_permutation", "clq_prepare_weights",
-           "clq_rotate_quant_act", "clq_w4a4_linear", "clq_fused_linear",
+           "clq_rotate_quant_act", "clq_expand_weights", "clq_w4a4_linear",
+           "clq_fused_linear_workspace_size", "clq_fused_linear",
            "clq_get_device_status", "clq_selftest_bounded_wait")
 
 _lib = None
 _P = ctypes.c_void_p
 _I = ctypes.c_int32
+_Z = ctypes.c_size_t
 _SIGS = {
     "clq_status_string": (ctypes.c_char_p, [_I]),
     "clq_version": (_I, []),
@@ -40,10 +43,12 @@ _SIGS = {
                                  _P]),
     "clq_rotate_quant_act": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P,
                                   _P]),
-    "clq_w4a4_linear": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P,
-                             _P]),
-    "clq_fused_linear": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _I, _P,
-                              _P]),
+    "clq_expand_weights": (_I, [_P, _I, _I, _P, _P]),
+    "clq_w4a4_linear": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P,
+                             _P, _P]),
+    "clq_fused_linear_workspace_size": (_Z, [_I, _I]),
+    "clq_fused_linear": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I, _P, _P, _I,
+                              _P, _P, _Z, _P]),
     "clq_get_device_status": (_I, [_P, _P]),
     "clq_selftest_bounded_wait": (_I, [ctypes.c_int64, _P]),
 }
@@ -100,16 +105,25 @@ def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, Xq, s_x, x_rot_dbg,
                                        x_rot_dbg, stream)
 
 
-def clq_w4a4_linear(Xq, s_x, Wq, s_w, bias, M, N, K, b, out_dtype, Y,
-                    acc_dbg, stream):
-    return load().clq_w4a4_linear(Xq, s_x, Wq, s_w, bias, M, N, K, b,
-                                  out_dtype, Y, acc_dbg, stream)
+def clq_expand_weights(Wq, N, K, We, stream):
+    return load().clq_expand_weights(Wq, N, K, We, stream)
 
 
-def clq_fused_linear(X, dtype, M, K, ldx, perm, b, Wq, s_w, bias, N, Y,
-                     stream):
-    return load().clq_fused_linear(X, dtype, M, K, ldx, perm, b, Wq, s_w,
-                                   bias, N, Y, stream)
+def clq_w4a4_linear(Xq, s_x, W, w_format, s_w, bias, M, N, K, b, out_dtype,
+                    Y, acc_dbg, stream):
+    return load().clq_w4a4_linear(Xq, s_x, W, w_format, s_w, bias, M, N, K,
+                                  b, out_dtype, Y, acc_dbg, stream)
+
+
+def clq_fused_linear_workspace_size(M, K):
+    return load().clq_fused_linear_workspace_size(M, K)
+
+
+def clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N,
+                     Y, workspace, workspace_bytes, stream):
+    return load().clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format,
+                                   s_w, bias, N, Y, workspace,
+                                   workspace_bytes, stream)
 
 
 def clq_get_device_status(stream, out):
@@ -202,11 +216,29 @@ def rotate_quant_act(X, perm, b, Xq=None, s_x=None, with_rot=False,
     return (Xq, s_x, rot) if with_rot else (Xq, s_x)
 
 
-def w4a4_linear(Xq, s_x, Wq, s_w, b, bias=None, out_dtype=torch.float16,
+def expand_weights(Wq, stream=None):
+    """Packed codes [N, K/2] -> E4M3 execution layout [N, K] (uint8)."""
+    N, Kh = Wq.shape
+    We = torch.empty((N, 2 * Kh), dtype=torch.uint8, device=Wq.device)
+    _check(clq_expand_weights(_ptr(Wq), N, 2 * Kh, _ptr(We), _stream(stream)),
+           "clq_expand_weights")
+    return We
+
+
+def _wformat(W, K):
+    if W.shape[1] == K:
+        return CLQ_W_E4M3
+    if 2 * W.shape[1] == K:
+        return CLQ_W_INT4_PACKED
+    raise ValueError("weights must be [N, K/2] packed or [N, K] E4M3")
+
+
+def w4a4_linear(Xq, s_x, W, s_w, b, bias=None, out_dtype=torch.float16,
                 Y=None, with_acc=False, stream=None):
-    """Packed codes -> Y [M, N] (out_dtype)[, acc int32 [M, N]]."""
+    """Packed activation codes x weight codes (packed [N, K/2] or E4M3
+    [N, K]) -> Y [M, N] (out_dtype)[, acc int32 [M, N]]."""
     M, Kh = Xq.shape
-    N = Wq.shape[0]
+    N = W.shape[0]
     K = 2 * Kh
     if Y is None:
         Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
@@ -214,21 +246,32 @@ def w4a4_linear(Xq, s_x, Wq, s_w, b, bias=None, out_dtype=torch.float16,
            if with_acc else None)
     if bias is not None and bias.dtype != Y.dtype:
         raise TypeError("bias must have the output dtype")
-    _check(clq_w4a4_linear(_ptr(Xq), _ptr(s_x), _ptr(Wq), _ptr(s_w),
-                           _ptr(bias), M, N, K, b, _dt(Y), _ptr(Y), _ptr(acc),
-                           _stream(stream)), "clq_w4a4_linear")
+    _check(clq_w4a4_linear(_ptr(Xq), _ptr(s_x), _ptr(W), _wformat(W, K),
+                           _ptr(s_w), _ptr(bias), M, N, K, b, _dt(Y), _ptr(Y),
+                           _ptr(acc), _stream(stream)), "clq_w4a4_linear")
     return (Y, acc) if with_acc else Y
 
 
-def fused_linear(X, perm, b, Wq, s_w, bias=None, Y=None, stream=None):
-    """X [M, K] -> Y [M, N] in X's dtype, rotate-quant fused into the GEMM."""
+def fused_workspace(M, K, device):
+    """A workspace tensor large enough for fused_linear on M x K inputs."""
+    n = clq_fused_linear_workspace_size(M, K)
+    return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+
+
+def fused_linear(X, perm, b, W, s_w, bias=None, Y=None, workspace=None,
+                 stream=None):
+    """X [M, K] -> Y [M, N] in X's dtype, rotate-quant and GEMM in one
+    kernel.  W is packed [N, K/2] or E4M3 [N, K]."""
     _row_major(X, "X")
     M, K = X.shape
-    N = Wq.shape[0]
+    N = W.shape[0]
     if Y is None:
         Y = torch.empty((M, N), dtype=X.dtype, device=X.device)
+    if workspace is None:
+        workspace = fused_workspace(M, K, X.device)
     _check(clq_fused_linear(_ptr(X), _dt(X), M, K, X.stride(0), _ptr(perm), b,
-                            _ptr(Wq), _ptr(s_w), _ptr(bias), N, _ptr(Y),
+                            _ptr(W), _wformat(W, K), _ptr(s_w), _ptr(bias), N,
+                            _ptr(Y), _ptr(workspace), workspace.numel(),
                             _stream(stream)), "clq_fused_linear")
     return Y
 
@@ -250,13 +293,16 @@ class PreparedLinear:
     """A quantized linear layer: the prepared-weight package (Wq, s_w, perm,
     b, bias) of Sec. 3.3, where the swap vector is the only stored part of G.
 
-    ``state_dict()`` / ``from_state_dict()`` hold plain tensors for
-    ``torch.save``.  Calling the object runs the separate rotate-quant and
-    GEMM kernels (``fused=False``) or the fused kernel.
+    Wq holds the packed INT4 codes (the storage format, 4 bits per weight);
+    We the same codes in the E4M3 execution layout the GEMM loads directly.
+    ``state_dict()`` keeps only the packed codes; ``from_state_dict()``
+    expands them again.  Calling the object runs the separate rotate-quant
+    and GEMM kernels (``fused=False``) or the fused kernel.
     """
 
-    def __init__(self, Wq, s_w, perm, b, bias=None):
+    def __init__(self, Wq, s_w, perm, b, bias=None, We=None):
         self.Wq, self.s_w, self.perm, self.b, self.bias = Wq, s_w, perm, b, bias
+        self.We = expand_weights(Wq) if We is None else We
 
     @classmethod
     def from_weight(cls, W, perm, b, bias=None, clip=None):
@@ -275,10 +321,10 @@ class PreparedLinear:
     def from_state_dict(cls, d):
         return cls(d["Wq"], d["s_w"], d["perm"], int(d["b"]), d.get("bias"))
 
-    def __call__(self, X, fused=False, stream=None):
+    def __call__(self, X, fused=False, workspace=None, stream=None):
         if fused:
-            return fused_linear(X, self.perm, self.b, self.Wq, self.s_w,
-                                self.bias, stream=stream)
+            return fused_linear(X, self.perm, self.b, self.We, self.s_w,
+                                self.bias, workspace=workspace, stream=stream)
         Xq, s_x = rotate_quant_act(X, self.perm, self.b, stream=stream)
-        return w4a4_linear(Xq, s_x, self.Wq, self.s_w, self.b, self.bias,
+        return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, self.bias,
                            out_dtype=X.dtype, stream=stream)

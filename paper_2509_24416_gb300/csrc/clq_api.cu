@@ -70,6 +70,40 @@ clq_status check_k_b(int K, int b) {
 
 bool valid_dtype(int d) { return d == CLQ_F16 || d == CLQ_BF16; }
 
+bool valid_wformat(int f) { return f == CLQ_W_INT4_PACKED || f == CLQ_W_E4M3; }
+
+// Launch of the fused kernel on a workspace laid out as `ws` (validated).
+clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
+                        const int32_t* perm, int32_t b, const uint8_t* W, clq_wformat w_format,
+                        const float* s_w, const void* bias, int32_t N, void* Y, uint8_t* wsp,
+                        const clq::FusedWorkspace& ws, int32_t* status, void* stream) {
+  clq::RotateQuantArgs rq{};
+  rq.X = X;
+  rq.M = M;
+  rq.K = K;
+  rq.ld = ldx;
+  rq.perm = perm;
+  rq.clip = nullptr;
+  rq.Q = wsp + ws.codes_off;
+  rq.S = reinterpret_cast<float*>(wsp + ws.scales_off);
+  rq.rot = nullptr;
+  rq.status = status;
+  clq::GemmArgs g{};
+  g.s_x = rq.S;
+  g.s_w = s_w;
+  g.bias = bias;
+  g.Y = Y;
+  g.acc_dbg = nullptr;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.inv_b = 1.0f / static_cast<float>(b);
+  g.status = status;
+  return from_cuda(clq::launch_fused_linear(rq, W, w_format, g, log2i(b), dtype,
+                                            reinterpret_cast<uint32_t*>(wsp + ws.ready_off),
+                                            static_cast<cudaStream_t>(stream)));
+}
+
 clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ld,
                                const int32_t* perm, int32_t b, const float* clip, uint8_t* Q,
                                float* S, float* rot, void* stream) {
@@ -97,6 +131,7 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   a.S = S;
   a.rot = rot;
   a.status = status;
+  a.logb = log2i(b);
   return from_cuda(
       clq::launch_rotate_quant(a, dtype, log2i(b), static_cast<cudaStream_t>(stream)));
 }
@@ -165,17 +200,31 @@ clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M, int32
   return rotate_quant_common(X, dtype, M, K, ldx, perm, b, nullptr, Xq, s_x, x_rot_dbg, stream);
 }
 
-clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x, const uint8_t* Wq,
-                           const float* s_w, const void* bias, int32_t M, int32_t N, int32_t K,
-                           int32_t b, clq_dtype out_dtype, void* Y, int32_t* acc_dbg,
-                           void* stream) {
-  if (!valid_dtype(out_dtype) || M < 0 || N < 0) return CLQ_ERR_INVALID_ARG;
+clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K, uint8_t* We,
+                              void* stream) {
+  if (N < 0 || K < 0) return CLQ_ERR_INVALID_ARG;
+  if (K < 32 || K > 16384 || K % 32 != 0) return CLQ_ERR_SHAPE;
+  if (N == 0) return CLQ_OK;
+  if (Wq == nullptr || We == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(Wq, 16) || !aligned(We, 16)) return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  return from_cuda(clq::launch_expand_weights(Wq, N, K, We, static_cast<cudaStream_t>(stream)));
+}
+
+clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x, const uint8_t* W,
+                           clq_wformat w_format, const float* s_w, const void* bias, int32_t M,
+                           int32_t N, int32_t K, int32_t b, clq_dtype out_dtype, void* Y,
+                           int32_t* acc_dbg, void* stream) {
+  if (!valid_dtype(out_dtype) || !valid_wformat(w_format) || M < 0 || N < 0)
+    return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
   if (M == 0 || N == 0) return CLQ_OK;
-  if (Xq == nullptr || s_x == nullptr || Wq == nullptr || s_w == nullptr || Y == nullptr)
+  if (Xq == nullptr || s_x == nullptr || W == nullptr || s_w == nullptr || Y == nullptr)
     return CLQ_ERR_INVALID_ARG;
-  if (!aligned(Xq, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_x, 4) ||
+  if (!aligned(Xq, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(s_x, 4) ||
       !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)) ||
       (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
     return CLQ_ERR_ALIGN;
@@ -193,40 +242,39 @@ clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x, const uint8_t* W
   g.K = K;
   g.inv_b = 1.0f / static_cast<float>(b);
   g.status = status;
-  return from_cuda(clq::launch_w4a4_gemm(Xq, Wq, g, out_dtype, static_cast<cudaStream_t>(stream)));
+  return from_cuda(
+      clq::launch_w4a4_gemm(Xq, W, w_format, g, out_dtype, static_cast<cudaStream_t>(stream)));
+}
+
+size_t clq_fused_linear_workspace_size(int32_t M, int32_t K) {
+  if (M < 0 || K < 32 || K > 16384 || K % 32 != 0) return 0;
+  return clq::fused_workspace_layout(M, K).bytes;
 }
 
 clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
-                            const int32_t* perm, int32_t b, const uint8_t* Wq, const float* s_w,
-                            const void* bias, int32_t N, void* Y, void* stream) {
-  if (!valid_dtype(dtype) || M < 0 || N < 0) return CLQ_ERR_INVALID_ARG;
+                            const int32_t* perm, int32_t b, const uint8_t* W,
+                            clq_wformat w_format, const float* s_w, const void* bias, int32_t N,
+                            void* Y, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!valid_dtype(dtype) || !valid_wformat(w_format) || M < 0 || N < 0)
+    return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
   if (ldx < K) return CLQ_ERR_SHAPE;
   if (ldx % 8 != 0) return CLQ_ERR_ALIGN;
   if (M == 0 || N == 0) return CLQ_OK;
-  if (X == nullptr || perm == nullptr || Wq == nullptr || s_w == nullptr || Y == nullptr)
+  if (X == nullptr || perm == nullptr || W == nullptr || s_w == nullptr || Y == nullptr ||
+      workspace == nullptr)
     return CLQ_ERR_INVALID_ARG;
-  if (!aligned(X, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(perm, 4) ||
-      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)))
+  const clq::FusedWorkspace ws = clq::fused_workspace_layout(M, K);
+  if (workspace_bytes < ws.bytes) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(X, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(perm, 4) ||
+      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)) || !aligned(workspace, 256))
     return CLQ_ERR_ALIGN;
   int32_t* status = nullptr;
   st = device_setup(&status);
   if (st != CLQ_OK) return st;
-  clq::FusedArgs f{};
-  f.X = X;
-  f.ld = ldx;
-  f.perm = perm;
-  f.logb = log2i(b);
-  f.s_w = s_w;
-  f.bias = bias;
-  f.Y = Y;
-  f.M = M;
-  f.N = N;
-  f.K = K;
-  f.inv_b = 1.0f / static_cast<float>(b);
-  f.status = status;
-  return from_cuda(clq::launch_fused_linear(Wq, f, dtype, static_cast<cudaStream_t>(stream)));
+  return fused_common(X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N, Y,
+                      static_cast<uint8_t*>(workspace), ws, status, stream);
 }
 
 clq_status clq_get_device_status(void* stream, int32_t* out) {

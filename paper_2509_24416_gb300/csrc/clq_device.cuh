@@ -104,6 +104,17 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
       : "memory");
 }
 
+// Untiled bulk copy global -> shared (16-byte aligned addresses, size a
+// multiple of 16), completing `bytes` of transaction count on `bar`.
+__device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(smem_addr(smem_dst)),
+      "l"(gsrc), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensor_map(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map))
                : "memory");
@@ -210,6 +221,11 @@ struct Num<__half> {
   static __device__ __forceinline__ uint16_t from_f(float v) {
     return __half_as_ushort(__float2half_rn(v));
   }
+  // two values rounded to nearest and packed, lo in the low half
+  static __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    const __half2 h = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+  }
 };
 template <>
 struct Num<__nv_bfloat16> {
@@ -219,19 +235,10 @@ struct Num<__nv_bfloat16> {
   static __device__ __forceinline__ uint16_t from_f(float v) {
     return __bfloat16_as_ushort(__float2bfloat16_rn(v));
   }
+  static __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+  }
 };
-
-// Per-row symmetric INT4 code of v with scale s > 0 (Eq. 1, symmetric
-// reading): clamp(rint(v / s), -7, 7) with IEEE fp32 division and ties to
-// even.  v * (1/s) is used first; when it lands within 1e-5 of a
-// half-integer, where it could round differently from the quotient, the
-// exact quotient decides.
-__device__ __forceinline__ int quant_code(float v, float s, float rcp) {
-  float r = v * rcp;
-  float q = rintf(r);
-  if (fabsf(fabsf(r - q) - 0.5f) < 1e-5f) q = rintf(__fdiv_rn(v, s));
-  q = fminf(fmaxf(q, -7.0f), 7.0f);
-  return static_cast<int>(q);
-}
 
 }  // namespace clq

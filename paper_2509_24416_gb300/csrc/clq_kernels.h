@@ -19,6 +19,7 @@ struct RotateQuantArgs {
   float* rot;            // [M][K] or null
   int32_t rows_per_tile; // filled in by the launcher
   int32_t* status;       // device status word
+  int32_t logb;          // log2(b)
 };
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
@@ -38,32 +39,36 @@ struct GemmArgs {
   int32_t* status;
 };
 
-// Packed INT4 operands are described by TMA maps built here from raw
-// pointers: A = Xq [M][K/2], B = Wq [N][K/2].
-cudaError_t launch_w4a4_gemm(const uint8_t* Xq, const uint8_t* Wq, const GemmArgs& g,
-                             int out_dtype, cudaStream_t st);
+// A = Xq [M][K/2] packed; B = weights in `w_format` (CLQ_W_INT4_PACKED
+// [N][K/2] or CLQ_W_E4M3 [N][K]); TMA maps are built here from raw pointers.
+cudaError_t launch_w4a4_gemm(const uint8_t* Xq, const uint8_t* W, int w_format,
+                             const GemmArgs& g, int out_dtype, cudaStream_t st);
 
-struct FusedArgs {
-  const void* X;        // [M][ld]
-  int32_t ld;
-  const int32_t* perm;  // [K]
-  int32_t logb;
-  const float* s_w;
-  const void* bias;
-  void* Y;
-  int32_t M, N, K;
-  float inv_b;
-  int32_t* status;
+cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st);
+
+// Workspace of the fused kernel: codes, scales, per-token-block row counters.
+struct FusedWorkspace {
+  size_t codes_off, scales_off, ready_off, bytes;
 };
+FusedWorkspace fused_workspace_layout(int M, int K);
 
-cudaError_t launch_fused_linear(const uint8_t* Wq, const FusedArgs& f, int dtype,
+// Fused rotate-quant + GEMM: `rq` describes the activation side (its Q / S
+// point into the workspace), `g` the product (s_x = workspace scales).
+cudaError_t launch_fused_linear(const RotateQuantArgs& rq, const uint8_t* W, int w_format,
+                                const GemmArgs& g, int logb, int dtype, uint32_t* ready,
                                 cudaStream_t st);
 
 // Bounded-wait self test (one CTA, one mbarrier nothing arrives at).
 cudaError_t launch_wait_selftest(uint64_t timeout_ns, int32_t* status, cudaStream_t st);
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point.
+bool encode_tma_2d(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize, const void* base,
+                   uint64_t inner, uint64_t rows, uint32_t box_inner, uint32_t box_rows,
+                   CUtensorMapSwizzle swz);
 bool encode_tma_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
                       uint64_t rows, uint32_t box_inner, uint32_t box_rows);
+// 2-byte output tile map for the epilogue stores (box 32 columns x 128 rows).
+bool encode_tma_out_tile(CUtensorMap* map, void* Y, int M, int N);
+int sm_count();
 
 }  // namespace clq

@@ -1,11 +1,158 @@
-// Fused rotate-quant + W4A4 GEMM (placeholder until the fused kernel lands).
-#include "clq_device.cuh"
-#include "clq_kernels.h"
+// Fused W4A4 OBS linear: rotate-quant and the tcgen05 GEMM in one persistent
+// kernel.
+//
+// Why not a per-tile prologue: quantizing a token needs the abs-max of its
+// whole rotated row before any code exists, and a K step of the product
+// needs permuted positions whose source columns are spread over the whole
+// row.  For the paper's hidden sizes a 128-token block of rows does not fit
+// in shared memory next to the operand pipeline, so each CTA cannot rotate
+// only "its" A tile.  Instead every CTA first rotates and quantizes its share
+// of token rows (rq::run, all threads) into the caller's workspace and
+// publishes, per 128-token block, how many rows are done (release: proxy
+// fence, __threadfence, atomicAdd).  Then the same CTA turns into a GEMM
+// pipeline (gemm::pipeline); its TMA producer waits (acquire, bounded) until
+// all rows of a tile's token block are published before loading that block's
+// codes.  One launch, no host round trip, and the codes stay in L2 for the
+// layer sizes of the paper's models.
+#include "gemm_pipeline.cuh"
+#include "rq_device.cuh"
 
 namespace clq {
 
-cudaError_t launch_fused_linear(const uint8_t*, const FusedArgs&, int, cudaStream_t) {
-  return cudaErrorNotSupported;
+namespace {
+
+using namespace gemm;
+
+constexpr int FT = 512;  // threads: the RQ phase uses all; the GEMM phase 448
+
+struct PublishRows {
+  uint32_t* ready;
+  __device__ void operator()(int row0, int rows) const {
+    fence_proxy_async_global();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      int r = row0;
+      const int end = row0 + rows;
+      while (r < end) {
+        const int mb = r / BM;
+        const int stop = min(end, (mb + 1) * BM);
+        atomicAdd(ready + mb, static_cast<unsigned>(stop - r));
+        r = stop;
+      }
+    }
+  }
+};
+
+template <typename T, bool BPACK>
+__global__ void __launch_bounds__(FT, 1)
+    fused_linear_kernel(const __grid_constant__ CUtensorMap mapA,
+                        const __grid_constant__ CUtensorMap mapB,
+                        const __grid_constant__ CUtensorMap mapY, RotateQuantArgs rq, GemmArgs g,
+                        uint32_t* ready, uint32_t* tile_counter, int use_tma_store,
+                        int rq_stages) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ Barriers bars;
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  setup<BPACK>(&bars);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars.tmem_slot;
+
+  rq::run<T, -1, false>(rq, smem, rq_stages, tile_counter, PublishRows{ready});
+  __syncthreads();
+
+  const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
+  pipeline<T, BPACK>(maps, g, smem, &bars, tmem, ready);
+  tc_fence_before();
+  __syncthreads();
+  teardown(tmem);
+}
+
+template <typename T, bool BPACK>
+cudaError_t launch_t(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
+                     const RotateQuantArgs& rq, const GemmArgs& g, uint32_t* ready,
+                     int use_tma_store, int rq_stages, size_t smem, int grid, cudaStream_t st) {
+  uint32_t* tile_counter = ready + (g.M + BM - 1) / BM;
+  auto k = fused_linear_kernel<T, BPACK>;
+  cudaError_t e =
+      cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store,
+                             rq_stages);
+  return cudaGetLastError();
+}
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+}  // namespace
+
+FusedWorkspace fused_workspace_layout(int M, int K) {
+  FusedWorkspace w{};
+  const size_t m = static_cast<size_t>(M < 0 ? 0 : M);
+  w.codes_off = 0;
+  w.scales_off = align256(m * static_cast<size_t>(K / 2));
+  w.ready_off = align256(w.scales_off + 4 * m);
+  w.bytes = align256(w.ready_off + 4 * ((m + BM - 1) / BM + 1));  // + tile counter
+  return w;
+}
+
+cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, int w_format,
+                                const GemmArgs& g, int logb, int dtype, uint32_t* ready,
+                                cudaStream_t st) {
+  const bool bpack = w_format == CLQ_W_INT4_PACKED;
+  const size_t gemm_bytes = bpack ? Cfg<true>::BYTES : Cfg<false>::BYTES;
+  const size_t limit = 227u * 1024u - 2048u;  // dynamic + static shared memory
+  // Rotate-quant phase: as many rows per tile as 512 threads cover, then as
+  // many raw stages (2..4) as fit next to them.
+  RotateQuantArgs rq = rq_in;
+  rq.logb = logb;
+  const int segs = rq.K / 32;
+  int R = std::max(1, FT / segs);
+  int stages = rq::kMaxStages;
+  while (stages > 2 && rq::smem_bytes(rq.K, R, stages) > limit) --stages;
+  while (R > 1 && rq::smem_bytes(rq.K, R, stages) > limit) --R;
+  if (rq::smem_bytes(rq.K, R, stages) > limit || R * segs > FT) return cudaErrorInvalidValue;
+  rq.rows_per_tile = R;
+  const size_t smem = std::max(gemm_bytes, rq::smem_bytes(rq.K, R, stages)) + 1024;
+
+  const int tiles_m = (g.M + BM - 1) / BM;
+  cudaError_t e =
+      cudaMemsetAsync(ready, 0, sizeof(uint32_t) * (static_cast<size_t>(tiles_m) + 1), st);
+  if (e != cudaSuccess) return e;
+
+  CUtensorMap mapA, mapB, mapY;
+  const uint64_t kb = static_cast<uint64_t>(g.K) / 2;
+  if (!encode_tma_2d_u8(&mapA, rq.Q, kb, static_cast<uint64_t>(g.M), BKP, BM))
+    return cudaErrorInvalidValue;
+  if (bpack) {
+    if (!encode_tma_2d_u8(&mapB, W, kb, static_cast<uint64_t>(g.N), BKP, BN))
+      return cudaErrorInvalidValue;
+  } else {
+    if (!encode_tma_2d(&mapB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, W, static_cast<uint64_t>(g.K),
+                       static_cast<uint64_t>(g.N), BK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  }
+  const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
+  if (use_tma_store) {
+    if (!encode_tma_out_tile(&mapY, g.Y, g.M, g.N)) return cudaErrorInvalidValue;
+  } else {
+    mapY = mapA;  // unused
+  }
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  const int grid = sms;
+  if (dtype == CLQ_F16)
+    return bpack ? launch_t<__half, true>(mapA, mapB, mapY, rq, g, ready, use_tma_store, stages,
+                                          smem, grid, st)
+                 : launch_t<__half, false>(mapA, mapB, mapY, rq, g, ready, use_tma_store, stages,
+                                           smem, grid, st);
+  return bpack ? launch_t<__nv_bfloat16, true>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
+                                               stages, smem, grid, st)
+               : launch_t<__nv_bfloat16, false>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
+                                                stages, smem, grid, st);
 }
 
 }  // namespace clq

@@ -1,0 +1,189 @@
+// Pieces shared by the W4A4 GEMM and the fused rotate-quant + GEMM kernels:
+// tile shape, nibble -> E4M3 unpacking into the tcgen05 operand layout, and
+// the TMEM -> fp16/bf16 epilogue with TMA stores.
+#pragma once
+
+#include "clq_device.cuh"
+
+namespace clq {
+namespace gemm {
+
+constexpr int BM = 128;           // rows of A (tokens) per tile
+constexpr int BN = 256;           // rows of B (output channels) per tile
+constexpr int BK = 128;           // codes per K step = one 128-byte swizzle row
+constexpr int BKP = BK / 2;       // packed bytes per row per K step
+constexpr int A_U = BM * BK;      // 16 KB unpacked A stage
+constexpr int B_U = BN * BK;      // 32 KB unpacked B stage
+constexpr int A_P = BM * BKP;     // 8 KB packed A stage
+constexpr int B_P = BN * BKP;     // 16 KB packed B stage
+constexpr int EPI_COLS = 32;      // output columns per epilogue store
+constexpr int EPI_BYTES = BM * EPI_COLS * 2;  // 8 KB staging buffer
+constexpr int TMEM_COLS = 512;    // two 128 x 256 fp32 accumulators
+constexpr uint32_t kEpiBarrier = 1;  // named barrier id of the epilogue warps
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
+__device__ __forceinline__ uint32_t pack2(uint16_t lo, uint16_t hi) {
+  return static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+}
+
+__device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+// Eight 4-bit two's-complement codes (code j in nibble j) -> eight E4M3
+// bytes.  Magnitude tables for the non-negative codes 0..7 and the negative
+// codes -8..-1 are looked up with prmt on the low three bits of each nibble;
+// the sign bit of each nibble, replicated to a byte mask by prmt's sign mode,
+// selects between them.
+__device__ __forceinline__ uint2 nibbles_to_e4m3(uint32_t w) {
+  const uint32_t P0 = 0x44403800u, P1 = 0x4E4C4A48u;  // e4m3(0..7)
+  const uint32_t N0 = 0xCACCCED0u, N1 = 0xB8C0C4C8u;  // e4m3(-8..-1)
+  const uint32_t sel_lo = w & 0x7777u;
+  const uint32_t sel_hi = (w >> 16) & 0x7777u;
+  const uint32_t w4 = w << 4;
+  const uint32_t m_lo = prmt(w4, w, 0xD9C8u);
+  const uint32_t m_hi = prmt(w4, w, 0xFBEAu);
+  const uint32_t p_lo = prmt(P0, P1, sel_lo), n_lo = prmt(N0, N1, sel_lo);
+  const uint32_t p_hi = prmt(P0, P1, sel_hi), n_hi = prmt(N0, N1, sel_hi);
+  return make_uint2((p_lo & ~m_lo) | (n_lo & m_lo), (p_hi & ~m_hi) | (n_hi & m_hi));
+}
+
+// Byte offset of 16-byte chunk c (0..7) of row r in a K-major E4M3 operand
+// tile with the 128-byte swizzle: 8-row atoms of 1024 bytes.
+__device__ __forceinline__ uint32_t sw128_offset(int r, int c) {
+  return static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// Unpack ROWS x 64 packed bytes (row-major staging) into the swizzled E4M3
+// tile, NT threads cooperating (thread index t).
+template <int ROWS, int NT>
+__device__ __forceinline__ void unpack_rows(const uint8_t* __restrict__ src,
+                                            uint8_t* __restrict__ dst, int t) {
+#pragma unroll
+  for (int i = 0; i < ROWS * 4 / NT; ++i) {
+    const int q = t + NT * i;
+    const int r = q >> 2;
+    const int c = q & 3;
+    const uint4 p = *reinterpret_cast<const uint4*>(src + r * BKP + c * 16);
+    const uint2 e0 = nibbles_to_e4m3(p.x), e1 = nibbles_to_e4m3(p.y);
+    const uint2 e2 = nibbles_to_e4m3(p.z), e3 = nibbles_to_e4m3(p.w);
+    *reinterpret_cast<uint4*>(dst + sw128_offset(r, 2 * c)) = make_uint4(e0.x, e0.y, e1.x, e1.y);
+    *reinterpret_cast<uint4*>(dst + sw128_offset(r, 2 * c + 1)) =
+        make_uint4(e2.x, e2.y, e3.x, e3.y);
+  }
+}
+
+// 32 lanes x 32 bit, 32 consecutive columns per thread.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* smem_src,
+                                             int32_t x, int32_t y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(smem_addr(smem_src)), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// Epilogue of one 128 x 256 tile by 128 threads (four warps, any warp order:
+// warp w reads TMEM lanes 32 * (w % 4) ..).  y = acc * s_x[row] * s_w[col] /
+// b + bias[col], rounded to OutT.  With a TMA map for Y, each 128 x 32 block
+// goes through a 64-byte-swizzled staging buffer and one bulk tensor store;
+// otherwise (N not a multiple of 8) threads store their row directly.
+// `store_count` numbers the staging buffers used so far (alternating).
+template <typename OutT>
+__device__ __forceinline__ void epilogue_tile(uint32_t tmem_acc, int warp_q, int et, int m0,
+                                              int n0, int M, int N, float sx,
+                                              const float* col_scale, const float* col_bias,
+                                              uint8_t* staging, const CUtensorMap* mapY,
+                                              void* Y, int32_t* acc_dbg, int& store_count) {
+  const int row_in_tile = warp_q * 32 + (et & 31);
+  const int row = m0 + row_in_tile;
+  const uint32_t lane_base = tmem_acc + (static_cast<uint32_t>(warp_q * 32) << 16);
+#pragma unroll 1
+  for (int c = 0; c < BN; c += EPI_COLS) {
+    if (n0 + c >= N) break;
+    uint32_t r[32];
+    tmem_ld32(lane_base + c, r);
+    tmem_ld_wait();
+    uint32_t o[16];
+    const float2 sx2 = make_float2(sx, sx);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float4 cs = *reinterpret_cast<const float4*>(col_scale + c + 4 * j);
+      const float4 cb = *reinterpret_cast<const float4*>(col_bias + c + 4 * j);
+      const float2 a0 = make_float2(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]));
+      const float2 a1 = make_float2(__uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+      const float2 y0 = __ffma2_rn(a0, __fmul2_rn(sx2, make_float2(cs.x, cs.y)),
+                                   make_float2(cb.x, cb.y));
+      const float2 y1 = __ffma2_rn(a1, __fmul2_rn(sx2, make_float2(cs.z, cs.w)),
+                                   make_float2(cb.z, cb.w));
+      o[2 * j] = Num<OutT>::pack2(y0.x, y0.y);
+      o[2 * j + 1] = Num<OutT>::pack2(y1.x, y1.y);
+    }
+    if (acc_dbg != nullptr && row < M) {
+      int32_t* arow = acc_dbg + static_cast<size_t>(row) * N + n0 + c;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (n0 + c + j < N) arow[j] = __float2int_rn(__uint_as_float(r[j]));
+    }
+    if (mapY != nullptr) {
+      uint8_t* sb = staging + (store_count & 1) * EPI_BYTES;
+      if (et == 0) bulk_wait_read<1>();
+      named_bar_sync(kEpiBarrier, 128);
+      uint8_t* srow = sb + row_in_tile * 64;
+      const int sw = (row_in_tile >> 1) & 3;
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        *reinterpret_cast<uint4*>(srow + ((q ^ sw) << 4)) =
+            make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+      fence_proxy_async_smem();
+      named_bar_sync(kEpiBarrier, 128);
+      if (et == 0) {
+        tma_store_2d(mapY, sb, n0 + c, m0);
+        bulk_commit();
+      }
+      ++store_count;
+    } else if (row < M) {
+      uint16_t* yrow = static_cast<uint16_t*>(Y) + static_cast<size_t>(row) * N + n0 + c;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        if (n0 + c + 2 * j < N) yrow[2 * j] = static_cast<uint16_t>(o[j] & 0xFFFFu);
+        if (n0 + c + 2 * j + 1 < N) yrow[2 * j + 1] = static_cast<uint16_t>(o[j] >> 16);
+      }
+    }
+  }
+}
+
+}  // namespace gemm
+}  // namespace clq

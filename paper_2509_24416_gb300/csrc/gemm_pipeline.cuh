@@ -1,0 +1,285 @@
+// Warp-specialized tcgen05 GEMM pipeline for the packed INT4 activations x
+// INT4 weights product, shared by the standalone GEMM and the fused kernel.
+//
+// acc[i][n] = sum_k qx[i][k] * qw[n][k] is an exact integer: |q| <= 7, so
+// every product is an integer of magnitude <= 49 and, for K <= 16384, every
+// partial sum stays below 2^24.  sm_103a has no integer tcgen05 MMA, so the
+// codes ride on E4M3, which holds every integer in [-7, 7] exactly, through
+// tcgen05.mma kind::f8f6f4 with fp32 accumulation in tensor memory; the
+// integer accumulators come out exact as long as the fp32 sums are exact
+// (checked bit for bit against the int64 oracle, +-7 codes at K = 16384).
+//
+// Persistent: one CTA per SM walks 128 (M) x 256 (N) tiles in a static
+// round-robin order, K step 128 codes.  Warp roles:
+//   warp 4       TMA producer: packed A (64 B x 128 rows) into a staging
+//                buffer and B either packed (64 B x 256 rows, BPACK) or as
+//                E4M3 bytes (128 B x 256 rows, 128-byte swizzle) straight
+//                into the MMA operand buffer;
+//   warps 6-13   unpack nibbles to E4M3 bytes in the 128-byte-swizzled
+//                K-major layout the MMA reads (A, and B when BPACK);
+//   warp 5       one lane issues tcgen05.mma (4 x K=32 per stage) and commits
+//                stage and tile completion;
+//   warps 0-3    epilogue: TMEM -> registers -> scale, bias, round ->
+//                swizzled staging -> TMA tensor store.  Two TMEM accumulators
+//                let the epilogue of tile i overlap the MMAs of tile i + 1.
+//   other warps  idle in this phase.
+// With `ready` counters (fused kernel), the producer waits until all rows of
+// a tile's token block have been published before loading its A tiles.
+// Every wait is bounded; on a timeout the roles drain their own copies and
+// MMAs and return (status word: CLQ_ERR_TIMEOUT).
+#pragma once
+
+#include "gemm_common.cuh"
+#include "clq_kernels.h"
+
+namespace clq {
+namespace gemm {
+
+constexpr int NUM_UNPACK = 256;
+constexpr int WARP_TMA = 4;
+constexpr int WARP_MMA = 5;
+constexpr int WARP_UNPACK0 = 6;
+constexpr int MIN_THREADS = (WARP_UNPACK0 + NUM_UNPACK / 32) * 32;  // 448
+
+template <bool BPACK>
+struct Cfg {
+  static constexpr int S = BPACK ? 2 : 3;  // pipeline stages
+  static constexpr size_t OFF_UA = 0;
+  static constexpr size_t OFF_UB = OFF_UA + S * A_U;
+  static constexpr size_t OFF_PA = OFF_UB + S * B_U;
+  static constexpr size_t OFF_PB = OFF_PA + S * A_P;
+  static constexpr size_t OFF_EPI = OFF_PB + (BPACK ? S * B_P : 0);
+  static constexpr size_t OFF_COL = OFF_EPI + 2 * EPI_BYTES;
+  static constexpr size_t BYTES = OFF_COL + 2 * BN * sizeof(float);
+  static constexpr uint32_t TX = A_P + (BPACK ? B_P : B_U);
+};
+
+struct __align__(8) Barriers {
+  uint64_t tma_full[3];  // packed A (+ B) landed
+  uint64_t unpacked[3];  // operand stage ready for the MMA
+  uint64_t mma_done[3];  // MMAs reading the stage completed
+  uint64_t acc_full[2];
+  uint64_t acc_empty[2];
+  uint64_t drained;
+  uint32_t tmem_slot;
+  int32_t abort;
+};
+
+struct Maps {
+  const CUtensorMap* A;
+  const CUtensorMap* B;
+  const CUtensorMap* Y;  // null: direct stores
+};
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Barrier init (thread 0) and TMEM allocation (warp WARP_MMA); the caller
+// follows with tcgen05 fences around a CTA barrier.
+template <bool BPACK>
+__device__ __forceinline__ void setup(Barriers* bars) {
+  constexpr int S = Cfg<BPACK>::S;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&bars->tma_full[s], 1);
+      mbar_init(&bars->unpacked[s], NUM_UNPACK);
+      mbar_init(&bars->mma_done[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bars->acc_full[s], 1);
+      mbar_init(&bars->acc_empty[s], 128);
+    }
+    mbar_init(&bars->drained, 1);
+    bars->abort = 0;
+    fence_mbarrier_init();
+  }
+  if ((threadIdx.x >> 5) == WARP_MMA) {
+    tmem_alloc(&bars->tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+}
+
+// Wait (bounded) until all rows of token block m are published.
+__device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, uint32_t need,
+                                                volatile int32_t* abort, int32_t* status) {
+  const uint64_t t0 = global_timer_ns();
+  while (ld_acquire_u32(ready + m) < need) {
+    if (*abort != 0) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      record_status(status, CLQ_ERR_TIMEOUT);
+      *abort = 1;
+      return false;
+    }
+    __nanosleep(128);
+  }
+  fence_proxy_async_global();
+  return true;
+}
+
+template <typename OutT, bool BPACK>
+__device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
+                                         Barriers* bars, uint32_t tmem, const uint32_t* ready) {
+  using C = Cfg<BPACK>;
+  constexpr int S = C::S;
+  float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL);
+  float* col_bias = col_scale + BN;
+  volatile int32_t* abort = &bars->abort;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int nk = (g.K + BK - 1) / BK;
+  const int tiles_n = (g.N + BN - 1) / BN;
+  const int tiles = ((g.M + BM - 1) / BM) * tiles_n;
+
+  if (warp == WARP_TMA) {
+    if (lane == 0) {
+      prefetch_tensor_map(maps.A);
+      prefetch_tensor_map(maps.B);
+      if (maps.Y != nullptr) prefetch_tensor_map(maps.Y);
+      int it = 0;  // K steps issued so far (all tiles)
+      int ready_m = -1;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        const int mb = t / tiles_n;
+        const int m0 = mb * BM;
+        const int n0 = (t % tiles_n) * BN;
+        if (ready != nullptr && mb != ready_m) {
+          if (!wait_rows_ready(ready, mb, static_cast<uint32_t>(min(BM, g.M - m0)), abort,
+                               g.status)) {
+            ok = false;
+            break;
+          }
+          ready_m = mb;
+        }
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait_bounded(&bars->mma_done[s], ((it / S) & 1) ^ 1, abort, g.status,
+                                 kWaitLimitNs)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&bars->tma_full[s], C::TX);
+          tma_load_2d(smem + C::OFF_PA + s * A_P, maps.A, kb * BKP, m0, &bars->tma_full[s]);
+          if (BPACK)
+            tma_load_2d(smem + C::OFF_PB + s * B_P, maps.B, kb * BKP, n0, &bars->tma_full[s]);
+          else
+            tma_load_2d(smem + C::OFF_UB + s * B_U, maps.B, kb * BK, n0, &bars->tma_full[s]);
+        }
+      }
+      // On an abort, the copies already in flight must land before exit.
+      if (!ok) {
+        for (int j = max(0, it - S); j < it; ++j)
+          mbar_wait_bounded(&bars->tma_full[j % S], (j / S) & 1, nullptr, nullptr, 10000000ull);
+      }
+    }
+  } else if (warp == WARP_MMA) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
+      int it = 0, tc = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tc) {
+        const int buf = tc & 1;
+        if (!mbar_wait_bounded(&bars->acc_empty[buf], ((tc >> 1) & 1) ^ 1, abort, g.status,
+                               kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + buf * BN;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait_bounded(&bars->unpacked[s], (it / S) & 1, abort, g.status,
+                                 kWaitLimitNs)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_addr(smem + C::OFF_UA + s * A_U);
+          const uint32_t b0 = smem_addr(smem + C::OFF_UB + s * B_U);
+#pragma unroll
+          for (int k = 0; k < BK / 32; ++k)
+            mma_e4m3(d, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc,
+                     (kb | k) != 0 ? 1u : 0u);
+          mma_commit(&bars->mma_done[s]);
+        }
+        if (ok) mma_commit(&bars->acc_full[buf]);
+      }
+      // Every MMA issued must complete before TMEM is released.
+      mma_commit(&bars->drained);
+      mbar_wait_bounded(&bars->drained, 0, nullptr, nullptr, 10000000ull);
+    }
+  } else if (warp >= WARP_UNPACK0 && warp < WARP_UNPACK0 + NUM_UNPACK / 32) {
+    const int ut = threadIdx.x - WARP_UNPACK0 * 32;
+    int it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int s = it % S;
+        if (!mbar_wait_bounded(&bars->tma_full[s], (it / S) & 1, abort, g.status,
+                               kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * A_U, ut);
+        if (BPACK)
+          unpack_rows<BN, NUM_UNPACK>(smem + C::OFF_PB + s * B_P, smem + C::OFF_UB + s * B_U,
+                                      ut);
+        fence_proxy_async_smem();
+        mbar_arrive(&bars->unpacked[s]);
+      }
+    }
+  } else if (warp < 4) {
+    // ---- epilogue warps 0-3 ----
+    const int et = threadIdx.x;  // 0..127
+    int tc = 0, stores = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tc) {
+      const int m0 = (t / tiles_n) * BM;
+      const int n0 = (t % tiles_n) * BN;
+      const int buf = tc & 1;
+      named_bar_sync(kEpiBarrier, 128);  // previous tile's column data consumed
+      for (int j = et; j < BN; j += 128) {
+        const int col = n0 + j;
+        float sc = 0.f, bi = 0.f;
+        if (col < g.N) {
+          sc = g.s_w[col] * g.inv_b;
+          if (g.bias != nullptr) bi = Num<OutT>::to_f(static_cast<const uint16_t*>(g.bias)[col]);
+        }
+        col_scale[j] = sc;
+        col_bias[j] = bi;
+      }
+      bool ok = mbar_wait_bounded(&bars->acc_full[buf], (tc >> 1) & 1, abort, g.status,
+                                  kWaitLimitNs);
+      ok = __all_sync(0xffffffffu, ok);
+      named_bar_sync(kEpiBarrier, 128);
+      if (!ok || *abort != 0) break;
+      tc_fence_after();
+      // s_x may have been written by other CTAs of this grid (fused kernel):
+      // read it from L2, after the tile's MMAs have completed.
+      const int row = m0 + et;
+      const float sx = row < g.M ? __ldcg(g.s_x + row) : 0.f;
+      epilogue_tile<OutT>(tmem + buf * BN, warp, et, m0, n0, g.M, g.N, sx, col_scale, col_bias,
+                          smem + C::OFF_EPI, maps.Y, g.Y, g.acc_dbg, stores);
+      tc_fence_before();
+      mbar_arrive(&bars->acc_empty[buf]);
+    }
+    if (et == 0) bulk_wait_all();
+  }
+}
+
+// After a CTA barrier that follows pipeline(): release TMEM.
+__device__ __forceinline__ void teardown(uint32_t tmem) {
+  if ((threadIdx.x >> 5) == WARP_MMA) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+}  // namespace gemm
+}  // namespace clq

@@ -67,27 +67,42 @@ def test_rotate_quant_host_validation(lib, args, code):
 
 
 @pytest.mark.parametrize("args,code", [
-    # (Xq, s_x, Wq, s_w, bias, M, N, K, b, out_dtype, Y, acc)
-    ((P, P, P, P, None, 4, 4, 64, 32, 3, P, None), 1),
-    ((P, P, P, P, None, 4, -2, 64, 32, 0, P, None), 1),
-    ((P, P, P, P, None, 4, 4, 96, 64, 0, P, None), 2),
-    ((P, P, P, P, None, 4, 4, 64, 32, 0, P + 2, None), 3),
-    ((P, P, P, P, P + 1, 4, 4, 64, 32, 0, P, None), 3),
-    ((None, P, P, P, None, 4, 4, 64, 32, 0, P, None), 1),
-    ((None, None, None, None, None, 0, 4, 64, 32, 0, None, None), 0),
-    ((None, None, None, None, None, 4, 0, 64, 32, 0, None, None), 0),
+    # (Xq, s_x, W, w_format, s_w, bias, M, N, K, b, out_dtype, Y, acc)
+    ((P, P, P, 0, P, None, 4, 4, 64, 32, 3, P, None), 1),     # bad out dtype
+    ((P, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad w_format
+    ((P, P, P, 0, P, None, 4, -2, 64, 32, 0, P, None), 1),    # negative N
+    ((P, P, P, 1, P, None, 4, 4, 96, 64, 0, P, None), 2),     # K % b
+    ((P, P, P, 0, P, None, 4, 4, 64, 32, 0, P + 2, None), 3), # misaligned Y
+    ((P, P, P, 0, P, P + 1, 4, 4, 64, 32, 0, P, None), 3),    # misaligned bias
+    ((None, P, P, 0, P, None, 4, 4, 64, 32, 0, P, None), 1),  # null Xq
+    ((None, None, None, 0, None, None, 0, 4, 64, 32, 0, None, None), 0),
+    ((None, None, None, 1, None, None, 4, 0, 64, 32, 0, None, None), 0),
 ])
 def test_w4a4_host_validation(lib, args, code):
     assert clq.clq_w4a4_linear(*args, None) == code
 
 
 def test_fused_and_prepare_host_validation(lib):
-    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 7, P, P, None, 4, P,
-                                None) == 2
-    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, P, None, 0, P,
-                                None) == 0
+    ws = clq.clq_fused_linear_workspace_size(256, 1152)
+    # 256 x 576 codes, 256 scales, 2 block counters + 1 tile counter
+    assert ws == 147456 + 1024 + 256
+    assert clq.clq_fused_linear_workspace_size(4, 48) == 0
+    # (X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N, Y, ws, bytes)
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 7, P, 0, P, None, 4, P, P,
+                                1 << 20, None) == 2
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, 0, P, None, 0, P,
+                                P, 1 << 20, None) == 0
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, 0, P, None, 4, P,
+                                P, 16, None) == 1         # workspace too small
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, 0, P, None, 4, P,
+                                P + 16, 1 << 20, None) == 3  # 256-B alignment
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, 5, P, None, 4, P,
+                                P, 1 << 20, None) == 1    # bad w_format
     assert clq.clq_prepare_weights(P, 0, 4, 64, 64, P, 32, P + 2, P, P, None,
                                    None) == 3
+    assert clq.clq_expand_weights(P, 4, 48, P, None) == 2
+    assert clq.clq_expand_weights(P, 0, 64, None, None) == 0
+    assert clq.clq_expand_weights(P + 8, 4, 64, P, None) == 3
     assert clq.clq_outlier_scores(P, 0, 0, 4, 4, P, None) == 1
     assert clq.clq_selftest_bounded_wait(10, None) == 1
     assert clq.clq_get_device_status(None, None) == 1

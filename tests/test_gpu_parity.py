@@ -178,6 +178,28 @@ def test_prepare_weights_with_clip():
 
 
 # -------------------------------------------------------------------- GEMM --
+def _decode_e4m3(byte):
+    """Value of an E4M3 byte (1 sign, 4 exponent bits with bias 7, 3 mantissa
+    bits; exponent 0 is subnormal), written out from the format definition."""
+    b = np.asarray(byte, np.int64)
+    sign = np.where(b & 0x80, -1.0, 1.0)
+    e = (b >> 3) & 0xF
+    m = b & 0x7
+    val = np.where(e == 0, m / 8.0 * 2.0 ** -6, (1 + m / 8.0) * 2.0 ** (e - 7.0))
+    return sign * val
+
+
+def test_expand_weights_is_exact_e4m3_of_codes():
+    rng = np.random.default_rng(4)
+    codes = rng.integers(-7, 8, (300, 1152)).astype(np.int8)
+    codes[0, :16] = np.arange(-7, 9)[:16].clip(-7, 7)
+    Wq = torch.from_numpy(oracle.pack_int4(codes)).to(DEV)
+    We = clq.expand_weights(Wq)
+    torch.cuda.synchronize()
+    assert We.shape == (300, 1152)
+    assert np.array_equal(_decode_e4m3(We.cpu().numpy()), codes.astype(np.float64))
+
+
 def _gemm_case(M, N, K, b, dtype, seed, bias=True):
     x_t, x32 = _inputs(M, K, dtype, seed)
     rng = np.random.default_rng(seed + 1)
@@ -189,15 +211,20 @@ def _gemm_case(M, N, K, b, dtype, seed, bias=True):
     oWq, os_w, _, _ = oracle.prepare_weights(w_t.float().numpy(), perm, b)
     b32 = None if bias_t is None else bias_t.float().numpy()
     y64, acc = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, b32)
-    Y, gacc = clq.w4a4_linear(torch.from_numpy(oXq).to(DEV), torch.from_numpy(os_x).to(DEV),
-                              torch.from_numpy(oWq).to(DEV), torch.from_numpy(os_w).to(DEV),
-                              b, None if bias_t is None else bias_t.to(DEV),
-                              out_dtype=TD[dtype], with_acc=True)
-    torch.cuda.synchronize()
-    assert np.array_equal(gacc.cpu().numpy(), acc)
-    y = Y.float().cpu().numpy()
-    check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
-    check_output_frobenius(y, y64)
+    Wq = torch.from_numpy(oWq).to(DEV)
+    outs = []
+    for W in (Wq, clq.expand_weights(Wq)):       # storage and execution layouts
+        Y, gacc = clq.w4a4_linear(torch.from_numpy(oXq).to(DEV), torch.from_numpy(os_x).to(DEV),
+                                  W, torch.from_numpy(os_w).to(DEV),
+                                  b, None if bias_t is None else bias_t.to(DEV),
+                                  out_dtype=TD[dtype], with_acc=True)
+        torch.cuda.synchronize()
+        assert np.array_equal(gacc.cpu().numpy(), acc)
+        y = Y.float().cpu().numpy()
+        check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
+        check_output_frobenius(y, y64)
+        outs.append(Y)
+    assert torch.equal(outs[0], outs[1])
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 1, 32), (3, 17, 64), (17, 64, 128),
@@ -233,11 +260,12 @@ def test_gemm_carrier_exact_at_extremes(K):
     acc = oracle.int_gemm(qx, qw)
     ones_x = torch.ones(M, dtype=torch.float32, device=DEV)
     ones_w = torch.ones(N, dtype=torch.float32, device=DEV)
-    _, gacc = clq.w4a4_linear(torch.from_numpy(Xq).to(DEV), ones_x,
-                              torch.from_numpy(Wq).to(DEV), ones_w, 32,
-                              out_dtype=torch.bfloat16, with_acc=True)
-    torch.cuda.synchronize()
-    assert np.array_equal(gacc.cpu().numpy(), acc)
+    Wd = torch.from_numpy(Wq).to(DEV)
+    for W in (Wd, clq.expand_weights(Wd)):
+        _, gacc = clq.w4a4_linear(torch.from_numpy(Xq).to(DEV), ones_x, W, ones_w, 32,
+                                  out_dtype=torch.bfloat16, with_acc=True)
+        torch.cuda.synchronize()
+        assert np.array_equal(gacc.cpu().numpy(), acc)
 
 
 def test_gemm_random_codes_all_values():
@@ -268,7 +296,7 @@ def _layer_e2e(cfg, li, M, rows=None):
     layer = clq.PreparedLinear.from_weight(d["W"].to(DEV), permd, b, bias=d["bias"].to(DEV))
     X = d["X"].to(DEV)
     Xq, s_x, rot = clq.rotate_quant_act(X, permd, b, with_rot=True)
-    Y = clq.w4a4_linear(Xq, s_x, layer.Wq, layer.s_w, b, layer.bias, out_dtype=X.dtype)
+    Y = clq.w4a4_linear(Xq, s_x, layer.We, layer.s_w, b, layer.bias, out_dtype=X.dtype)
     torch.cuda.synchronize()
     rows = np.arange(M) if rows is None else rows
     p = perm.numpy()
@@ -282,6 +310,9 @@ def _layer_e2e(cfg, li, M, rows=None):
     check_codes(oracle.unpack_int4(Xq.cpu().numpy()[rows]), oc, orot, os_x)
     y64, _ = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, d["bias32"])
     check_output_frobenius(Y.float().cpu().numpy()[rows], y64)
+    Yf = layer(X, fused=True)
+    torch.cuda.synchronize()
+    assert torch.equal(Yf, Y)          # fused = separate kernels, bit for bit
     return d, layer, Y
 
 
@@ -319,6 +350,45 @@ def test_prepared_linear_state_roundtrip(tmp_path):
     layer2 = clq.PreparedLinear.from_state_dict(torch.load(tmp_path / "l.pt"))
     X = d["X"].to(DEV)
     assert torch.equal(layer(X), layer2(X))
+
+
+# ------------------------------------------------------------------- fused --
+@pytest.mark.parametrize("M,N,K,b,dtype", [(1, 16, 64, 32, "f16"), (3, 17, 96, 32, "f16"),
+                                           (200, 300, 1152, 64, "f16"),
+                                           (300, 600, 1152, 128, "bf16"),
+                                           (129, 264, 4608, 256, "f16"),
+                                           (64, 256, 12288, 128, "bf16"),
+                                           (40, 128, 16384, 64, "f16")])
+def test_fused_matches_separate_and_oracle(M, N, K, b, dtype):
+    x_t, x32 = _inputs(M, K, dtype, seed=M + K)
+    rng = np.random.default_rng(K)
+    w_t = torch.from_numpy((rng.standard_normal((N, K)) * 0.02).astype(np.float32)).to(TD[dtype])
+    bias_t = torch.from_numpy((rng.standard_normal(N) * 0.01).astype(np.float32)).to(TD[dtype])
+    perm = torch.from_numpy(_perm(K, "random", M))
+    layer = clq.PreparedLinear.from_weight(w_t.to(DEV), perm.to(DEV), b, bias=bias_t.to(DEV))
+    X = x_t.to(DEV)
+    Y_sep = layer(X)
+    ws = clq.fused_workspace(M, K, DEV)
+    for W in (layer.We, layer.Wq):
+        Y_f = clq.fused_linear(X, layer.perm, b, W, layer.s_w, layer.bias, workspace=ws)
+        torch.cuda.synchronize()
+        assert torch.equal(Y_f, Y_sep)
+    Y_again = clq.fused_linear(X, layer.perm, b, layer.We, layer.s_w, layer.bias, workspace=ws)
+    assert torch.equal(Y_again, Y_sep)   # workspace reuse
+    oWq, os_w, _, _ = oracle.prepare_weights(w_t.float().numpy(), perm.numpy(), b)
+    y64 = oracle.fused_linear(x32, perm.numpy(), b, oWq, os_w, bias_t.float().numpy())
+    check_output_frobenius(Y_sep.float().cpu().numpy(), y64)
+
+
+def test_fused_small_workspace_rejected():
+    X = torch.zeros((8, 64), dtype=torch.float16, device=DEV)
+    perm = torch.arange(64, dtype=torch.int32, device=DEV)
+    W = torch.zeros((16, 32), dtype=torch.uint8, device=DEV)
+    s_w = torch.ones(16, device=DEV)
+    small = torch.empty(64, dtype=torch.uint8, device=DEV)
+    with pytest.raises(clq.ClqError) as e:
+        clq.fused_linear(X, perm, 32, W, s_w, workspace=small)
+    assert e.value.status == 1
 
 
 # ------------------------------------------------------- failure handling --
