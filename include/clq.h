@@ -58,6 +58,8 @@ typedef int32_t clq_status;
 #define CLQ_ERR_CUDA 5        /* a CUDA runtime call failed                */
 #define CLQ_ERR_TIMEOUT 6     /* a bounded device-side wait ran out        */
 #define CLQ_ERR_DEVICE_INDEX 7 /* perm held an index outside [0, K)        */
+#define CLQ_ERR_SCRATCH_LIMIT 8 /* problem needs more than the static     */
+                                /* scratch of clq_fused_linear_noalloc     */
 
 typedef int32_t clq_dtype;
 #define CLQ_F16 0
@@ -177,6 +179,35 @@ clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M,
                             const float* s_w, const void* bias, int32_t N,
                             void* Y, void* workspace, size_t workspace_bytes,
                             void* stream);
+
+/*
+ * Scratch-free variant of clq_fused_linear.  The paper has no counterpart;
+ * this entry point exists for callers that cannot allocate device memory
+ * where they run the layer: plugin enqueue hooks of inference engines,
+ * serving loops that forbid allocation once started, code that holds no
+ * allocator.  It takes no workspace.  Instead it uses one scratch array of
+ * CLQ_NOALLOC_SCRATCH_BYTES bytes that the library defines in static device
+ * memory; every GPU that loads the library holds that array until the
+ * process exits.  The call allocates and frees nothing and otherwise behaves
+ * exactly like clq_fused_linear (same arguments minus the workspace, same
+ * results).
+ *  - Problems whose clq_fused_linear_workspace_size(M, K) exceeds
+ *    CLQ_NOALLOC_SCRATCH_BYTES are rejected with CLQ_ERR_SCRATCH_LIMIT and
+ *    nothing is launched.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress); make that first call before any stream capture.
+ *  - All calls on a device share the one array.  Each call resets the
+ *    counters it needs before its kernel runs, but leaves the codes of the
+ *    previous call in place; calls whose kernels may overlap on the GPU
+ *    (unordered streams) race on the array and must not be issued.
+ */
+#define CLQ_NOALLOC_SCRATCH_BYTES (64u << 20) /* 64 MiB */
+clq_status clq_fused_linear_noalloc(const void* X, clq_dtype dtype, int32_t M,
+                                    int32_t K, int32_t ldx,
+                                    const int32_t* perm, int32_t b,
+                                    const uint8_t* W, clq_wformat w_format,
+                                    const float* s_w, const void* bias,
+                                    int32_t N, void* Y, void* stream);
 
 /*
  * Synchronize `stream`, then read and clear the device status word of the

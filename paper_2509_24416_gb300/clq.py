@@ -23,12 +23,14 @@ CLQ_F16, CLQ_BF16 = 0, 1
 CLQ_W_INT4_PACKED, CLQ_W_E4M3 = 0, 1
 STATUS = {0: "CLQ_OK", 1: "CLQ_ERR_INVALID_ARG", 2: "CLQ_ERR_SHAPE",
           3: "CLQ_ERR_ALIGN", 4: "CLQ_ERR_UNSUPPORTED", 5: "CLQ_ERR_CUDA",
-          6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX"}
+          6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX",
+          8: "CLQ_ERR_SCRATCH_LIMIT"}
 EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_build_permutation", "clq_prepare_weights",
            "clq_rotate_quant_act", "clq_expand_weights", "clq_w4a4_linear",
            "clq_fused_linear_workspace_size", "clq_fused_linear",
-           "clq_get_device_status", "clq_selftest_bounded_wait")
+           "clq_fused_linear_noalloc", "clq_get_device_status",
+           "clq_selftest_bounded_wait")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -49,6 +51,8 @@ _SIGS = {
     "clq_fused_linear_workspace_size": (_Z, [_I, _I]),
     "clq_fused_linear": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I, _P, _P, _I,
                               _P, _P, _Z, _P]),
+    "clq_fused_linear_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I, _P,
+                                      _P, _I, _P, _P]),
     "clq_get_device_status": (_I, [_P, _P]),
     "clq_selftest_bounded_wait": (_I, [ctypes.c_int64, _P]),
 }
@@ -124,6 +128,12 @@ def clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N,
     return load().clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format,
                                    s_w, bias, N, Y, workspace,
                                    workspace_bytes, stream)
+
+
+def clq_fused_linear_noalloc(X, dtype, M, K, ldx, perm, b, W, w_format, s_w,
+                             bias, N, Y, stream):
+    return load().clq_fused_linear_noalloc(X, dtype, M, K, ldx, perm, b, W,
+                                           w_format, s_w, bias, N, Y, stream)
 
 
 def clq_get_device_status(stream, out):

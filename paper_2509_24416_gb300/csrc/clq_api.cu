@@ -150,6 +150,9 @@ const char* clq_status_string(clq_status s) {
     case CLQ_ERR_CUDA: return "CLQ_ERR_CUDA: a CUDA runtime call failed";
     case CLQ_ERR_TIMEOUT: return "CLQ_ERR_TIMEOUT: a bounded device-side wait ran out";
     case CLQ_ERR_DEVICE_INDEX: return "CLQ_ERR_DEVICE_INDEX: perm index outside [0, K)";
+    case CLQ_ERR_SCRATCH_LIMIT:
+      return "CLQ_ERR_SCRATCH_LIMIT: M x K needs more than the static scratch of "
+             "clq_fused_linear_noalloc";
     default: return "unknown clq_status";
   }
 }
