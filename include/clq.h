@@ -65,11 +65,22 @@ typedef int32_t clq_dtype;
 #define CLQ_F16 0
 #define CLQ_BF16 1
 
-/* Layout of the prepared weight codes handed to the GEMM calls. */
-typedef int32_t clq_wformat;
-#define CLQ_W_INT4_PACKED 0 /* [N][K/2] bytes, two codes per byte (storage)   */
-#define CLQ_W_E4M3 1        /* [N][K] bytes, each code as its exact E4M3      */
-                            /* value (execution layout, clq_expand_weights)   */
+/*
+ * Layout of an array of INT4 codes (activations or weights), `rows` x K:
+ *  CLQ_CODES_INT4_PACKED  [rows][K/2] bytes, two codes per byte (code 2j in
+ *                         the low nibble), 4-bit two's complement; the
+ *                         storage format.
+ *  CLQ_CODES_E4M3         [rows][K] bytes, one code per byte holding the
+ *                         code's exact E4M3 encoding (every integer in
+ *                         [-7, 7] is an E4M3 value); the execution layout the
+ *                         tensor-core GEMM loads with TMA directly, without
+ *                         expanding nibbles in every CTA.
+ * The codes are the same INT4 values in both layouts and every call gives
+ * identical results for either.
+ */
+typedef int32_t clq_codes;
+#define CLQ_CODES_INT4_PACKED 0
+#define CLQ_CODES_E4M3 1
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char* clq_status_string(clq_status status);
@@ -118,22 +129,22 @@ clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N,
  * Sec. 3.3's online fast Hadamard): X~ = X_p H in fp32, s_x[i] =
  * max_k |X~[i][k]| / 7, Xq[i] = pack(clamp(rint(X~[i] / s_x[i]), -7, 7)).
  * One HBM pass over X.  X: device [M][ldx] of `dtype`.  perm: device int32
- * [K].  Xq: device uint8 [M][K/2].  s_x: device fp32 [M].  x_rot_dbg: device
- * fp32 [M][K] or NULL (receives X~).
+ * [K].  Xq: device uint8 codes in layout `x_codes` ([M][K/2] packed or
+ * [M][K] E4M3).  s_x: device fp32 [M].  x_rot_dbg: device fp32 [M][K] or
+ * NULL (receives X~).
  */
 clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M,
                                 int32_t K, int32_t ldx, const int32_t* perm,
-                                int32_t b, uint8_t* Xq, float* s_x,
-                                float* x_rot_dbg, void* stream);
+                                int32_t b, clq_codes x_codes, uint8_t* Xq,
+                                float* s_x, float* x_rot_dbg, void* stream);
 
 /*
- * Execution layout of prepared weights: every packed INT4 code of Wq
- * [N][K/2] becomes one byte of We [N][K] holding the code's exact E4M3
- * encoding (every integer in [-7, 7] is an E4M3 value).  The codes are
- * unchanged; only the container widens to 8 bits, so the GEMM can load
- * weight tiles with TMA straight into the tensor-core operand layout instead
- * of expanding nibbles in every CTA.  Offline, once per layer.  Wq: device
- * [N][K/2]; We: device [N][K].  Requires N >= 0, K % 32 == 0, K <= 16384.
+ * Packed INT4 codes [N][K/2] (CLQ_CODES_INT4_PACKED) -> the E4M3 execution
+ * layout [N][K] (CLQ_CODES_E4M3).  The codes are unchanged; only the
+ * container widens to 8 bits.  Used offline, once per layer, on the weights
+ * (weights are static, so expanding them in every CTA of every call would
+ * only repeat work).  Wq: device [N][K/2]; We: device [N][K].  Requires
+ * N >= 0, K % 32 == 0, K <= 16384.
  */
 clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K,
                               uint8_t* We, void* stream);
@@ -141,23 +152,23 @@ clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K,
 /*
  * INT4 x INT4 product with the dequant + bias epilogue:
  * Y[i][n] = out_dtype(acc[i][n] * s_x[i] * s_w[n] / b + bias[n]).
- * Xq: device uint8 [M][K/2] packed activation codes; s_x: device fp32 [M];
- * W: device weight codes in layout `w_format` (CLQ_W_INT4_PACKED: [N][K/2],
- * CLQ_W_E4M3: [N][K]); s_w: device fp32 [N]; bias: device [N] of
+ * Xq: device activation codes in layout `x_codes` ([M][K/2] or [M][K]);
+ * s_x: device fp32 [M]; W: device weight codes in layout `w_codes`
+ * ([N][K/2] or [N][K]); s_w: device fp32 [N]; bias: device [N] of
  * `out_dtype` or NULL; Y: device [M][N] of `out_dtype`.  acc_dbg: device
  * int32 [M][N] or NULL; when given it receives the exact integer
- * accumulators.  Both weight layouts give identical results.
+ * accumulators.  All four layout combinations give identical results.
  */
-clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x,
-                           const uint8_t* W, clq_wformat w_format,
-                           const float* s_w, const void* bias, int32_t M,
-                           int32_t N, int32_t K, int32_t b,
-                           clq_dtype out_dtype, void* Y, int32_t* acc_dbg,
-                           void* stream);
+clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes,
+                           const float* s_x, const uint8_t* W,
+                           clq_codes w_codes, const float* s_w,
+                           const void* bias, int32_t M, int32_t N, int32_t K,
+                           int32_t b, clq_dtype out_dtype, void* Y,
+                           int32_t* acc_dbg, void* stream);
 
 /*
  * Bytes of device workspace clq_fused_linear needs for M tokens of K
- * channels (activation codes, scales and per-tile readiness counters).
+ * channels (E4M3 activation codes, scales and per-tile readiness counters).
  */
 size_t clq_fused_linear_workspace_size(int32_t M, int32_t K);
 
@@ -168,14 +179,14 @@ size_t clq_fused_linear_workspace_size(int32_t M, int32_t K);
  * starts as soon as the rows of its token block are published.  Same
  * arithmetic and results as clq_rotate_quant_act followed by
  * clq_w4a4_linear.  X: device [M][ldx] of `dtype`; Y: device [M][N] of
- * `dtype`; bias: device [N] of `dtype` or NULL; W / w_format as for
+ * `dtype`; bias: device [N] of `dtype` or NULL; W / w_codes as for
  * clq_w4a4_linear; workspace: device, 256-byte aligned, at least
  * clq_fused_linear_workspace_size(M, K) bytes, owned by the caller and
  * overwritten by the call.
  */
 clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M,
                             int32_t K, int32_t ldx, const int32_t* perm,
-                            int32_t b, const uint8_t* W, clq_wformat w_format,
+                            int32_t b, const uint8_t* W, clq_codes w_codes,
                             const float* s_w, const void* bias, int32_t N,
                             void* Y, void* workspace, size_t workspace_bytes,
                             void* stream);
@@ -205,7 +216,7 @@ clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M,
 clq_status clq_fused_linear_noalloc(const void* X, clq_dtype dtype, int32_t M,
                                     int32_t K, int32_t ldx,
                                     const int32_t* perm, int32_t b,
-                                    const uint8_t* W, clq_wformat w_format,
+                                    const uint8_t* W, clq_codes w_codes,
                                     const float* s_w, const void* bias,
                                     int32_t N, void* Y, void* stream);
 

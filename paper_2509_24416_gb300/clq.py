@@ -20,7 +20,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libclq.so")
 
 CLQ_F16, CLQ_BF16 = 0, 1
-CLQ_W_INT4_PACKED, CLQ_W_E4M3 = 0, 1
+CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3 = 0, 1
 STATUS = {0: "CLQ_OK", 1: "CLQ_ERR_INVALID_ARG", 2: "CLQ_ERR_SHAPE",
           3: "CLQ_ERR_ALIGN", 4: "CLQ_ERR_UNSUPPORTED", 5: "CLQ_ERR_CUDA",
           6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX",
@@ -43,11 +43,11 @@ _SIGS = {
     "clq_build_permutation": (_I, [_P, _I, _P]),
     "clq_prepare_weights": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P,
                                  _P]),
-    "clq_rotate_quant_act": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P,
+    "clq_rotate_quant_act": (_I, [_P, _I, _I, _I, _I, _P, _I, _I, _P, _P, _P,
                                   _P]),
     "clq_expand_weights": (_I, [_P, _I, _I, _P, _P]),
-    "clq_w4a4_linear": (_I, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P,
-                             _P, _P]),
+    "clq_w4a4_linear": (_I, [_P, _I, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I,
+                             _P, _P, _P]),
     "clq_fused_linear_workspace_size": (_Z, [_I, _I]),
     "clq_fused_linear": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I, _P, _P, _I,
                               _P, _P, _Z, _P]),
@@ -103,37 +103,37 @@ def clq_prepare_weights(W, dtype, N, K, ldw, perm, b, clip, Wq, s_w,
                                       s_w, w_rot_dbg, stream)
 
 
-def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, Xq, s_x, x_rot_dbg,
-                         stream):
-    return load().clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, Xq, s_x,
-                                       x_rot_dbg, stream)
+def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, x_codes, Xq, s_x,
+                         x_rot_dbg, stream):
+    return load().clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, x_codes,
+                                       Xq, s_x, x_rot_dbg, stream)
 
 
 def clq_expand_weights(Wq, N, K, We, stream):
     return load().clq_expand_weights(Wq, N, K, We, stream)
 
 
-def clq_w4a4_linear(Xq, s_x, W, w_format, s_w, bias, M, N, K, b, out_dtype,
-                    Y, acc_dbg, stream):
-    return load().clq_w4a4_linear(Xq, s_x, W, w_format, s_w, bias, M, N, K,
-                                  b, out_dtype, Y, acc_dbg, stream)
+def clq_w4a4_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b,
+                    out_dtype, Y, acc_dbg, stream):
+    return load().clq_w4a4_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M,
+                                  N, K, b, out_dtype, Y, acc_dbg, stream)
 
 
 def clq_fused_linear_workspace_size(M, K):
     return load().clq_fused_linear_workspace_size(M, K)
 
 
-def clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N,
+def clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w, bias, N,
                      Y, workspace, workspace_bytes, stream):
-    return load().clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format,
+    return load().clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_codes,
                                    s_w, bias, N, Y, workspace,
                                    workspace_bytes, stream)
 
 
-def clq_fused_linear_noalloc(X, dtype, M, K, ldx, perm, b, W, w_format, s_w,
+def clq_fused_linear_noalloc(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w,
                              bias, N, Y, stream):
     return load().clq_fused_linear_noalloc(X, dtype, M, K, ldx, perm, b, W,
-                                           w_format, s_w, bias, N, Y, stream)
+                                           w_codes, s_w, bias, N, Y, stream)
 
 
 def clq_get_device_status(stream, out):
@@ -208,21 +208,24 @@ def prepare_weights(W, perm, b, clip=None, with_rot=False, stream=None):
     return (Wq, s_w, rot) if with_rot else (Wq, s_w)
 
 
-def rotate_quant_act(X, perm, b, Xq=None, s_x=None, with_rot=False,
-                     stream=None):
-    """X [M, K] -> (Xq uint8 [M, K/2], s_x fp32 [M][, x_rot fp32 [M, K]])."""
+def rotate_quant_act(X, perm, b, codes=CLQ_CODES_INT4_PACKED, Xq=None, s_x=None,
+                     with_rot=False, stream=None):
+    """X [M, K] -> (Xq uint8, s_x fp32 [M][, x_rot fp32 [M, K]]); Xq is
+    [M, K/2] packed (CLQ_CODES_INT4_PACKED) or [M, K] E4M3 (CLQ_CODES_E4M3)."""
     _row_major(X, "X")
     M, K = X.shape
     dev = X.device
     if Xq is None:
-        Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+        width = K if codes == CLQ_CODES_E4M3 else K // 2
+        Xq = torch.empty((M, width), dtype=torch.uint8, device=dev)
     if s_x is None:
         s_x = torch.empty(M, dtype=torch.float32, device=dev)
     rot = (torch.empty((M, K), dtype=torch.float32, device=dev)
            if with_rot else None)
     _check(clq_rotate_quant_act(_ptr(X), _dt(X), M, K, X.stride(0),
-                                _ptr(perm), b, _ptr(Xq), _ptr(s_x), _ptr(rot),
-                                _stream(stream)), "clq_rotate_quant_act")
+                                _ptr(perm), b, codes, _ptr(Xq), _ptr(s_x),
+                                _ptr(rot), _stream(stream)),
+           "clq_rotate_quant_act")
     return (Xq, s_x, rot) if with_rot else (Xq, s_x)
 
 
@@ -235,30 +238,31 @@ def expand_weights(Wq, stream=None):
     return We
 
 
-def _wformat(W, K):
-    if W.shape[1] == K:
-        return CLQ_W_E4M3
-    if 2 * W.shape[1] == K:
-        return CLQ_W_INT4_PACKED
-    raise ValueError("weights must be [N, K/2] packed or [N, K] E4M3")
+def codes_layout(t, K):
+    """Layout of a code array of K codes per row, from its width."""
+    if t.shape[1] == K:
+        return CLQ_CODES_E4M3
+    if 2 * t.shape[1] == K:
+        return CLQ_CODES_INT4_PACKED
+    raise ValueError("codes must be [rows, K/2] packed or [rows, K] E4M3")
 
 
-def w4a4_linear(Xq, s_x, W, s_w, b, bias=None, out_dtype=torch.float16,
+def w4a4_linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
                 Y=None, with_acc=False, stream=None):
-    """Packed activation codes x weight codes (packed [N, K/2] or E4M3
-    [N, K]) -> Y [M, N] (out_dtype)[, acc int32 [M, N]]."""
-    M, Kh = Xq.shape
+    """Activation codes x weight codes (each packed [rows, K/2] or E4M3
+    [rows, K]) -> Y [M, N] (out_dtype)[, acc int32 [M, N]]."""
+    M = Xq.shape[0]
     N = W.shape[0]
-    K = 2 * Kh
     if Y is None:
         Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
     acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
            if with_acc else None)
     if bias is not None and bias.dtype != Y.dtype:
         raise TypeError("bias must have the output dtype")
-    _check(clq_w4a4_linear(_ptr(Xq), _ptr(s_x), _ptr(W), _wformat(W, K),
-                           _ptr(s_w), _ptr(bias), M, N, K, b, _dt(Y), _ptr(Y),
-                           _ptr(acc), _stream(stream)), "clq_w4a4_linear")
+    _check(clq_w4a4_linear(_ptr(Xq), codes_layout(Xq, K), _ptr(s_x), _ptr(W),
+                           codes_layout(W, K), _ptr(s_w), _ptr(bias), M, N, K,
+                           b, _dt(Y), _ptr(Y), _ptr(acc), _stream(stream)),
+           "clq_w4a4_linear")
     return (Y, acc) if with_acc else Y
 
 
@@ -280,7 +284,7 @@ def fused_linear(X, perm, b, W, s_w, bias=None, Y=None, workspace=None,
     if workspace is None:
         workspace = fused_workspace(M, K, X.device)
     _check(clq_fused_linear(_ptr(X), _dt(X), M, K, X.stride(0), _ptr(perm), b,
-                            _ptr(W), _wformat(W, K), _ptr(s_w), _ptr(bias), N,
+                            _ptr(W), codes_layout(W, K), _ptr(s_w), _ptr(bias), N,
                             _ptr(Y), _ptr(workspace), workspace.numel(),
                             _stream(stream)), "clq_fused_linear")
     return Y
@@ -305,6 +309,8 @@ class PreparedLinear:
 
     Wq holds the packed INT4 codes (the storage format, 4 bits per weight);
     We the same codes in the E4M3 execution layout the GEMM loads directly.
+    Activation codes are produced in the E4M3 layout too (they are transient,
+    so their container is chosen for the GEMM).
     ``state_dict()`` keeps only the packed codes; ``from_state_dict()``
     expands them again.  Calling the object runs the separate rotate-quant
     and GEMM kernels (``fused=False``) or the fused kernel.
@@ -335,6 +341,7 @@ class PreparedLinear:
         if fused:
             return fused_linear(X, self.perm, self.b, self.We, self.s_w,
                                 self.bias, workspace=workspace, stream=stream)
-        Xq, s_x = rotate_quant_act(X, self.perm, self.b, stream=stream)
-        return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, self.bias,
-                           out_dtype=X.dtype, stream=stream)
+        Xq, s_x = rotate_quant_act(X, self.perm, self.b, CLQ_CODES_E4M3,
+                                   stream=stream)
+        return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, X.shape[1],
+                           self.bias, out_dtype=X.dtype, stream=stream)

@@ -70,11 +70,11 @@ clq_status check_k_b(int K, int b) {
 
 bool valid_dtype(int d) { return d == CLQ_F16 || d == CLQ_BF16; }
 
-bool valid_wformat(int f) { return f == CLQ_W_INT4_PACKED || f == CLQ_W_E4M3; }
+bool valid_codes(int f) { return f == CLQ_CODES_INT4_PACKED || f == CLQ_CODES_E4M3; }
 
 // Launch of the fused kernel on a workspace laid out as `ws` (validated).
 clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
-                        const int32_t* perm, int32_t b, const uint8_t* W, clq_wformat w_format,
+                        const int32_t* perm, int32_t b, const uint8_t* W, clq_codes w_codes,
                         const float* s_w, const void* bias, int32_t N, void* Y, uint8_t* wsp,
                         const clq::FusedWorkspace& ws, int32_t* status, void* stream) {
   clq::RotateQuantArgs rq{};
@@ -99,15 +99,15 @@ clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, in
   g.K = K;
   g.inv_b = 1.0f / static_cast<float>(b);
   g.status = status;
-  return from_cuda(clq::launch_fused_linear(rq, W, w_format, g, log2i(b), dtype,
+  return from_cuda(clq::launch_fused_linear(rq, W, w_codes, g, log2i(b), dtype,
                                             reinterpret_cast<uint32_t*>(wsp + ws.ready_off),
                                             static_cast<cudaStream_t>(stream)));
 }
 
 clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ld,
-                               const int32_t* perm, int32_t b, const float* clip, uint8_t* Q,
-                               float* S, float* rot, void* stream) {
-  if (!valid_dtype(dtype) || M < 0) return CLQ_ERR_INVALID_ARG;
+                               const int32_t* perm, int32_t b, const float* clip, int codes,
+                               uint8_t* Q, float* S, float* rot, void* stream) {
+  if (!valid_dtype(dtype) || !valid_codes(codes) || M < 0) return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
   if (ld < K) return CLQ_ERR_SHAPE;
@@ -132,6 +132,7 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   a.rot = rot;
   a.status = status;
   a.logb = log2i(b);
+  a.e4m3 = codes == CLQ_CODES_E4M3 ? 1 : 0;
   return from_cuda(
       clq::launch_rotate_quant(a, dtype, log2i(b), static_cast<cudaStream_t>(stream)));
 }
@@ -194,13 +195,15 @@ clq_status clq_outlier_scores(const void* calib, clq_dtype dtype, int32_t B, int
 clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N, int32_t K, int32_t ldw,
                                const int32_t* perm, int32_t b, const float* clip, uint8_t* Wq,
                                float* s_w, float* w_rot_dbg, void* stream) {
-  return rotate_quant_common(W, dtype, N, K, ldw, perm, b, clip, Wq, s_w, w_rot_dbg, stream);
+  return rotate_quant_common(W, dtype, N, K, ldw, perm, b, clip, CLQ_CODES_INT4_PACKED, Wq, s_w,
+                             w_rot_dbg, stream);
 }
 
 clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
-                                const int32_t* perm, int32_t b, uint8_t* Xq, float* s_x,
-                                float* x_rot_dbg, void* stream) {
-  return rotate_quant_common(X, dtype, M, K, ldx, perm, b, nullptr, Xq, s_x, x_rot_dbg, stream);
+                                const int32_t* perm, int32_t b, clq_codes x_codes, uint8_t* Xq,
+                                float* s_x, float* x_rot_dbg, void* stream) {
+  return rotate_quant_common(X, dtype, M, K, ldx, perm, b, nullptr, x_codes, Xq, s_x, x_rot_dbg,
+                             stream);
 }
 
 clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K, uint8_t* We,
@@ -216,11 +219,12 @@ clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K, uint8_t* 
   return from_cuda(clq::launch_expand_weights(Wq, N, K, We, static_cast<cudaStream_t>(stream)));
 }
 
-clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x, const uint8_t* W,
-                           clq_wformat w_format, const float* s_w, const void* bias, int32_t M,
-                           int32_t N, int32_t K, int32_t b, clq_dtype out_dtype, void* Y,
-                           int32_t* acc_dbg, void* stream) {
-  if (!valid_dtype(out_dtype) || !valid_wformat(w_format) || M < 0 || N < 0)
+clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x,
+                           const uint8_t* W, clq_codes w_codes, const float* s_w,
+                           const void* bias, int32_t M, int32_t N, int32_t K, int32_t b,
+                           clq_dtype out_dtype, void* Y, int32_t* acc_dbg, void* stream) {
+  if (!valid_dtype(out_dtype) || !valid_codes(x_codes) || !valid_codes(w_codes) || M < 0 ||
+      N < 0)
     return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
@@ -246,7 +250,8 @@ clq_status clq_w4a4_linear(const uint8_t* Xq, const float* s_x, const uint8_t* W
   g.inv_b = 1.0f / static_cast<float>(b);
   g.status = status;
   return from_cuda(
-      clq::launch_w4a4_gemm(Xq, W, w_format, g, out_dtype, static_cast<cudaStream_t>(stream)));
+      clq::launch_w4a4_gemm(Xq, x_codes, W, w_codes, g, out_dtype,
+                            static_cast<cudaStream_t>(stream)));
 }
 
 size_t clq_fused_linear_workspace_size(int32_t M, int32_t K) {
@@ -256,9 +261,9 @@ size_t clq_fused_linear_workspace_size(int32_t M, int32_t K) {
 
 clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
                             const int32_t* perm, int32_t b, const uint8_t* W,
-                            clq_wformat w_format, const float* s_w, const void* bias, int32_t N,
+                            clq_codes w_codes, const float* s_w, const void* bias, int32_t N,
                             void* Y, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!valid_dtype(dtype) || !valid_wformat(w_format) || M < 0 || N < 0)
+  if (!valid_dtype(dtype) || !valid_codes(w_codes) || M < 0 || N < 0)
     return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
@@ -276,7 +281,7 @@ clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M, int32_t K
   int32_t* status = nullptr;
   st = device_setup(&status);
   if (st != CLQ_OK) return st;
-  return fused_common(X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N, Y,
+  return fused_common(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w, bias, N, Y,
                       static_cast<uint8_t*>(workspace), ws, status, stream);
 }
 

@@ -14,12 +14,13 @@ struct RotateQuantArgs {
   int32_t M, K, ld;
   const int32_t* perm;   // [K]
   const float* clip;     // [M] or null (weights only)
-  uint8_t* Q;            // [M][K/2]
+  uint8_t* Q;            // [M][K/2] packed, or [M][K] E4M3 when e4m3 != 0
   float* S;              // [M]
   float* rot;            // [M][K] or null
   int32_t rows_per_tile; // filled in by the launcher
   int32_t* status;       // device status word
   int32_t logb;          // log2(b)
+  int32_t e4m3;          // codes layout: 0 packed nibbles, 1 one E4M3 byte each
 };
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
@@ -39,9 +40,9 @@ struct GemmArgs {
   int32_t* status;
 };
 
-// A = Xq [M][K/2] packed; B = weights in `w_format` (CLQ_W_INT4_PACKED
-// [N][K/2] or CLQ_W_E4M3 [N][K]); TMA maps are built here from raw pointers.
-cudaError_t launch_w4a4_gemm(const uint8_t* Xq, const uint8_t* W, int w_format,
+// A = activation codes, B = weight codes, each in layout CLQ_CODES_INT4_PACKED
+// ([rows][K/2]) or CLQ_CODES_E4M3 ([rows][K]); TMA maps are built here.
+cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st);
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st);
@@ -54,7 +55,7 @@ FusedWorkspace fused_workspace_layout(int M, int K);
 
 // Fused rotate-quant + GEMM: `rq` describes the activation side (its Q / S
 // point into the workspace), `g` the product (s_x = workspace scales).
-cudaError_t launch_fused_linear(const RotateQuantArgs& rq, const uint8_t* W, int w_format,
+cudaError_t launch_fused_linear(const RotateQuantArgs& rq, const uint8_t* W, int w_codes,
                                 const GemmArgs& g, int logb, int dtype, uint32_t* ready,
                                 cudaStream_t st);
 
@@ -69,6 +70,13 @@ bool encode_tma_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
                       uint64_t rows, uint32_t box_inner, uint32_t box_rows);
 // 2-byte output tile map for the epilogue stores (box 32 columns x 128 rows).
 bool encode_tma_out_tile(CUtensorMap* map, void* Y, int M, int N);
-int sm_count();
+int sm_count();  // cached per device
+// TMA map of an INT4 code array (rows x K) in layout `codes`, box_rows rows.
+bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows, int K,
+                      int box_rows);
+// Raise `func`'s dynamic shared-memory limit to the device maximum once per
+// device, and (per_sm != null) return its occupancy for (threads, smem),
+// cached, so that launches make no per-call attribute queries.
+cudaError_t kernel_setup(const void* func, size_t smem, int threads, int* per_sm);
 
 }  // namespace clq

@@ -10,7 +10,8 @@
 // of token rows (rq::run, all threads) into the caller's workspace and
 // publishes, per 128-token block, how many rows are done (release: proxy
 // fence, __threadfence, atomicAdd).  Then the same CTA turns into a GEMM
-// pipeline (gemm::pipeline); its TMA producer waits (acquire, bounded) until
+// pipeline (gemm::pipeline), with the codes in E4M3 so that TMA loads them
+// straight into the MMA operand layout; its TMA producer waits (acquire, bounded) until
 // all rows of a tile's token block are published before loading that block's
 // codes.  One launch, no host round trip, and the codes stay in L2 for the
 // layer sizes of the paper's models.
@@ -55,7 +56,7 @@ __global__ void __launch_bounds__(FT, 1)
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  setup<BPACK>(&bars);
+  setup<false, BPACK>(&bars);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -65,7 +66,7 @@ __global__ void __launch_bounds__(FT, 1)
   __syncthreads();
 
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
-  pipeline<T, BPACK>(maps, g, smem, &bars, tmem, ready);
+  pipeline<T, false, BPACK>(maps, g, smem, &bars, tmem, ready);
   tc_fence_before();
   __syncthreads();
   teardown(tmem);
@@ -77,8 +78,7 @@ cudaError_t launch_t(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUt
                      int use_tma_store, int rq_stages, size_t smem, int grid, cudaStream_t st) {
   uint32_t* tile_counter = ready + (g.M + BM - 1) / BM;
   auto k = fused_linear_kernel<T, BPACK>;
-  cudaError_t e =
-      cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, FT, nullptr);
   if (e != cudaSuccess) return e;
   k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store,
                              rq_stages);
@@ -93,22 +93,23 @@ FusedWorkspace fused_workspace_layout(int M, int K) {
   FusedWorkspace w{};
   const size_t m = static_cast<size_t>(M < 0 ? 0 : M);
   w.codes_off = 0;
-  w.scales_off = align256(m * static_cast<size_t>(K / 2));
+  w.scales_off = align256(m * static_cast<size_t>(K));  // E4M3 codes
   w.ready_off = align256(w.scales_off + 4 * m);
   w.bytes = align256(w.ready_off + 4 * ((m + BM - 1) / BM + 1));  // + tile counter
   return w;
 }
 
-cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, int w_format,
+cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, int w_codes,
                                 const GemmArgs& g, int logb, int dtype, uint32_t* ready,
                                 cudaStream_t st) {
-  const bool bpack = w_format == CLQ_W_INT4_PACKED;
-  const size_t gemm_bytes = bpack ? Cfg<true>::BYTES : Cfg<false>::BYTES;
+  const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
+  const size_t gemm_bytes = bpack ? Cfg<false, true>::BYTES : Cfg<false, false>::BYTES;
   const size_t limit = 227u * 1024u - 2048u;  // dynamic + static shared memory
   // Rotate-quant phase: as many rows per tile as 512 threads cover, then as
   // many raw stages (2..4) as fit next to them.
   RotateQuantArgs rq = rq_in;
   rq.logb = logb;
+  rq.e4m3 = 1;  // the workspace holds the codes in the GEMM's operand layout
   const int segs = rq.K / 32;
   int R = std::max(1, FT / segs);
   int stages = rq::kMaxStages;
@@ -124,17 +125,9 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   if (e != cudaSuccess) return e;
 
   CUtensorMap mapA, mapB, mapY;
-  const uint64_t kb = static_cast<uint64_t>(g.K) / 2;
-  if (!encode_tma_2d_u8(&mapA, rq.Q, kb, static_cast<uint64_t>(g.M), BKP, BM))
+  if (!encode_codes_map(&mapA, rq.Q, CLQ_CODES_E4M3, g.M, g.K, BM) ||
+      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, BN))
     return cudaErrorInvalidValue;
-  if (bpack) {
-    if (!encode_tma_2d_u8(&mapB, W, kb, static_cast<uint64_t>(g.N), BKP, BN))
-      return cudaErrorInvalidValue;
-  } else {
-    if (!encode_tma_2d(&mapB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, W, static_cast<uint64_t>(g.K),
-                       static_cast<uint64_t>(g.N), BK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
-      return cudaErrorInvalidValue;
-  }
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
   if (use_tma_store) {
     if (!encode_tma_out_tile(&mapY, g.Y, g.M, g.N)) return cudaErrorInvalidValue;

@@ -45,7 +45,7 @@ clq_status scratch_address(void** out) {
 extern "C" clq_status clq_fused_linear_noalloc(const void* X, clq_dtype dtype, int32_t M,
                                                int32_t K, int32_t ldx, const int32_t* perm,
                                                int32_t b, const uint8_t* W,
-                                               clq_wformat w_format, const float* s_w,
+                                               clq_codes w_codes, const float* s_w,
                                                const void* bias, int32_t N, void* Y,
                                                void* stream) {
   if (M > 0 && K >= 32 && K <= 16384 && K % 32 == 0 &&
@@ -58,6 +58,6 @@ extern "C" clq_status clq_fused_linear_noalloc(const void* X, clq_dtype dtype, i
   }
   // The forwarded call validates every other argument, clears the counters
   // it needs in the scratch array and launches on `stream`.
-  return clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N, Y, scratch,
+  return clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w, bias, N, Y, scratch,
                           CLQ_NOALLOC_SCRATCH_BYTES, stream);
 }

@@ -17,7 +17,9 @@ constexpr int B_U = BN * BK;      // 32 KB unpacked B stage
 constexpr int A_P = BM * BKP;     // 8 KB packed A stage
 constexpr int B_P = BN * BKP;     // 16 KB packed B stage
 constexpr int EPI_COLS = 32;      // output columns per epilogue store
-constexpr int EPI_BYTES = BM * EPI_COLS * 2;  // 8 KB staging buffer
+constexpr int EPI_ROWS = 32;      // rows per store: one warp's TMEM lanes
+constexpr int EPI_BYTES = EPI_ROWS * EPI_COLS * 2;  // 2 KB staging buffer
+constexpr int EPI_TOTAL = 4 * 2 * EPI_BYTES;        // 4 warps x 2 buffers
 constexpr int TMEM_COLS = 512;    // two 128 x 256 fp32 accumulators
 constexpr uint32_t kEpiBarrier = 1;  // named barrier id of the epilogue warps
 
@@ -115,21 +117,23 @@ __device__ __forceinline__ void bulk_wait_all() {
   asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
-// Epilogue of one 128 x 256 tile by 128 threads (four warps, any warp order:
-// warp w reads TMEM lanes 32 * (w % 4) ..).  y = acc * s_x[row] * s_w[col] /
-// b + bias[col], rounded to OutT.  With a TMA map for Y, each 128 x 32 block
-// goes through a 64-byte-swizzled staging buffer and one bulk tensor store;
-// otherwise (N not a multiple of 8) threads store their row directly.
-// `store_count` numbers the staging buffers used so far (alternating).
+// Epilogue of one 128 x 256 tile: each of four warps drains its own 32 TMEM
+// lanes (rows) independently.  y = acc * s_x[row] * s_w[col] / b +
+// bias[col], rounded to OutT; col_scale / col_bias hold s_w / b and bias for
+// the tile's columns.  With a TMA map for Y, each 32 x 32 block goes through
+// the warp's own 64-byte-swizzled staging buffer (two, alternating) and one
+// bulk tensor store issued by lane 0; otherwise (N not a multiple of 8) lanes
+// store their row directly.  `store_count` counts this warp's stores.
 template <typename OutT>
-__device__ __forceinline__ void epilogue_tile(uint32_t tmem_acc, int warp_q, int et, int m0,
+__device__ __forceinline__ void epilogue_tile(uint32_t tmem_acc, int warp_q, int lane, int m0,
                                               int n0, int M, int N, float sx,
                                               const float* col_scale, const float* col_bias,
                                               uint8_t* staging, const CUtensorMap* mapY,
                                               void* Y, int32_t* acc_dbg, int& store_count) {
-  const int row_in_tile = warp_q * 32 + (et & 31);
+  const int row_in_tile = warp_q * 32 + lane;
   const int row = m0 + row_in_tile;
   const uint32_t lane_base = tmem_acc + (static_cast<uint32_t>(warp_q * 32) << 16);
+  uint8_t* my_staging = staging + warp_q * 2 * EPI_BYTES;
 #pragma unroll 1
   for (int c = 0; c < BN; c += EPI_COLS) {
     if (n0 + c >= N) break;
@@ -158,19 +162,19 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tmem_acc, int warp_q, int
         if (n0 + c + j < N) arow[j] = __float2int_rn(__uint_as_float(r[j]));
     }
     if (mapY != nullptr) {
-      uint8_t* sb = staging + (store_count & 1) * EPI_BYTES;
-      if (et == 0) bulk_wait_read<1>();
-      named_bar_sync(kEpiBarrier, 128);
-      uint8_t* srow = sb + row_in_tile * 64;
-      const int sw = (row_in_tile >> 1) & 3;
+      uint8_t* sb = my_staging + (store_count & 1) * EPI_BYTES;
+      if (lane == 0) bulk_wait_read<1>();  // the store that used sb is done reading
+      __syncwarp();
+      uint8_t* srow = sb + lane * 64;
+      const int sw = (lane >> 1) & 3;
 #pragma unroll
       for (int q = 0; q < 4; ++q)
         *reinterpret_cast<uint4*>(srow + ((q ^ sw) << 4)) =
             make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
       fence_proxy_async_smem();
-      named_bar_sync(kEpiBarrier, 128);
-      if (et == 0) {
-        tma_store_2d(mapY, sb, n0 + c, m0);
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(mapY, sb, n0 + c, m0 + warp_q * 32);
         bulk_commit();
       }
       ++store_count;

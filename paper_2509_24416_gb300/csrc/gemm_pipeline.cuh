@@ -1,5 +1,5 @@
-// Warp-specialized tcgen05 GEMM pipeline for the packed INT4 activations x
-// INT4 weights product, shared by the standalone GEMM and the fused kernel.
+// Warp-specialized tcgen05 GEMM pipeline for the INT4 activation x INT4
+// weight product, shared by the standalone GEMM and the fused kernel.
 //
 // acc[i][n] = sum_k qx[i][k] * qw[n][k] is an exact integer: |q| <= 7, so
 // every product is an integer of magnitude <= 49 and, for K <= 16384, every
@@ -10,18 +10,18 @@
 // (checked bit for bit against the int64 oracle, +-7 codes at K = 16384).
 //
 // Persistent: one CTA per SM walks 128 (M) x 256 (N) tiles in a static
-// round-robin order, K step 128 codes.  Warp roles:
-//   warp 4       TMA producer: packed A (64 B x 128 rows) into a staging
-//                buffer and B either packed (64 B x 256 rows, BPACK) or as
-//                E4M3 bytes (128 B x 256 rows, 128-byte swizzle) straight
-//                into the MMA operand buffer;
-//   warps 6-13   unpack nibbles to E4M3 bytes in the 128-byte-swizzled
-//                K-major layout the MMA reads (A, and B when BPACK);
+// round-robin order, K step 128 codes.  Each operand arrives either as E4M3
+// bytes, which TMA writes straight into the MMA operand buffer with the
+// 128-byte swizzle, or as packed nibbles (APACK / BPACK), which TMA stages and
+// unpack warps expand into that layout.  Warp roles:
+//   warp 4       TMA producer;
+//   warps 6-13   unpack (only when an operand is packed);
 //   warp 5       one lane issues tcgen05.mma (4 x K=32 per stage) and commits
 //                stage and tile completion;
-//   warps 0-3    epilogue: TMEM -> registers -> scale, bias, round ->
-//                swizzled staging -> TMA tensor store.  Two TMEM accumulators
-//                let the epilogue of tile i overlap the MMAs of tile i + 1.
+//   warps 0-3    epilogue, each warp on its own 32 accumulator rows: TMEM ->
+//                registers -> scale, bias, round -> swizzled staging -> TMA
+//                tensor store.  Two TMEM accumulators let the epilogue of
+//                tile i overlap the MMAs of tile i + 1.
 //   other warps  idle in this phase.
 // With `ready` counters (fused kernel), the producer waits until all rows of
 // a tile's token block have been published before loading its A tiles.
@@ -40,24 +40,26 @@ constexpr int WARP_TMA = 4;
 constexpr int WARP_MMA = 5;
 constexpr int WARP_UNPACK0 = 6;
 constexpr int MIN_THREADS = (WARP_UNPACK0 + NUM_UNPACK / 32) * 32;  // 448
+constexpr int MAX_STAGES = 4;
 
-template <bool BPACK>
+template <bool APACK, bool BPACK>
 struct Cfg {
-  static constexpr int S = BPACK ? 2 : 3;  // pipeline stages
-  static constexpr size_t OFF_UA = 0;
+  static constexpr bool UNPACK = APACK || BPACK;
+  static constexpr int S = (APACK && BPACK) ? 2 : (UNPACK ? 3 : 4);  // pipeline stages
+  static constexpr size_t OFF_UA = 0;                                 // E4M3 operands
   static constexpr size_t OFF_UB = OFF_UA + S * A_U;
-  static constexpr size_t OFF_PA = OFF_UB + S * B_U;
-  static constexpr size_t OFF_PB = OFF_PA + S * A_P;
+  static constexpr size_t OFF_PA = OFF_UB + S * B_U;                  // packed staging
+  static constexpr size_t OFF_PB = OFF_PA + (APACK ? S * A_P : 0);
   static constexpr size_t OFF_EPI = OFF_PB + (BPACK ? S * B_P : 0);
-  static constexpr size_t OFF_COL = OFF_EPI + 2 * EPI_BYTES;
-  static constexpr size_t BYTES = OFF_COL + 2 * BN * sizeof(float);
-  static constexpr uint32_t TX = A_P + (BPACK ? B_P : B_U);
+  static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;              // [2][2][BN] floats
+  static constexpr size_t BYTES = OFF_COL + 4 * BN * sizeof(float);
+  static constexpr uint32_t TX = (APACK ? A_P : A_U) + (BPACK ? B_P : B_U);
 };
 
 struct __align__(8) Barriers {
-  uint64_t tma_full[3];  // packed A (+ B) landed
-  uint64_t unpacked[3];  // operand stage ready for the MMA
-  uint64_t mma_done[3];  // MMAs reading the stage completed
+  uint64_t tma_full[MAX_STAGES];  // operand bytes landed
+  uint64_t unpacked[MAX_STAGES];  // packed operands expanded (unpack warps)
+  uint64_t mma_done[MAX_STAGES];  // MMAs reading the stage completed
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drained;
@@ -83,9 +85,9 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 
 // Barrier init (thread 0) and TMEM allocation (warp WARP_MMA); the caller
 // follows with tcgen05 fences around a CTA barrier.
-template <bool BPACK>
+template <bool APACK, bool BPACK>
 __device__ __forceinline__ void setup(Barriers* bars) {
-  constexpr int S = Cfg<BPACK>::S;
+  constexpr int S = Cfg<APACK, BPACK>::S;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&bars->tma_full[s], 1);
@@ -123,13 +125,11 @@ __device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, ui
   return true;
 }
 
-template <typename OutT, bool BPACK>
+template <typename OutT, bool APACK, bool BPACK>
 __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
                                          Barriers* bars, uint32_t tmem, const uint32_t* ready) {
-  using C = Cfg<BPACK>;
+  using C = Cfg<APACK, BPACK>;
   constexpr int S = C::S;
-  float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL);
-  float* col_bias = col_scale + BN;
   volatile int32_t* abort = &bars->abort;
 
   const int warp = threadIdx.x >> 5;
@@ -166,7 +166,10 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
             break;
           }
           mbar_arrive_expect_tx(&bars->tma_full[s], C::TX);
-          tma_load_2d(smem + C::OFF_PA + s * A_P, maps.A, kb * BKP, m0, &bars->tma_full[s]);
+          if (APACK)
+            tma_load_2d(smem + C::OFF_PA + s * A_P, maps.A, kb * BKP, m0, &bars->tma_full[s]);
+          else
+            tma_load_2d(smem + C::OFF_UA + s * A_U, maps.A, kb * BK, m0, &bars->tma_full[s]);
           if (BPACK)
             tma_load_2d(smem + C::OFF_PB + s * B_P, maps.B, kb * BKP, n0, &bars->tma_full[s]);
           else
@@ -195,8 +198,8 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
         const uint32_t d = tmem + buf * BN;
         for (int kb = 0; kb < nk; ++kb, ++it) {
           const int s = it % S;
-          if (!mbar_wait_bounded(&bars->unpacked[s], (it / S) & 1, abort, g.status,
-                                 kWaitLimitNs)) {
+          uint64_t* ready_bar = C::UNPACK ? &bars->unpacked[s] : &bars->tma_full[s];
+          if (!mbar_wait_bounded(ready_bar, (it / S) & 1, abort, g.status, kWaitLimitNs)) {
             ok = false;
             break;
           }
@@ -216,23 +219,27 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       mbar_wait_bounded(&bars->drained, 0, nullptr, nullptr, 10000000ull);
     }
   } else if (warp >= WARP_UNPACK0 && warp < WARP_UNPACK0 + NUM_UNPACK / 32) {
-    const int ut = threadIdx.x - WARP_UNPACK0 * 32;
-    int it = 0;
-    bool ok = true;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-      for (int kb = 0; kb < nk; ++kb, ++it) {
-        const int s = it % S;
-        if (!mbar_wait_bounded(&bars->tma_full[s], (it / S) & 1, abort, g.status,
-                               kWaitLimitNs)) {
-          ok = false;
-          break;
+    if (C::UNPACK) {
+      const int ut = threadIdx.x - WARP_UNPACK0 * 32;
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait_bounded(&bars->tma_full[s], (it / S) & 1, abort, g.status,
+                                 kWaitLimitNs)) {
+            ok = false;
+            break;
+          }
+          if (APACK)
+            unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * A_U,
+                                        ut);
+          if (BPACK)
+            unpack_rows<BN, NUM_UNPACK>(smem + C::OFF_PB + s * B_P, smem + C::OFF_UB + s * B_U,
+                                        ut);
+          fence_proxy_async_smem();
+          mbar_arrive(&bars->unpacked[s]);
         }
-        unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * A_U, ut);
-        if (BPACK)
-          unpack_rows<BN, NUM_UNPACK>(smem + C::OFF_PB + s * B_P, smem + C::OFF_UB + s * B_U,
-                                      ut);
-        fence_proxy_async_smem();
-        mbar_arrive(&bars->unpacked[s]);
       }
     }
   } else if (warp < 4) {
@@ -243,7 +250,10 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       const int m0 = (t / tiles_n) * BM;
       const int n0 = (t % tiles_n) * BN;
       const int buf = tc & 1;
-      named_bar_sync(kEpiBarrier, 128);  // previous tile's column data consumed
+      // Column data of this tile into the buffer of its parity; the buffer of
+      // the other parity may still be read by slower warps (previous tile).
+      float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL) + buf * 2 * BN;
+      float* col_bias = col_scale + BN;
       for (int j = et; j < BN; j += 128) {
         const int col = n0 + j;
         float sc = 0.f, bi = 0.f;
@@ -257,19 +267,19 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       bool ok = mbar_wait_bounded(&bars->acc_full[buf], (tc >> 1) & 1, abort, g.status,
                                   kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok);
-      named_bar_sync(kEpiBarrier, 128);
+      named_bar_sync(kEpiBarrier, 128);  // column data of this tile written
       if (!ok || *abort != 0) break;
       tc_fence_after();
       // s_x may have been written by other CTAs of this grid (fused kernel):
       // read it from L2, after the tile's MMAs have completed.
       const int row = m0 + et;
       const float sx = row < g.M ? __ldcg(g.s_x + row) : 0.f;
-      epilogue_tile<OutT>(tmem + buf * BN, warp, et, m0, n0, g.M, g.N, sx, col_scale, col_bias,
-                          smem + C::OFF_EPI, maps.Y, g.Y, g.acc_dbg, stores);
+      epilogue_tile<OutT>(tmem + buf * BN, warp, lane, m0, n0, g.M, g.N, sx, col_scale,
+                          col_bias, smem + C::OFF_EPI, maps.Y, g.Y, g.acc_dbg, stores);
       tc_fence_before();
       mbar_arrive(&bars->acc_empty[buf]);
     }
-    if (et == 0) bulk_wait_all();
+    if (lane == 0) bulk_wait_all();
   }
 }
 

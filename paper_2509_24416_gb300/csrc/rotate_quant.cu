@@ -9,7 +9,7 @@ namespace {
 constexpr int kStages = rq::kMaxStages;  // raw tiles in flight per CTA
 
 template <typename T, int LOGB, bool CLIP>
-__global__ void __launch_bounds__(512) rotate_quant_kernel(RotateQuantArgs a) {
+__global__ void __maxnreg__(96) rotate_quant_kernel(RotateQuantArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   rq::run<T, LOGB, CLIP>(a, smem, kStages, nullptr, rq::NoPublish());
 }
@@ -41,11 +41,8 @@ template <typename T, int LOGB, bool CLIP>
 cudaError_t launch_rq_t(const RotateQuantArgs& a, int threads, size_t smem, int sms,
                         cudaStream_t st) {
   auto kern = rotate_quant_kernel<T, LOGB, CLIP>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
   int per_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(kern), smem, threads, &per_sm);
   if (e != cudaSuccess) return e;
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
   const int ntiles = (a.M + a.rows_per_tile - 1) / a.rows_per_tile;
@@ -105,11 +102,8 @@ cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
   int threads = 0;
   size_t smem = 0;
   rotate_quant_config(a.K, &args.rows_per_tile, &threads, &smem);
-  int dev = 0, sms = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return e;
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
   const bool clip = a.clip != nullptr;
   if (dtype == CLQ_F16)
     return clip ? launch_rq_b<__half, true>(args, logb, threads, smem, sms, st)

@@ -18,9 +18,10 @@
 //           fp32x2 arithmetic) and the remaining log2(b / 32) across lanes
 //           with shuffles, and reduces |x| per row;
 //  phase 3: s = absmax / 7, codes rint(x * (1 / s)) via the 1.5 * 2^23
-//           rounding constant (ties to even; the code's two's-complement
-//           nibble is the low nibble of the sum's bits), packing, one 16-byte
-//           store per thread.
+//           rounding constant (ties to even), then either packed nibbles
+//           (the code's two's complement is the low nibble of the sum's bits;
+//           one 16-byte store per thread) or one E4M3 byte per code (cvt of
+//           the integer-valued float; two 16-byte stores per thread).
 #pragma once
 
 #include "clq_device.cuh"
@@ -40,10 +41,16 @@ __device__ __forceinline__ uint32_t rowbuf_offset(uint32_t j) {
   return (phys << 4) | ((j & 7u) << 1);
 }
 
+// Two packed 16-bit values (low half first) -> float2, exactly.
 template <typename T>
-__device__ __forceinline__ float2 to_f2(uint32_t w) {
-  return make_float2(Num<T>::to_f(static_cast<uint16_t>(w & 0xFFFFu)),
-                     Num<T>::to_f(static_cast<uint16_t>(w >> 16)));
+__device__ __forceinline__ float2 to_f2(uint32_t w);
+template <>
+__device__ __forceinline__ float2 to_f2<__half>(uint32_t w) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&w));
+}
+template <>
+__device__ __forceinline__ float2 to_f2<__nv_bfloat16>(uint32_t w) {
+  return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
 }
 
 __device__ __forceinline__ uint32_t prmt_b32(uint32_t a, uint32_t b, uint32_t c) {
@@ -173,6 +180,32 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem, int
   const int pairs = R * cpr;
   bool aborted = false;
 
+  // Phase-1 work of this thread is the same for every tile: at most four
+  // (row, 16-byte chunk) pairs p = tid + u * blockDim.x (R * K / 8 <= 4 *
+  // blockDim.x).  Pair p reads bytes [16p, 16p + 16) of a raw stage (rows of
+  // 2K bytes are contiguous) and is live when p < rows * K / 8.  The shared
+  // address of each of its 8 elements' permuted positions is computed once.
+  const uint32_t rowbuf_base = smem_addr(sh.rowbuf);
+  const uint32_t raw_base = smem_addr(sh.raw);
+  uint32_t dst[4][8];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int p = tid + u * nthr;
+    const int r = p < pairs ? p / cpr : 0;
+    const int c = p < pairs ? p - r * cpr : 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      dst[u][e] = rowbuf_base + static_cast<uint32_t>(r * row_bytes) + sh.off[c * 8 + e];
+  }
+  // Phase-2 addresses of this thread's four 16-byte chunks.
+  uint32_t seg_addr[4];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    const uint32_t q = static_cast<uint32_t>(seg * 4 + c);
+    seg_addr[c] = rowbuf_base + static_cast<uint32_t>(r_local * row_bytes) +
+                  ((q ^ ((q >> 3) & 3u)) << 4);
+  }
+
   for (int i = 0;; ++i) {
     const int s = i % stages;
     const int par = i & 1;
@@ -186,23 +219,23 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem, int
     const int rows = min(R, a.M - row0);
 
     // ---- phase 1: raw rows -> permuted row buffer --------------------------
-    const uint8_t* raw = sh.raw + static_cast<size_t>(s) * R * row_bytes;
-    for (int p = tid; p < pairs; p += nthr) {
-      const int r = p / cpr;
-      const int c = p - r * cpr;
-      if (r >= rows) continue;
-      const uint4 v = *reinterpret_cast<const uint4*>(raw + r * row_bytes + c * 16);
-      const uint4 o0 = *reinterpret_cast<const uint4*>(sh.off + c * 8);
-      const uint4 o1 = *reinterpret_cast<const uint4*>(sh.off + c * 8 + 4);
-      uint8_t* rb = sh.rowbuf + r * row_bytes;
-      *reinterpret_cast<uint16_t*>(rb + o0.x) = static_cast<uint16_t>(v.x);
-      *reinterpret_cast<uint16_t*>(rb + o0.y) = static_cast<uint16_t>(v.x >> 16);
-      *reinterpret_cast<uint16_t*>(rb + o0.z) = static_cast<uint16_t>(v.y);
-      *reinterpret_cast<uint16_t*>(rb + o0.w) = static_cast<uint16_t>(v.y >> 16);
-      *reinterpret_cast<uint16_t*>(rb + o1.x) = static_cast<uint16_t>(v.z);
-      *reinterpret_cast<uint16_t*>(rb + o1.y) = static_cast<uint16_t>(v.z >> 16);
-      *reinterpret_cast<uint16_t*>(rb + o1.z) = static_cast<uint16_t>(v.w);
-      *reinterpret_cast<uint16_t*>(rb + o1.w) = static_cast<uint16_t>(v.w >> 16);
+    const uint32_t stage_base = raw_base + static_cast<uint32_t>(s * R * row_bytes);
+    const int live = rows * cpr;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int p = tid + u * nthr;
+      if (p < live) {
+        uint4 v;
+        asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                     : "r"(stage_base + 16u * static_cast<uint32_t>(p)));
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const uint16_t h = static_cast<uint16_t>(e & 1 ? (w[e >> 1] >> 16) : w[e >> 1]);
+          asm volatile("st.shared.u16 [%0], %1;" ::"r"(dst[u][e]), "h"(h) : "memory");
+        }
+      }
     }
     __syncthreads();
     // raw stage s is free again: refill it with the tile `stages` ahead
@@ -210,18 +243,17 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem, int
 
     // ---- phase 2: block Walsh-Hadamard transform and row abs-max ----------
     float2 v[16];  // v[k] holds positions 2k, 2k+1 of the segment
-    {
-      const uint8_t* rb = sh.rowbuf + r_local * row_bytes;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const uint32_t q = static_cast<uint32_t>(seg * 4 + c);
-        const uint32_t phys = q ^ ((q >> 3) & 3u);
-        const uint4 raw4 = *reinterpret_cast<const uint4*>(rb + (phys << 4));
-        v[4 * c + 0] = to_f2<T>(raw4.x);
-        v[4 * c + 1] = to_f2<T>(raw4.y);
-        v[4 * c + 2] = to_f2<T>(raw4.z);
-        v[4 * c + 3] = to_f2<T>(raw4.w);
-      }
+    for (int c = 0; c < 4; ++c) {
+      uint4 raw4;
+      asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                   : "=r"(raw4.x), "=r"(raw4.y), "=r"(raw4.z), "=r"(raw4.w)
+                   : "r"(seg_addr[c])
+                   : "memory");
+      v[4 * c + 0] = to_f2<T>(raw4.x);
+      v[4 * c + 1] = to_f2<T>(raw4.y);
+      v[4 * c + 2] = to_f2<T>(raw4.z);
+      v[4 * c + 3] = to_f2<T>(raw4.w);
     }
     const float2 neg1 = make_float2(-1.f, -1.f);
     if (lb >= 1) {  // stride 1: inside each pair
@@ -276,11 +308,35 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem, int
       float amax = __uint_as_float(sh.amax[par * R + r_local]);
       if (CLIP) amax = fminf(amax, __ldg(a.clip + row));
       const float s_row = __fdiv_rn(amax, 7.0f);
-      uint32_t w[4] = {0u, 0u, 0u, 0u};
-      if (s_row > 0.f) {
-        const float rcp = __frcp_rn(s_row);
-        const float2 rc2 = make_float2(rcp, rcp);
-        const float2 magic = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
+      const float rcp = s_row > 0.f ? __frcp_rn(s_row) : 0.f;
+      const float2 rc2 = make_float2(rcp, rcp);
+      const float2 magic = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
+      if (a.e4m3) {
+        // one byte per code: the E4M3 encoding of the integer code
+        uint32_t w[8];
+#pragma unroll
+        for (int k = 0; k < 16; k += 2) {
+          uint32_t h[2];
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            float2 r = __fmul2_rn(v[k + j], rc2);
+            if (CLIP) {
+              r.x = fminf(fmaxf(r.x, -7.f), 7.f);
+              r.y = fminf(fmaxf(r.y, -7.f), 7.f);
+            }
+            const float2 q = __fadd2_rn(__fadd2_rn(r, magic), make_float2(-12582912.0f, -12582912.0f));
+            uint16_t e;
+            asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(e) : "f"(q.y), "f"(q.x));
+            h[j] = e;
+          }
+          w[k >> 1] = h[0] | (h[1] << 16);
+        }
+        uint4* qrow = reinterpret_cast<uint4*>(a.Q + static_cast<size_t>(row) * K + seg * 32);
+        qrow[0] = make_uint4(w[0], w[1], w[2], w[3]);
+        qrow[1] = make_uint4(w[4], w[5], w[6], w[7]);
+      } else {
+        // two codes per byte: the low nibble of (x / s + 1.5 * 2^23)'s bits
+        // is the code's two's complement
         uint32_t by[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
@@ -293,13 +349,14 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem, int
           const uint32_t b0 = __float_as_uint(t.x), b1 = __float_as_uint(t.y);
           by[k] = (b0 & 0xFu) | ((b1 << 4) & 0xF0u);
         }
+        uint32_t w[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           w[q] = prmt_b32(prmt_b32(by[4 * q], by[4 * q + 1], 0x0040u),
                           prmt_b32(by[4 * q + 2], by[4 * q + 3], 0x0040u), 0x5410u);
+        uint8_t* qrow = a.Q + static_cast<size_t>(row) * (K >> 1);
+        *reinterpret_cast<uint4*>(qrow + seg * 16) = make_uint4(w[0], w[1], w[2], w[3]);
       }
-      uint8_t* qrow = a.Q + static_cast<size_t>(row) * (K >> 1);
-      *reinterpret_cast<uint4*>(qrow + seg * 16) = make_uint4(w[0], w[1], w[2], w[3]);
       if (seg == 0) a.S[row] = s_row;
       if (a.rot != nullptr) {
         float4* dst = reinterpret_cast<float4*>(a.rot + static_cast<size_t>(row) * K + seg * 32);

@@ -4,6 +4,12 @@
 
 #include <cudaTypedefs.h>
 
+#include <atomic>
+#include <map>
+#include <mutex>
+#include <set>
+#include <tuple>
+
 namespace clq {
 
 namespace {
@@ -12,12 +18,12 @@ using namespace gemm;
 
 constexpr int THREADS = MIN_THREADS;  // 448
 
-template <bool BPACK>
+template <bool APACK, bool BPACK>
 constexpr size_t smem_bytes() {
-  return Cfg<BPACK>::BYTES + 1024;  // + alignment slack
+  return Cfg<APACK, BPACK>::BYTES + 1024;  // + alignment slack
 }
 
-template <typename OutT, bool BPACK>
+template <typename OutT, bool APACK, bool BPACK>
 __global__ void __launch_bounds__(THREADS, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                      const __grid_constant__ CUtensorMap mapB,
@@ -26,13 +32,13 @@ __global__ void __launch_bounds__(THREADS, 1)
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  setup<BPACK>(&bars);
+  setup<APACK, BPACK>(&bars);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars.tmem_slot;
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
-  pipeline<OutT, BPACK>(maps, g, smem, &bars, tmem, nullptr);
+  pipeline<OutT, APACK, BPACK>(maps, g, smem, &bars, tmem, nullptr);
   tc_fence_before();
   __syncthreads();
   teardown(tmem);
@@ -86,44 +92,99 @@ bool encode_tma_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes, 
 
 bool encode_tma_out_tile(CUtensorMap* map, void* Y, int M, int N) {
   return encode_tma_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, Y, static_cast<uint64_t>(N),
-                       static_cast<uint64_t>(M), EPI_COLS, BM, CU_TENSOR_MAP_SWIZZLE_64B);
+                       static_cast<uint64_t>(M), EPI_COLS, EPI_ROWS, CU_TENSOR_MAP_SWIZZLE_64B);
 }
 
 int sm_count() {
+  static std::atomic<int> cached[64];
   int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  sms = cached[dev].load(std::memory_order_relaxed);
+  if (sms > 0) return sms;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  cached[dev].store(sms, std::memory_order_relaxed);
   return sms;
 }
 
-template <typename OutT, bool BPACK>
+cudaError_t kernel_setup(const void* func, size_t smem, int threads, int* per_sm) {
+  static std::mutex mu;
+  static std::map<std::tuple<const void*, int, size_t, int>, int> occupancy;
+  static std::set<std::pair<const void*, int>> raised;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  if (raised.count({func, dev}) == 0) {
+    int optin = 0;
+    e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e != cudaSuccess) return e;
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, func);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             optin - static_cast<int>(fa.sharedSizeBytes));
+    if (e != cudaSuccess) return e;
+    raised.insert({func, dev});
+  }
+  if (per_sm != nullptr) {
+    const auto key = std::make_tuple(func, dev, smem, threads);
+    auto it = occupancy.find(key);
+    if (it == occupancy.end()) {
+      int n = 0;
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, func, threads, smem);
+      if (e != cudaSuccess) return e;
+      it = occupancy.emplace(key, n).first;
+    }
+    *per_sm = it->second;
+  }
+  return cudaSuccess;
+}
+
+namespace {
+
+template <typename OutT, bool APACK, bool BPACK>
 cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB,
                           const CUtensorMap& mapY, const GemmArgs& g, int use_tma_store,
                           int grid, cudaStream_t st) {
-  auto k = w4a4_gemm_kernel<OutT, BPACK>;
-  constexpr size_t smem = smem_bytes<BPACK>();
-  cudaError_t e =
-      cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK>;
+  constexpr size_t smem = smem_bytes<APACK, BPACK>();
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, THREADS, nullptr);
   if (e != cudaSuccess) return e;
   k<<<grid, THREADS, smem, st>>>(mapA, mapB, mapY, g, use_tma_store);
   return cudaGetLastError();
 }
 
-cudaError_t launch_w4a4_gemm(const uint8_t* Xq, const uint8_t* W, int w_format,
+template <typename OutT>
+cudaError_t launch_gemm_dt(const CUtensorMap& mapA, const CUtensorMap& mapB,
+                           const CUtensorMap& mapY, const GemmArgs& g, bool apack, bool bpack,
+                           int use_tma_store, int grid, cudaStream_t st) {
+  if (apack)
+    return bpack ? launch_gemm_t<OutT, true, true>(mapA, mapB, mapY, g, use_tma_store, grid, st)
+                 : launch_gemm_t<OutT, true, false>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+  return bpack ? launch_gemm_t<OutT, false, true>(mapA, mapB, mapY, g, use_tma_store, grid, st)
+               : launch_gemm_t<OutT, false, false>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+}
+
+}  // namespace
+
+// TMA map of an INT4 code array (rows x K codes) in either layout: packed
+// boxes of 64 bytes x box_rows (no swizzle, staged for unpacking) or E4M3
+// boxes of 128 bytes x box_rows with the 128-byte swizzle (MMA operand).
+bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows, int K,
+                      int box_rows) {
+  if (codes == CLQ_CODES_INT4_PACKED)
+    return encode_tma_2d_u8(map, base, static_cast<uint64_t>(K) / 2, static_cast<uint64_t>(rows),
+                            BKP, box_rows);
+  return encode_tma_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, base, static_cast<uint64_t>(K),
+                       static_cast<uint64_t>(rows), BK, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st) {
   CUtensorMap mapA, mapB, mapY;
-  const uint64_t kb = static_cast<uint64_t>(g.K) / 2;
-  const bool bpack = w_format == CLQ_W_INT4_PACKED;
-  if (!encode_tma_2d_u8(&mapA, Xq, kb, static_cast<uint64_t>(g.M), BKP, BM))
+  if (!encode_codes_map(&mapA, Xq, x_codes, g.M, g.K, BM) ||
+      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, BN))
     return cudaErrorInvalidValue;
-  if (bpack) {
-    if (!encode_tma_2d_u8(&mapB, W, kb, static_cast<uint64_t>(g.N), BKP, BN))
-      return cudaErrorInvalidValue;
-  } else {
-    if (!encode_tma_2d(&mapB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, W, static_cast<uint64_t>(g.K),
-                       static_cast<uint64_t>(g.N), BK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
-      return cudaErrorInvalidValue;
-  }
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
   if (use_tma_store) {
     if (!encode_tma_out_tile(&mapY, g.Y, g.M, g.N)) return cudaErrorInvalidValue;
@@ -134,11 +195,12 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, const uint8_t* W, int w_format,
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
   const int grid = std::min(tiles, sms);
+  const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
+  const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
   if (out_dtype == CLQ_F16)
-    return bpack ? launch_gemm_t<__half, true>(mapA, mapB, mapY, g, use_tma_store, grid, st)
-                 : launch_gemm_t<__half, false>(mapA, mapB, mapY, g, use_tma_store, grid, st);
-  return bpack ? launch_gemm_t<__nv_bfloat16, true>(mapA, mapB, mapY, g, use_tma_store, grid, st)
-               : launch_gemm_t<__nv_bfloat16, false>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+    return launch_gemm_dt<__half>(mapA, mapB, mapY, g, apack, bpack, use_tma_store, grid, st);
+  return launch_gemm_dt<__nv_bfloat16>(mapA, mapB, mapY, g, apack, bpack, use_tma_store, grid,
+                                       st);
 }
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st) {

@@ -46,37 +46,39 @@ P = 1 << 20  # a fake, 16-byte aligned "device" address; never dereferenced
 
 
 @pytest.mark.parametrize("args,code", [
-    # (X, dtype, M, K, ldx, perm, b, Xq, s_x, rot) -> expected status
-    ((P, 2, 4, 64, 64, P, 32, P, P, None), 1),      # bad dtype
-    ((P, 0, -1, 64, 64, P, 32, P, P, None), 1),     # negative M
-    ((P, 0, 4, 64, 64, P, 3, P, P, None), 2),       # b not a power of two
-    ((P, 0, 4, 64, 64, P, 512, P, P, None), 2),     # b > 256
-    ((P, 0, 4, 48, 48, P, 16, P, P, None), 2),      # K % 32
-    ((P, 0, 4, 1152, 1152, P, 256, P, P, None), 2), # K % b (1152 / 256)
-    ((P, 0, 4, 32768, 32768, P, 32, P, P, None), 2),  # K too large
-    ((P, 0, 4, 64, 32, P, 32, P, P, None), 2),      # ldx < K
-    ((P, 0, 4, 64, 68, P, 32, P, P, None), 3),      # ldx % 8
-    ((None, 0, 4, 64, 64, P, 32, P, P, None), 1),   # null X
-    ((P, 0, 4, 64, 64, None, 32, P, P, None), 1),   # null perm
-    ((P + 8, 0, 4, 64, 64, P, 32, P, P, None), 3),  # misaligned X
-    ((P, 0, 4, 64, 64, P, 32, P + 4, P, None), 3),  # misaligned Xq
-    ((P, 0, 0, 64, 64, None, 32, None, None, None), 0),  # empty: no-op
+    # (X, dtype, M, K, ldx, perm, b, codes, Xq, s_x, rot) -> expected status
+    ((P, 2, 4, 64, 64, P, 32, 0, P, P, None), 1),      # bad dtype
+    ((P, 0, 4, 64, 64, P, 32, 3, P, P, None), 1),      # bad code layout
+    ((P, 0, -1, 64, 64, P, 32, 0, P, P, None), 1),     # negative M
+    ((P, 0, 4, 64, 64, P, 3, 0, P, P, None), 2),       # b not a power of two
+    ((P, 0, 4, 64, 64, P, 512, 1, P, P, None), 2),     # b > 256
+    ((P, 0, 4, 48, 48, P, 16, 0, P, P, None), 2),      # K % 32
+    ((P, 0, 4, 1152, 1152, P, 256, 0, P, P, None), 2), # K % b (1152 / 256)
+    ((P, 0, 4, 32768, 32768, P, 32, 0, P, P, None), 2),  # K too large
+    ((P, 0, 4, 64, 32, P, 32, 0, P, P, None), 2),      # ldx < K
+    ((P, 0, 4, 64, 68, P, 32, 0, P, P, None), 3),      # ldx % 8
+    ((None, 0, 4, 64, 64, P, 32, 0, P, P, None), 1),   # null X
+    ((P, 0, 4, 64, 64, None, 32, 1, P, P, None), 1),   # null perm
+    ((P + 8, 0, 4, 64, 64, P, 32, 0, P, P, None), 3),  # misaligned X
+    ((P, 0, 4, 64, 64, P, 32, 1, P + 4, P, None), 3),  # misaligned Xq
+    ((P, 0, 0, 64, 64, None, 32, 0, None, None, None), 0),  # empty: no-op
 ])
 def test_rotate_quant_host_validation(lib, args, code):
     assert clq.clq_rotate_quant_act(*args, None) == code
 
 
 @pytest.mark.parametrize("args,code", [
-    # (Xq, s_x, W, w_format, s_w, bias, M, N, K, b, out_dtype, Y, acc)
-    ((P, P, P, 0, P, None, 4, 4, 64, 32, 3, P, None), 1),     # bad out dtype
-    ((P, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad w_format
-    ((P, P, P, 0, P, None, 4, -2, 64, 32, 0, P, None), 1),    # negative N
-    ((P, P, P, 1, P, None, 4, 4, 96, 64, 0, P, None), 2),     # K % b
-    ((P, P, P, 0, P, None, 4, 4, 64, 32, 0, P + 2, None), 3), # misaligned Y
-    ((P, P, P, 0, P, P + 1, 4, 4, 64, 32, 0, P, None), 3),    # misaligned bias
-    ((None, P, P, 0, P, None, 4, 4, 64, 32, 0, P, None), 1),  # null Xq
-    ((None, None, None, 0, None, None, 0, 4, 64, 32, 0, None, None), 0),
-    ((None, None, None, 1, None, None, 4, 0, 64, 32, 0, None, None), 0),
+    # (Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b, out_dtype, Y, acc)
+    ((P, 0, P, P, 0, P, None, 4, 4, 64, 32, 3, P, None), 1),     # bad out dtype
+    ((P, 0, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad w layout
+    ((P, 5, P, P, 0, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad x layout
+    ((P, 0, P, P, 0, P, None, 4, -2, 64, 32, 0, P, None), 1),    # negative N
+    ((P, 1, P, P, 1, P, None, 4, 4, 96, 64, 0, P, None), 2),     # K % b
+    ((P, 0, P, P, 0, P, None, 4, 4, 64, 32, 0, P + 2, None), 3), # misaligned Y
+    ((P, 0, P, P, 0, P, P + 1, 4, 4, 64, 32, 0, P, None), 3),    # misaligned bias
+    ((None, 0, P, P, 0, P, None, 4, 4, 64, 32, 0, P, None), 1),  # null Xq
+    ((None, 0, None, None, 0, None, None, 0, 4, 64, 32, 0, None, None), 0),
+    ((None, 1, None, None, 1, None, None, 4, 0, 64, 32, 0, None, None), 0),
 ])
 def test_w4a4_host_validation(lib, args, code):
     assert clq.clq_w4a4_linear(*args, None) == code
@@ -84,8 +86,8 @@ def test_w4a4_host_validation(lib, args, code):
 
 def test_fused_and_prepare_host_validation(lib):
     ws = clq.clq_fused_linear_workspace_size(256, 1152)
-    # 256 x 576 codes, 256 scales, 2 block counters + 1 tile counter
-    assert ws == 147456 + 1024 + 256
+    # 256 x 1152 E4M3 codes, 256 scales, 2 block counters + 1 tile counter
+    assert ws == 294912 + 1024 + 256
     assert clq.clq_fused_linear_workspace_size(4, 48) == 0
     # (X, dtype, M, K, ldx, perm, b, W, w_format, s_w, bias, N, Y, ws, bytes)
     assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 7, P, 0, P, None, 4, P, P,

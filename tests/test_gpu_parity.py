@@ -39,19 +39,44 @@ def _perm(K, kind, seed=0):
     return np.random.default_rng(seed).permutation(K).astype(np.int32)
 
 
-def _rq_gpu(x, perm, b):
+def _decode_e4m3(byte):
+    """Value of an E4M3 byte (1 sign, 4 exponent bits with bias 7, 3 mantissa
+    bits; exponent 0 is subnormal), written out from the format definition."""
+    b = np.asarray(byte, np.int64)
+    sign = np.where(b & 0x80, -1.0, 1.0)
+    e = (b >> 3) & 0xF
+    m = b & 0x7
+    val = np.where(e == 0, m / 8.0 * 2.0 ** -6, (1 + m / 8.0) * 2.0 ** (e - 7.0))
+    return sign * val
+
+
+def _codes(Xq, K):
+    """Integer codes of a GPU code array in either layout."""
+    Xq = np.asarray(Xq)
+    if Xq.shape[1] == K:
+        v = _decode_e4m3(Xq)
+        assert np.array_equal(v, np.rint(v)) and np.abs(v).max(initial=0) <= 7
+        return v.astype(np.int8)
+    return oracle.unpack_int4(Xq)
+
+
+def _rq_gpu(x, perm, b, codes=clq.CLQ_CODES_INT4_PACKED):
     Xq, s_x, rot = clq.rotate_quant_act(x.to(DEV), torch.from_numpy(perm).to(DEV),
-                                        b, with_rot=True)
+                                        b, codes, with_rot=True)
     torch.cuda.synchronize()
     return Xq.cpu().numpy(), s_x.cpu().numpy(), rot.cpu().numpy()
 
 
 def _check_rq(x_t, x32, perm, b):
+    K = x32.shape[1]
     gq, gs, grot = _rq_gpu(x_t, perm, b)
+    eq, es, erot = _rq_gpu(x_t, perm, b, clq.CLQ_CODES_E4M3)
     oq, os_, orot, oc = oracle.rotate_quant_act(x32, perm, b)
     check_rot(grot, orot)
     check_scales(gs, os_)
-    check_codes(oracle.unpack_int4(gq), oc, orot, os_)
+    check_codes(_codes(gq, K), oc, orot, os_)
+    # both layouts carry the same codes and scales
+    assert np.array_equal(_codes(eq, K), _codes(gq, K)) and np.array_equal(es, gs)
     return gq, gs
 
 
@@ -178,17 +203,6 @@ def test_prepare_weights_with_clip():
 
 
 # -------------------------------------------------------------------- GEMM --
-def _decode_e4m3(byte):
-    """Value of an E4M3 byte (1 sign, 4 exponent bits with bias 7, 3 mantissa
-    bits; exponent 0 is subnormal), written out from the format definition."""
-    b = np.asarray(byte, np.int64)
-    sign = np.where(b & 0x80, -1.0, 1.0)
-    e = (b >> 3) & 0xF
-    m = b & 0x7
-    val = np.where(e == 0, m / 8.0 * 2.0 ** -6, (1 + m / 8.0) * 2.0 ** (e - 7.0))
-    return sign * val
-
-
 def test_expand_weights_is_exact_e4m3_of_codes():
     rng = np.random.default_rng(4)
     codes = rng.integers(-7, 8, (300, 1152)).astype(np.int8)
@@ -212,19 +226,23 @@ def _gemm_case(M, N, K, b, dtype, seed, bias=True):
     b32 = None if bias_t is None else bias_t.float().numpy()
     y64, acc = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, b32)
     Wq = torch.from_numpy(oWq).to(DEV)
+    Xq = torch.from_numpy(oXq).to(DEV)
     outs = []
-    for W in (Wq, clq.expand_weights(Wq)):       # storage and execution layouts
-        Y, gacc = clq.w4a4_linear(torch.from_numpy(oXq).to(DEV), torch.from_numpy(os_x).to(DEV),
-                                  W, torch.from_numpy(os_w).to(DEV),
-                                  b, None if bias_t is None else bias_t.to(DEV),
-                                  out_dtype=TD[dtype], with_acc=True)
-        torch.cuda.synchronize()
-        assert np.array_equal(gacc.cpu().numpy(), acc)
-        y = Y.float().cpu().numpy()
-        check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
-        check_output_frobenius(y, y64)
-        outs.append(Y)
-    assert torch.equal(outs[0], outs[1])
+    # every combination of storage (packed) and execution (E4M3) layouts
+    for Xc in (Xq, clq.expand_weights(Xq)):
+        for W in (Wq, clq.expand_weights(Wq)):
+            Y, gacc = clq.w4a4_linear(Xc, torch.from_numpy(os_x).to(DEV), W,
+                                      torch.from_numpy(os_w).to(DEV), b, K,
+                                      None if bias_t is None else bias_t.to(DEV),
+                                      out_dtype=TD[dtype], with_acc=True)
+            torch.cuda.synchronize()
+            assert np.array_equal(gacc.cpu().numpy(), acc)
+            y = Y.float().cpu().numpy()
+            check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
+            check_output_frobenius(y, y64)
+            outs.append(Y)
+    for Y in outs[1:]:
+        assert torch.equal(outs[0], Y)
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 1, 32), (3, 17, 64), (17, 64, 128),
@@ -261,11 +279,13 @@ def test_gemm_carrier_exact_at_extremes(K):
     ones_x = torch.ones(M, dtype=torch.float32, device=DEV)
     ones_w = torch.ones(N, dtype=torch.float32, device=DEV)
     Wd = torch.from_numpy(Wq).to(DEV)
-    for W in (Wd, clq.expand_weights(Wd)):
-        _, gacc = clq.w4a4_linear(torch.from_numpy(Xq).to(DEV), ones_x, W, ones_w, 32,
-                                  out_dtype=torch.bfloat16, with_acc=True)
-        torch.cuda.synchronize()
-        assert np.array_equal(gacc.cpu().numpy(), acc)
+    Xd = torch.from_numpy(Xq).to(DEV)
+    for Xc in (Xd, clq.expand_weights(Xd)):
+        for W in (Wd, clq.expand_weights(Wd)):
+            _, gacc = clq.w4a4_linear(Xc, ones_x, W, ones_w, 32, K,
+                                      out_dtype=torch.bfloat16, with_acc=True)
+            torch.cuda.synchronize()
+            assert np.array_equal(gacc.cpu().numpy(), acc)
 
 
 def test_gemm_random_codes_all_values():
@@ -276,7 +296,7 @@ def test_gemm_random_codes_all_values():
     acc = oracle.int_gemm(qx, qw)
     s = torch.ones(max(M, N), dtype=torch.float32, device=DEV)
     _, gacc = clq.w4a4_linear(torch.from_numpy(oracle.pack_int4(qx)).to(DEV), s[:M],
-                              torch.from_numpy(oracle.pack_int4(qw)).to(DEV), s[:N], 32,
+                              torch.from_numpy(oracle.pack_int4(qw)).to(DEV), s[:N], 32, K,
                               with_acc=True)
     torch.cuda.synchronize()
     assert np.array_equal(gacc.cpu().numpy(), acc)
@@ -295,9 +315,11 @@ def _layer_e2e(cfg, li, M, rows=None):
     permd = perm.to(DEV)
     layer = clq.PreparedLinear.from_weight(d["W"].to(DEV), permd, b, bias=d["bias"].to(DEV))
     X = d["X"].to(DEV)
+    K = X.shape[1]
     Xq, s_x, rot = clq.rotate_quant_act(X, permd, b, with_rot=True)
-    Y = clq.w4a4_linear(Xq, s_x, layer.We, layer.s_w, b, layer.bias, out_dtype=X.dtype)
+    Y = clq.w4a4_linear(Xq, s_x, layer.Wq, layer.s_w, b, K, layer.bias, out_dtype=X.dtype)
     torch.cuda.synchronize()
+    assert torch.equal(layer(X), Y)    # execution layouts (E4M3 codes) = storage
     rows = np.arange(M) if rows is None else rows
     p = perm.numpy()
     oWq, os_w, orot_w, owc = oracle.prepare_weights(d["W32"], p, b)
@@ -307,7 +329,7 @@ def _layer_e2e(cfg, li, M, rows=None):
     oXq, os_x, orot, oc = oracle.rotate_quant_act(x32, p, b)
     check_rot(rot.cpu().numpy()[rows], orot)
     check_scales(s_x.cpu().numpy()[rows], os_x)
-    check_codes(oracle.unpack_int4(Xq.cpu().numpy()[rows]), oc, orot, os_x)
+    check_codes(_codes(Xq.cpu().numpy()[rows], K), oc, orot, os_x)
     y64, _ = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, d["bias32"])
     check_output_frobenius(Y.float().cpu().numpy()[rows], y64)
     Yf = layer(X, fused=True)
@@ -407,5 +429,5 @@ def test_empty_inputs_are_noops():
     Xq, s_x = clq.rotate_quant_act(z, perm, 32)
     assert Xq.shape == (0, 32) and s_x.shape == (0,)
     Wq = torch.zeros((0, 32), dtype=torch.uint8, device=DEV)
-    Y = clq.w4a4_linear(Xq, s_x, Wq, torch.empty(0, device=DEV), 32)
+    Y = clq.w4a4_linear(Xq, s_x, Wq, torch.empty(0, device=DEV), 32, 64)
     assert Y.shape == (0, 0)

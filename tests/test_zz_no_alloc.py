@@ -35,7 +35,7 @@ def _noalloc(X, layer, Y):
     N = layer.We.shape[0]
     st = clq.clq_fused_linear_noalloc(
         X.data_ptr(), clq.CLQ_F16, M, K, X.stride(0), layer.perm.data_ptr(), layer.b,
-        layer.We.data_ptr(), clq.CLQ_W_E4M3, layer.s_w.data_ptr(), layer.bias.data_ptr(),
+        layer.We.data_ptr(), clq.CLQ_CODES_E4M3, layer.s_w.data_ptr(), layer.bias.data_ptr(),
         N, Y.data_ptr(), torch.cuda.current_stream().cuda_stream)
     return st
 
@@ -56,10 +56,10 @@ def test_noalloc_matches_fused_on_two_calls_in_a_row():
 
 
 def test_noalloc_refuses_problems_beyond_the_scratch_limit():
-    # 65536 tokens x 2048 channels need 64 MiB of codes plus scales: too big.
+    # 65536 tokens x 2048 channels need 128 MiB of E4M3 codes: too big.
     M, K = 65536, 2048
     assert clq.clq_fused_linear_workspace_size(M, K) > (64 << 20)
     P = 1 << 20  # never dereferenced: the call must return before launching
     st = clq.clq_fused_linear_noalloc(P, clq.CLQ_F16, M, K, K, P, 64, P,
-                                      clq.CLQ_W_E4M3, P, None, 128, P, None)
+                                      clq.CLQ_CODES_E4M3, P, None, 128, P, None)
     assert st == 8  # CLQ_ERR_SCRATCH_LIMIT
