@@ -24,7 +24,7 @@ namespace {
 
 using namespace gemm;
 
-constexpr int FT = 512;  // threads: the RQ phase uses all; the GEMM phase 448
+constexpr int FT = 512;  // threads: the RQ phase uses all, the GEMM phase up to 448
 
 struct PublishRows {
   uint32_t* ready;
@@ -45,7 +45,7 @@ struct PublishRows {
   }
 };
 
-template <typename T, bool BPACK>
+template <typename T, bool BPACK, int BNT>
 __global__ void __launch_bounds__(FT, 1)
     fused_linear_kernel(const __grid_constant__ CUtensorMap mapA,
                         const __grid_constant__ CUtensorMap mapB,
@@ -56,7 +56,7 @@ __global__ void __launch_bounds__(FT, 1)
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  setup<false, BPACK>(&bars);
+  setup<false, BPACK, BNT>(&bars);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -66,18 +66,18 @@ __global__ void __launch_bounds__(FT, 1)
   __syncthreads();
 
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
-  pipeline<T, false, BPACK>(maps, g, smem, &bars, tmem, ready);
+  pipeline<T, false, BPACK, BNT, false>(maps, g, smem, &bars, tmem, ready);
   tc_fence_before();
   __syncthreads();
-  teardown(tmem);
+  teardown(tmem, Cfg<false, BPACK, BNT>::TMEM);
 }
 
-template <typename T, bool BPACK>
+template <typename T, bool BPACK, int BNT>
 cudaError_t launch_t(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                      const RotateQuantArgs& rq, const GemmArgs& g, uint32_t* ready,
                      int use_tma_store, int rq_stages, size_t smem, int grid, cudaStream_t st) {
   uint32_t* tile_counter = ready + (g.M + BM - 1) / BM;
-  auto k = fused_linear_kernel<T, BPACK>;
+  auto k = fused_linear_kernel<T, BPACK, BNT>;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, FT, nullptr);
   if (e != cudaSuccess) return e;
   k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store,
@@ -103,6 +103,9 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
                                 const GemmArgs& g, int logb, int dtype, uint32_t* ready,
                                 cudaStream_t st) {
   const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  const int bn = BN;
   const size_t gemm_bytes = bpack ? Cfg<false, true>::BYTES : Cfg<false, false>::BYTES;
   const size_t limit = 227u * 1024u - 2048u;  // dynamic + static shared memory
   // Rotate-quant phase: as many rows per tile as 512 threads cover, then as
@@ -126,7 +129,7 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
 
   CUtensorMap mapA, mapB, mapY;
   if (!encode_codes_map(&mapA, rq.Q, CLQ_CODES_E4M3, g.M, g.K, BM) ||
-      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, BN))
+      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn))
     return cudaErrorInvalidValue;
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
   if (use_tma_store) {
@@ -134,18 +137,16 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   } else {
     mapY = mapA;  // unused
   }
-  const int sms = sm_count();
-  if (sms <= 0) return cudaErrorInvalidDevice;
   const int grid = sms;
   if (dtype == CLQ_F16)
-    return bpack ? launch_t<__half, true>(mapA, mapB, mapY, rq, g, ready, use_tma_store, stages,
-                                          smem, grid, st)
-                 : launch_t<__half, false>(mapA, mapB, mapY, rq, g, ready, use_tma_store, stages,
-                                           smem, grid, st);
-  return bpack ? launch_t<__nv_bfloat16, true>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                               stages, smem, grid, st)
-               : launch_t<__nv_bfloat16, false>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                                stages, smem, grid, st);
+    return bpack ? launch_t<__half, true, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
+                                              stages, smem, grid, st)
+                 : launch_t<__half, false, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
+                                               stages, smem, grid, st);
+  return bpack ? launch_t<__nv_bfloat16, true, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
+                                                   stages, smem, grid, st)
+               : launch_t<__nv_bfloat16, false, BN>(mapA, mapB, mapY, rq, g, ready,
+                                                    use_tma_store, stages, smem, grid, st);
 }
 
 }  // namespace clq

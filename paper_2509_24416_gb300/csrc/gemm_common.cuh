@@ -9,7 +9,7 @@ namespace clq {
 namespace gemm {
 
 constexpr int BM = 128;           // rows of A (tokens) per tile
-constexpr int BN = 256;           // rows of B (output channels) per tile
+constexpr int BN = 256;           // rows of B (output channels) per tile (widest)
 constexpr int BK = 128;           // codes per K step = one 128-byte swizzle row
 constexpr int BKP = BK / 2;       // packed bytes per row per K step
 constexpr int A_U = BM * BK;      // 16 KB unpacked A stage
@@ -19,7 +19,7 @@ constexpr int B_P = BN * BKP;     // 16 KB packed B stage
 constexpr int EPI_COLS = 32;      // output columns per epilogue store
 constexpr int EPI_ROWS = 32;      // rows per store: one warp's TMEM lanes
 constexpr int EPI_BYTES = EPI_ROWS * EPI_COLS * 2;  // 2 KB staging buffer
-constexpr int EPI_TOTAL = 4 * 2 * EPI_BYTES;        // 4 warps x 2 buffers
+constexpr int EPI_TOTAL = 8 * EPI_BYTES;            // 4 warps x 2 or 8 warps x 1
 constexpr int TMEM_COLS = 512;    // two 128 x 256 fp32 accumulators
 constexpr uint32_t kEpiBarrier = 1;  // named barrier id of the epilogue warps
 
@@ -117,75 +117,120 @@ __device__ __forceinline__ void bulk_wait_all() {
   asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
-// Epilogue of one 128 x 256 tile: each of four warps drains its own 32 TMEM
-// lanes (rows) independently.  y = acc * s_x[row] * s_w[col] / b +
-// bias[col], rounded to OutT; col_scale / col_bias hold s_w / b and bias for
-// the tile's columns.  With a TMA map for Y, each 32 x 32 block goes through
-// the warp's own 64-byte-swizzled staging buffer (two, alternating) and one
-// bulk tensor store issued by lane 0; otherwise (N not a multiple of 8) lanes
-// store their row directly.  `store_count` counts this warp's stores.
-template <typename OutT>
-__device__ __forceinline__ void epilogue_tile(uint32_t tmem_acc, int warp_q, int lane, int m0,
-                                              int n0, int M, int N, float sx,
+// Wait for this thread's outstanding tcgen05.ld and make every register of
+// r depend on that wait, so that no use of r is scheduled before it.
+__device__ __forceinline__ void tmem_ld_wait_tie(uint32_t (&r)[32]) {
+  tmem_ld_wait();
+#pragma unroll
+  for (int i = 0; i < 32; ++i) asm volatile("" : "+r"(r[i]));
+}
+
+// One 32-row x 32-column block of the epilogue (the block at tile column c):
+// y = acc * s_x[row] * s_w[col] / b + bias[col], rounded to OutT, where
+// col_scale / col_bias hold s_w / b and bias for the tile's columns.  With a
+// TMA map for Y the block goes through one of the warp's NBUF 64-byte-swizzled
+// staging buffers and one bulk tensor store issued by lane 0; otherwise (N not
+// a multiple of 8) each lane stores its row directly.
+template <typename OutT, int NBUF>
+__device__ __forceinline__ void epilogue_block(const uint32_t (&r)[32], int c, int quarter,
+                                               int lane, int m0, int n0, int M, int N,
+                                               float sx, const float* col_scale,
+                                               const float* col_bias, uint8_t* staging,
+                                               const CUtensorMap* mapY, void* Y,
+                                               int32_t* acc_dbg, int& store_count) {
+  const int row = m0 + quarter * 32 + lane;
+  uint32_t o[16];
+  const float2 sx2 = make_float2(sx, sx);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const float4 cs = *reinterpret_cast<const float4*>(col_scale + c + 4 * j);
+    const float4 cb = *reinterpret_cast<const float4*>(col_bias + c + 4 * j);
+    const float2 a0 = make_float2(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]));
+    const float2 a1 = make_float2(__uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+    const float2 y0 =
+        __ffma2_rn(a0, __fmul2_rn(sx2, make_float2(cs.x, cs.y)), make_float2(cb.x, cb.y));
+    const float2 y1 =
+        __ffma2_rn(a1, __fmul2_rn(sx2, make_float2(cs.z, cs.w)), make_float2(cb.z, cb.w));
+    o[2 * j] = Num<OutT>::pack2(y0.x, y0.y);
+    o[2 * j + 1] = Num<OutT>::pack2(y1.x, y1.y);
+  }
+  if (acc_dbg != nullptr && row < M) {
+    int32_t* arow = acc_dbg + static_cast<size_t>(row) * N + n0 + c;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (n0 + c + j < N) arow[j] = __float2int_rn(__uint_as_float(r[j]));
+  }
+  if (mapY != nullptr) {
+    uint8_t* sb = staging + (NBUF > 1 ? (store_count & 1) * EPI_BYTES : 0);
+    // The store that last used sb has finished reading it.
+    if (lane == 0) bulk_wait_read<NBUF - 1>();
+    __syncwarp();
+    uint8_t* srow = sb + lane * 64;
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      *reinterpret_cast<uint4*>(srow + ((q ^ sw) << 4)) =
+          make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(mapY, sb, n0 + c, m0 + quarter * 32);
+      bulk_commit();
+    }
+    ++store_count;
+  } else if (row < M) {
+    uint16_t* yrow = static_cast<uint16_t*>(Y) + static_cast<size_t>(row) * N + n0 + c;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (n0 + c + 2 * j < N) yrow[2 * j] = static_cast<uint16_t>(o[j] & 0xFFFFu);
+      if (n0 + c + 2 * j + 1 < N) yrow[2 * j + 1] = static_cast<uint16_t>(o[j] >> 16);
+    }
+  }
+}
+
+// One warp's share of a tile's epilogue: TMEM lanes 32 * quarter .. + 31
+// (the warp's rows) and tile columns [col0, col0 + NCOL).  With PREFETCH the
+// TMEM load of the next 32 columns is issued before the current block is
+// processed, so its latency hides behind the arithmetic and the store (32
+// more registers a thread).  `store_count` counts this warp's stores (it
+// selects the staging buffer).
+template <typename OutT, int NCOL, int NBUF, bool PREFETCH>
+__device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, int col0,
+                                              int lane, int m0, int n0, int M, int N, float sx,
                                               const float* col_scale, const float* col_bias,
                                               uint8_t* staging, const CUtensorMap* mapY,
                                               void* Y, int32_t* acc_dbg, int& store_count) {
-  const int row_in_tile = warp_q * 32 + lane;
-  const int row = m0 + row_in_tile;
-  const uint32_t lane_base = tmem_acc + (static_cast<uint32_t>(warp_q * 32) << 16);
-  uint8_t* my_staging = staging + warp_q * 2 * EPI_BYTES;
+  static_assert(NCOL % (2 * EPI_COLS) == 0, "column share must be an even number of blocks");
+  const uint32_t lane_base = tmem_acc + (static_cast<uint32_t>(quarter * 32) << 16);
+  if (n0 + col0 >= N) return;
+  if (!PREFETCH) {
 #pragma unroll 1
-  for (int c = 0; c < BN; c += EPI_COLS) {
-    if (n0 + c >= N) break;
-    uint32_t r[32];
-    tmem_ld32(lane_base + c, r);
-    tmem_ld_wait();
-    uint32_t o[16];
-    const float2 sx2 = make_float2(sx, sx);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float4 cs = *reinterpret_cast<const float4*>(col_scale + c + 4 * j);
-      const float4 cb = *reinterpret_cast<const float4*>(col_bias + c + 4 * j);
-      const float2 a0 = make_float2(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]));
-      const float2 a1 = make_float2(__uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
-      const float2 y0 = __ffma2_rn(a0, __fmul2_rn(sx2, make_float2(cs.x, cs.y)),
-                                   make_float2(cb.x, cb.y));
-      const float2 y1 = __ffma2_rn(a1, __fmul2_rn(sx2, make_float2(cs.z, cs.w)),
-                                   make_float2(cb.z, cb.w));
-      o[2 * j] = Num<OutT>::pack2(y0.x, y0.y);
-      o[2 * j + 1] = Num<OutT>::pack2(y1.x, y1.y);
+    for (int c = col0; c < col0 + NCOL && n0 + c < N; c += EPI_COLS) {
+      uint32_t r[32];
+      tmem_ld32(lane_base + c, r);
+      tmem_ld_wait_tie(r);
+      epilogue_block<OutT, NBUF>(r, c, quarter, lane, m0, n0, M, N, sx, col_scale, col_bias,
+                                 staging, mapY, Y, acc_dbg, store_count);
     }
-    if (acc_dbg != nullptr && row < M) {
-      int32_t* arow = acc_dbg + static_cast<size_t>(row) * N + n0 + c;
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (n0 + c + j < N) arow[j] = __float2int_rn(__uint_as_float(r[j]));
-    }
-    if (mapY != nullptr) {
-      uint8_t* sb = my_staging + (store_count & 1) * EPI_BYTES;
-      if (lane == 0) bulk_wait_read<1>();  // the store that used sb is done reading
-      __syncwarp();
-      uint8_t* srow = sb + lane * 64;
-      const int sw = (lane >> 1) & 3;
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        *reinterpret_cast<uint4*>(srow + ((q ^ sw) << 4)) =
-            make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        tma_store_2d(mapY, sb, n0 + c, m0 + warp_q * 32);
-        bulk_commit();
-      }
-      ++store_count;
-    } else if (row < M) {
-      uint16_t* yrow = static_cast<uint16_t*>(Y) + static_cast<size_t>(row) * N + n0 + c;
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        if (n0 + c + 2 * j < N) yrow[2 * j] = static_cast<uint16_t>(o[j] & 0xFFFFu);
-        if (n0 + c + 2 * j + 1 < N) yrow[2 * j + 1] = static_cast<uint16_t>(o[j] >> 16);
-      }
-    }
+    return;
+  }
+  uint32_t ra[32], rb[32];
+  tmem_ld32(lane_base + col0, ra);
+#pragma unroll 1
+  for (int c = col0; c < col0 + NCOL; c += 2 * EPI_COLS) {
+    // ra holds block c (issued earlier); warp-uniform conditions throughout.
+    tmem_ld_wait_tie(ra);
+    const bool more1 = n0 + c + EPI_COLS < N;
+    if (more1) tmem_ld32(lane_base + c + EPI_COLS, rb);
+    epilogue_block<OutT, NBUF>(ra, c, quarter, lane, m0, n0, M, N, sx, col_scale, col_bias,
+                               staging, mapY, Y, acc_dbg, store_count);
+    if (!more1) break;
+    tmem_ld_wait_tie(rb);
+    const bool more2 = c + 2 * EPI_COLS < col0 + NCOL && n0 + c + 2 * EPI_COLS < N;
+    if (more2) tmem_ld32(lane_base + c + 2 * EPI_COLS, ra);
+    epilogue_block<OutT, NBUF>(rb, c + EPI_COLS, quarter, lane, m0, n0, M, N, sx, col_scale,
+                               col_bias, staging, mapY, Y, acc_dbg, store_count);
+    if (!more2) break;
   }
 }
 

@@ -15,13 +15,17 @@
 // 128-byte swizzle, or as packed nibbles (APACK / BPACK), which TMA stages and
 // unpack warps expand into that layout.  Warp roles:
 //   warp 4       TMA producer;
-//   warps 6-13   unpack (only when an operand is packed);
+//   warps 6-13   unpack (only when an operand is packed; 448 threads);
 //   warp 5       one lane issues tcgen05.mma (4 x K=32 per stage) and commits
 //                stage and tile completion;
-//   warps 0-3    epilogue, each warp on its own 32 accumulator rows: TMEM ->
-//                registers -> scale, bias, round -> swizzled staging -> TMA
-//                tensor store.  Two TMEM accumulators let the epilogue of
-//                tile i overlap the MMAs of tile i + 1.
+//   warps 0-3    epilogue (and warps 6-9 too when no operand is packed; 320
+//                threads then, so 168 registers a thread): warp w drains accumulator
+//                rows 32 * (w % 4) .. + 31 (the TMEM lanes its SM sub-
+//                partition may read), all 256 columns with four warps, one
+//                half each with eight: TMEM -> registers -> scale, bias,
+//                round -> swizzled staging -> TMA tensor store.  Two TMEM
+//                accumulators let the epilogue of tile i overlap the MMAs of
+//                tile i + 1.
 //   other warps  idle in this phase.
 // With `ready` counters (fused kernel), the producer waits until all rows of
 // a tile's token block have been published before loading its A tiles.
@@ -40,20 +44,33 @@ constexpr int WARP_TMA = 4;
 constexpr int WARP_MMA = 5;
 constexpr int WARP_UNPACK0 = 6;
 constexpr int MIN_THREADS = (WARP_UNPACK0 + NUM_UNPACK / 32) * 32;  // 448
-constexpr int MAX_STAGES = 4;
+constexpr int MAX_STAGES = 6;
 
-template <bool APACK, bool BPACK>
+// Tile BM x BNT (the kernels use BNT = 256).
+template <bool APACK, bool BPACK, int BNT = BN>
 struct Cfg {
   static constexpr bool UNPACK = APACK || BPACK;
-  static constexpr int S = (APACK && BPACK) ? 2 : (UNPACK ? 3 : 4);  // pipeline stages
-  static constexpr size_t OFF_UA = 0;                                 // E4M3 operands
+  static constexpr int EPI_WARPS = UNPACK ? 4 : 8;
+  static constexpr int THREADS = UNPACK ? MIN_THREADS : 320;
+  static constexpr int EPI_THREADS = 32 * EPI_WARPS;
+  static constexpr int EPI_NBUF = 8 / EPI_WARPS;  // staging buffers per warp
+  static constexpr int EPI_NCOL = BNT * 4 / EPI_WARPS;  // columns per warp
+  static constexpr int BU = BNT * BK;    // E4M3 B stage
+  static constexpr int BP = BNT * BKP;   // packed B stage
+  static constexpr int STAGE = A_U + BU + (APACK ? A_P : 0) + (BPACK ? BP : 0);
+  static constexpr int FIXED = EPI_TOTAL + 4 * BNT * 4;
+  static constexpr int S0 = (212 * 1024 - FIXED) / STAGE;
+  static constexpr int S = S0 > MAX_STAGES ? MAX_STAGES : S0;  // pipeline stages
+  static constexpr size_t OFF_UA = 0;                           // E4M3 operands
   static constexpr size_t OFF_UB = OFF_UA + S * A_U;
-  static constexpr size_t OFF_PA = OFF_UB + S * B_U;                  // packed staging
+  static constexpr size_t OFF_PA = OFF_UB + S * BU;             // packed staging
   static constexpr size_t OFF_PB = OFF_PA + (APACK ? S * A_P : 0);
-  static constexpr size_t OFF_EPI = OFF_PB + (BPACK ? S * B_P : 0);
-  static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;              // [2][2][BN] floats
-  static constexpr size_t BYTES = OFF_COL + 4 * BN * sizeof(float);
-  static constexpr uint32_t TX = (APACK ? A_P : A_U) + (BPACK ? B_P : B_U);
+  static constexpr size_t OFF_EPI = OFF_PB + (BPACK ? S * BP : 0);
+  static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;        // [2][2][BNT] floats
+  static constexpr size_t BYTES = OFF_COL + 4 * BNT * sizeof(float);
+  static constexpr uint32_t TX = (APACK ? A_P : A_U) + (BPACK ? BP : BU);
+  static constexpr uint32_t TMEM = 2 * BNT;                     // two accumulators
+  static_assert(S >= 2, "pipeline needs two stages");
 };
 
 struct __align__(8) Barriers {
@@ -85,9 +102,10 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 
 // Barrier init (thread 0) and TMEM allocation (warp WARP_MMA); the caller
 // follows with tcgen05 fences around a CTA barrier.
-template <bool APACK, bool BPACK>
+template <bool APACK, bool BPACK, int BNT = BN>
 __device__ __forceinline__ void setup(Barriers* bars) {
-  constexpr int S = Cfg<APACK, BPACK>::S;
+  using C = Cfg<APACK, BPACK, BNT>;
+  constexpr int S = C::S;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&bars->tma_full[s], 1);
@@ -96,14 +114,14 @@ __device__ __forceinline__ void setup(Barriers* bars) {
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bars->acc_full[s], 1);
-      mbar_init(&bars->acc_empty[s], 128);
+      mbar_init(&bars->acc_empty[s], C::EPI_THREADS);
     }
     mbar_init(&bars->drained, 1);
     bars->abort = 0;
     fence_mbarrier_init();
   }
   if ((threadIdx.x >> 5) == WARP_MMA) {
-    tmem_alloc(&bars->tmem_slot, TMEM_COLS);
+    tmem_alloc(&bars->tmem_slot, C::TMEM);
     tmem_relinquish();
   }
 }
@@ -125,17 +143,19 @@ __device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, ui
   return true;
 }
 
-template <typename OutT, bool APACK, bool BPACK>
+// EPI_PREFETCH: let the epilogue prefetch TMEM (taken only in the 320-thread
+// configuration, where registers allow it).
+template <typename OutT, bool APACK, bool BPACK, int BNT = BN, bool EPI_PREFETCH = true>
 __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
                                          Barriers* bars, uint32_t tmem, const uint32_t* ready) {
-  using C = Cfg<APACK, BPACK>;
+  using C = Cfg<APACK, BPACK, BNT>;
   constexpr int S = C::S;
   volatile int32_t* abort = &bars->abort;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int nk = (g.K + BK - 1) / BK;
-  const int tiles_n = (g.N + BN - 1) / BN;
+  const int tiles_n = (g.N + BNT - 1) / BNT;
   const int tiles = ((g.M + BM - 1) / BM) * tiles_n;
 
   if (warp == WARP_TMA) {
@@ -149,7 +169,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
         const int mb = t / tiles_n;
         const int m0 = mb * BM;
-        const int n0 = (t % tiles_n) * BN;
+        const int n0 = (t % tiles_n) * BNT;
         if (ready != nullptr && mb != ready_m) {
           if (!wait_rows_ready(ready, mb, static_cast<uint32_t>(min(BM, g.M - m0)), abort,
                                g.status)) {
@@ -171,9 +191,9 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
           else
             tma_load_2d(smem + C::OFF_UA + s * A_U, maps.A, kb * BK, m0, &bars->tma_full[s]);
           if (BPACK)
-            tma_load_2d(smem + C::OFF_PB + s * B_P, maps.B, kb * BKP, n0, &bars->tma_full[s]);
+            tma_load_2d(smem + C::OFF_PB + s * C::BP, maps.B, kb * BKP, n0, &bars->tma_full[s]);
           else
-            tma_load_2d(smem + C::OFF_UB + s * B_U, maps.B, kb * BK, n0, &bars->tma_full[s]);
+            tma_load_2d(smem + C::OFF_UB + s * C::BU, maps.B, kb * BK, n0, &bars->tma_full[s]);
         }
       }
       // On an abort, the copies already in flight must land before exit.
@@ -184,7 +204,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
     }
   } else if (warp == WARP_MMA) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
+      constexpr uint32_t idesc = idesc_e4m3_f32(BM, BNT);
       int it = 0, tc = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tc) {
@@ -195,7 +215,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
           break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + buf * BN;
+        const uint32_t d = tmem + buf * BNT;
         for (int kb = 0; kb < nk; ++kb, ++it) {
           const int s = it % S;
           uint64_t* ready_bar = C::UNPACK ? &bars->unpacked[s] : &bars->tma_full[s];
@@ -205,7 +225,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
           }
           tc_fence_after();
           const uint32_t a0 = smem_addr(smem + C::OFF_UA + s * A_U);
-          const uint32_t b0 = smem_addr(smem + C::OFF_UB + s * B_U);
+          const uint32_t b0 = smem_addr(smem + C::OFF_UB + s * C::BU);
 #pragma unroll
           for (int k = 0; k < BK / 32; ++k)
             mma_e4m3(d, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc,
@@ -218,43 +238,22 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       mma_commit(&bars->drained);
       mbar_wait_bounded(&bars->drained, 0, nullptr, nullptr, 10000000ull);
     }
-  } else if (warp >= WARP_UNPACK0 && warp < WARP_UNPACK0 + NUM_UNPACK / 32) {
-    if (C::UNPACK) {
-      const int ut = threadIdx.x - WARP_UNPACK0 * 32;
-      int it = 0;
-      bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        for (int kb = 0; kb < nk; ++kb, ++it) {
-          const int s = it % S;
-          if (!mbar_wait_bounded(&bars->tma_full[s], (it / S) & 1, abort, g.status,
-                                 kWaitLimitNs)) {
-            ok = false;
-            break;
-          }
-          if (APACK)
-            unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * A_U,
-                                        ut);
-          if (BPACK)
-            unpack_rows<BN, NUM_UNPACK>(smem + C::OFF_PB + s * B_P, smem + C::OFF_UB + s * B_U,
-                                        ut);
-          fence_proxy_async_smem();
-          mbar_arrive(&bars->unpacked[s]);
-        }
-      }
-    }
-  } else if (warp < 4) {
-    // ---- epilogue warps 0-3 ----
-    const int et = threadIdx.x;  // 0..127
+  } else if (warp < 4 || (C::EPI_WARPS == 8 && warp >= 6 && warp < 10)) {
+    // ---- epilogue ----
+    const int quarter = warp & 3;
+    const int part = warp < 4 ? 0 : 1;                // 0: warps 0-3, 1: warps 6-9
+    const int et = part * 128 + quarter * 32 + lane;  // 0 .. EPI_THREADS - 1
+    uint8_t* staging = smem + C::OFF_EPI + (part * 4 + quarter) * C::EPI_NBUF * EPI_BYTES;
     int tc = 0, stores = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tc) {
       const int m0 = (t / tiles_n) * BM;
-      const int n0 = (t % tiles_n) * BN;
+      const int n0 = (t % tiles_n) * BNT;
       const int buf = tc & 1;
       // Column data of this tile into the buffer of its parity; the buffer of
       // the other parity may still be read by slower warps (previous tile).
-      float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL) + buf * 2 * BN;
-      float* col_bias = col_scale + BN;
-      for (int j = et; j < BN; j += 128) {
+      float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL) + buf * 2 * BNT;
+      float* col_bias = col_scale + BNT;
+      for (int j = et; j < BNT; j += C::EPI_THREADS) {
         const int col = n0 + j;
         float sc = 0.f, bi = 0.f;
         if (col < g.N) {
@@ -267,27 +266,50 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       bool ok = mbar_wait_bounded(&bars->acc_full[buf], (tc >> 1) & 1, abort, g.status,
                                   kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok);
-      named_bar_sync(kEpiBarrier, 128);  // column data of this tile written
+      named_bar_sync(kEpiBarrier, C::EPI_THREADS);  // column data of this tile written
       if (!ok || *abort != 0) break;
       tc_fence_after();
       // s_x may have been written by other CTAs of this grid (fused kernel):
       // read it from L2, after the tile's MMAs have completed.
-      const int row = m0 + et;
+      const int row = m0 + quarter * 32 + lane;
       const float sx = row < g.M ? __ldcg(g.s_x + row) : 0.f;
-      epilogue_tile<OutT>(tmem + buf * BN, warp, lane, m0, n0, g.M, g.N, sx, col_scale,
-                          col_bias, smem + C::OFF_EPI, maps.Y, g.Y, g.acc_dbg, stores);
+      epilogue_part<OutT, C::EPI_NCOL, C::EPI_NBUF, EPI_PREFETCH && !C::UNPACK>(
+          tmem + buf * BNT, quarter, part * C::EPI_NCOL, lane, m0, n0, g.M, g.N, sx, col_scale,
+          col_bias, staging, maps.Y, g.Y, g.acc_dbg, stores);
       tc_fence_before();
       mbar_arrive(&bars->acc_empty[buf]);
     }
     if (lane == 0) bulk_wait_all();
+  } else if (C::UNPACK && warp >= WARP_UNPACK0 && warp < WARP_UNPACK0 + NUM_UNPACK / 32) {
+    const int ut = threadIdx.x - WARP_UNPACK0 * 32;
+    int it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int s = it % S;
+        if (!mbar_wait_bounded(&bars->tma_full[s], (it / S) & 1, abort, g.status,
+                               kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        if (APACK)
+          unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * A_U,
+                                      ut);
+        if (BPACK)
+          unpack_rows<BNT, NUM_UNPACK>(smem + C::OFF_PB + s * C::BP,
+                                       smem + C::OFF_UB + s * C::BU, ut);
+        fence_proxy_async_smem();
+        mbar_arrive(&bars->unpacked[s]);
+      }
+    }
   }
 }
 
 // After a CTA barrier that follows pipeline(): release TMEM.
-__device__ __forceinline__ void teardown(uint32_t tmem) {
+__device__ __forceinline__ void teardown(uint32_t tmem, uint32_t cols) {
   if ((threadIdx.x >> 5) == WARP_MMA) {
     tc_fence_after();
-    tmem_dealloc(tmem, TMEM_COLS);
+    tmem_dealloc(tmem, cols);
   }
 }
 

@@ -292,23 +292,30 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem, int
     float m = 0.f;
 #pragma unroll
     for (int k = 0; k < 16; ++k) m = fmaxf(m, fmaxf(fabsf(v[k].x), fabsf(v[k].y)));
+    // Lanes of this warp on the same row; padding lanes (tid >= items) only
+    // keep the shuffles convergent, their values are not data of any row and
+    // must not reach a row maximum.
+    const unsigned grp = __match_any_sync(0xffffffffu, active ? r_local : -1);
+    const int leader = __ffs(grp) - 1;
     {
-      // Padding lanes (tid >= items) only keep the shuffles convergent; their
-      // values are not data of any row and must not reach a row maximum.
-      const int key = active ? r_local : -1;
-      const unsigned grp = __match_any_sync(0xffffffffu, key);
       const unsigned mx = __reduce_max_sync(grp, __float_as_uint(m));
-      if (active && lane == __ffs(grp) - 1) atomicMax(&sh.amax[par * R + r_local], mx);
+      if (active && lane == leader) atomicMax(&sh.amax[par * R + r_local], mx);
     }
     __syncthreads();
 
     // ---- phase 3: scale, codes, pack, store --------------------------------
     if (active && r_local < rows) {
       const int row = row0 + r_local;
-      float amax = __uint_as_float(sh.amax[par * R + r_local]);
-      if (CLIP) amax = fminf(amax, __ldg(a.clip + row));
-      const float s_row = __fdiv_rn(amax, 7.0f);
-      const float rcp = s_row > 0.f ? __frcp_rn(s_row) : 0.f;
+      // One lane per (row, warp) computes the scale and its reciprocal.
+      float s_row = 0.f, rcp = 0.f;
+      if (lane == leader) {
+        float amax = __uint_as_float(sh.amax[par * R + r_local]);
+        if (CLIP) amax = fminf(amax, __ldg(a.clip + row));
+        s_row = __fdiv_rn(amax, 7.0f);
+        rcp = s_row > 0.f ? __frcp_rn(s_row) : 0.f;
+      }
+      s_row = __shfl_sync(grp, s_row, leader);
+      rcp = __shfl_sync(grp, rcp, leader);
       const float2 rc2 = make_float2(rcp, rcp);
       const float2 magic = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
       if (a.e4m3) {

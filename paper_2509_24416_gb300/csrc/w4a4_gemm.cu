@@ -16,15 +16,13 @@ namespace {
 
 using namespace gemm;
 
-constexpr int THREADS = MIN_THREADS;  // 448
-
-template <bool APACK, bool BPACK>
+template <bool APACK, bool BPACK, int BNT>
 constexpr size_t smem_bytes() {
-  return Cfg<APACK, BPACK>::BYTES + 1024;  // + alignment slack
+  return Cfg<APACK, BPACK, BNT>::BYTES + 1024;  // + alignment slack
 }
 
-template <typename OutT, bool APACK, bool BPACK>
-__global__ void __launch_bounds__(THREADS, 1)
+template <typename OutT, bool APACK, bool BPACK, int BNT>
+__global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT>::THREADS), 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                      const __grid_constant__ CUtensorMap mapB,
                      const __grid_constant__ CUtensorMap mapY, GemmArgs g, int use_tma_store) {
@@ -32,16 +30,16 @@ __global__ void __launch_bounds__(THREADS, 1)
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  setup<APACK, BPACK>(&bars);
+  setup<APACK, BPACK, BNT>(&bars);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars.tmem_slot;
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
-  pipeline<OutT, APACK, BPACK>(maps, g, smem, &bars, tmem, nullptr);
+  pipeline<OutT, APACK, BPACK, BNT>(maps, g, smem, &bars, tmem, nullptr);
   tc_fence_before();
   __syncthreads();
-  teardown(tmem);
+  teardown(tmem, Cfg<APACK, BPACK, BNT>::TMEM);
 }
 
 // Packed INT4 weights -> E4M3 execution layout (one code per byte, the byte
@@ -142,15 +140,16 @@ cudaError_t kernel_setup(const void* func, size_t smem, int threads, int* per_sm
 
 namespace {
 
-template <typename OutT, bool APACK, bool BPACK>
+template <typename OutT, bool APACK, bool BPACK, int BNT>
 cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB,
                           const CUtensorMap& mapY, const GemmArgs& g, int use_tma_store,
                           int grid, cudaStream_t st) {
-  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK>;
-  constexpr size_t smem = smem_bytes<APACK, BPACK>();
-  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, THREADS, nullptr);
+  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT>;
+  constexpr size_t smem = smem_bytes<APACK, BPACK, BNT>();
+  constexpr int threads = Cfg<APACK, BPACK, BNT>::THREADS;
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, threads, nullptr);
   if (e != cudaSuccess) return e;
-  k<<<grid, THREADS, smem, st>>>(mapA, mapB, mapY, g, use_tma_store);
+  k<<<grid, threads, smem, st>>>(mapA, mapB, mapY, g, use_tma_store);
   return cudaGetLastError();
 }
 
@@ -159,10 +158,13 @@ cudaError_t launch_gemm_dt(const CUtensorMap& mapA, const CUtensorMap& mapB,
                            const CUtensorMap& mapY, const GemmArgs& g, bool apack, bool bpack,
                            int use_tma_store, int grid, cudaStream_t st) {
   if (apack)
-    return bpack ? launch_gemm_t<OutT, true, true>(mapA, mapB, mapY, g, use_tma_store, grid, st)
-                 : launch_gemm_t<OutT, true, false>(mapA, mapB, mapY, g, use_tma_store, grid, st);
-  return bpack ? launch_gemm_t<OutT, false, true>(mapA, mapB, mapY, g, use_tma_store, grid, st)
-               : launch_gemm_t<OutT, false, false>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+    return bpack ? launch_gemm_t<OutT, true, true, BN>(mapA, mapB, mapY, g, use_tma_store, grid,
+                                                       st)
+                 : launch_gemm_t<OutT, true, false, BN>(mapA, mapB, mapY, g, use_tma_store, grid,
+                                                        st);
+  if (bpack)
+    return launch_gemm_t<OutT, false, true, BN>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+  return launch_gemm_t<OutT, false, false, BN>(mapA, mapB, mapY, g, use_tma_store, grid, st);
 }
 
 }  // namespace
@@ -181,9 +183,17 @@ bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows
 
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st) {
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
+  const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
+  // 256-wide tiles: measured faster than 128-wide ones even where 128 fills
+  // the last wave of tiles better (the narrower tile moves more operand bytes
+  // through shared memory per multiply-add).
+  const int bn = BN;
   CUtensorMap mapA, mapB, mapY;
   if (!encode_codes_map(&mapA, Xq, x_codes, g.M, g.K, BM) ||
-      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, BN))
+      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn))
     return cudaErrorInvalidValue;
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
   if (use_tma_store) {
@@ -191,16 +201,13 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   } else {
     mapY = mapA;  // unused
   }
-  const int tiles = ((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN);
-  const int sms = sm_count();
-  if (sms <= 0) return cudaErrorInvalidDevice;
+  const int tiles = ((g.M + BM - 1) / BM) * ((g.N + bn - 1) / bn);
   const int grid = std::min(tiles, sms);
-  const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
-  const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
   if (out_dtype == CLQ_F16)
-    return launch_gemm_dt<__half>(mapA, mapB, mapY, g, apack, bpack, use_tma_store, grid, st);
-  return launch_gemm_dt<__nv_bfloat16>(mapA, mapB, mapY, g, apack, bpack, use_tma_store, grid,
-                                       st);
+    return launch_gemm_dt<__half>(mapA, mapB, mapY, g, apack, bpack, use_tma_store, grid,
+                                  st);
+  return launch_gemm_dt<__nv_bfloat16>(mapA, mapB, mapY, g, apack, bpack, use_tma_store,
+                                       grid, st);
 }
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st) {
