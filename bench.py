@@ -70,19 +70,31 @@ def peaks():
         return 6800.0, 1900.0, "fallback"
 
 
-def kernel_source_sha():
-    h = hashlib.sha256()
+# Source files each kernel is built from (globs under csrc/): a recorded ncu
+# figure stays valid while these files are unchanged.
+KERNEL_SOURCES = {
+    "w4a4_gemm": ("w4a4_gemm.cu", "gemm_*.cuh", "clq_device.cuh", "clq_kernels.h"),
+    "rotate_quant": ("rotate_quant*.cu", "rq_*.cuh", "clq_device.cuh", "clq_kernels.h"),
+    "fused_linear": ("fused_linear.cu", "gemm_*.cuh", "rq_*.cuh", "clq_device.cuh",
+                     "clq_kernels.h"),
+}
+
+
+def kernel_source_sha(kernel):
+    import glob
     csrc = os.path.join(ROOT, "paper_2509_24416_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + f.read())
+    files = sorted({f for pat in KERNEL_SOURCES[kernel]
+                    for f in glob.glob(os.path.join(csrc, pat))})
+    h = hashlib.sha256()
+    for path in files:
+        with open(path, "rb") as f:
+            h.update(os.path.basename(path).encode() + f.read())
     return h.hexdigest()[:16]
 
 
 def recorded_traffic(kernel, workload):
     """DRAM bytes per launch from a committed ncu summary, if it was taken
-    on the current kernel sources; else None."""
+    on the kernel's current sources; else None."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.json")
     try:
         with open(path) as f:
@@ -90,7 +102,7 @@ def recorded_traffic(kernel, workload):
     except (OSError, ValueError):
         return None
     e = d.get(kernel, {}).get(workload)
-    if not e or e.get("source_sha") != kernel_source_sha():
+    if not e or e.get("source_sha") != kernel_source_sha(kernel):
         return None
     return e.get("bytes_per_launch")
 
