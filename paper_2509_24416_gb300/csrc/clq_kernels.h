@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -25,7 +26,8 @@ struct RotateQuantArgs {
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
                                 cudaStream_t st);
-void rotate_quant_config(int K, int* rows_per_tile, int* threads, size_t* smem);
+void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads,
+                         size_t* smem);
 cudaError_t launch_outlier_scores(const void* calib, int dtype, int B, int T, int K,
                                   float* scores, cudaStream_t st);
 
@@ -78,5 +80,25 @@ bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows
 // device, and (per_sm != null) return its occupancy for (threads, smem),
 // cached, so that launches make no per-call attribute queries.
 cudaError_t kernel_setup(const void* func, size_t smem, int threads, int* per_sm);
+
+// Launch with programmatic stream serialization: the kernel may start while
+// the previous kernel on `st` finishes and must call pdl_wait() before it
+// reads global memory.  (Only kernel-to-kernel edges overlap; after a copy or
+// a memset the launch waits as usual.)
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), int grid, int threads, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(static_cast<unsigned>(threads));
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 }  // namespace clq

@@ -45,13 +45,18 @@ struct PublishRows {
   }
 };
 
+// Rotate-quant stage geometry of the fused kernel: its shared memory is sized
+// for the GEMM pipeline anyway, so 32 KB stages let 512 threads cover as many
+// rows per tile as they can (14 rows at K = 1152, 3 at K = 4608).
+constexpr int kRqStride = 32 * 1024;
+constexpr int kRqStages = 4;
+
 template <typename T, bool BPACK, int BNT>
 __global__ void __launch_bounds__(FT, 1)
     fused_linear_kernel(const __grid_constant__ CUtensorMap mapA,
                         const __grid_constant__ CUtensorMap mapB,
                         const __grid_constant__ CUtensorMap mapY, RotateQuantArgs rq, GemmArgs g,
-                        uint32_t* ready, uint32_t* tile_counter, int use_tma_store,
-                        int rq_stages) {
+                        uint32_t* ready, uint32_t* tile_counter, int use_tma_store) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -62,7 +67,7 @@ __global__ void __launch_bounds__(FT, 1)
   tc_fence_after();
   const uint32_t tmem = bars.tmem_slot;
 
-  rq::run<T, -1, false>(rq, smem, rq_stages, tile_counter, PublishRows{ready});
+  rq::run<T, -1, false, kRqStride, kRqStages>(rq, smem, tile_counter, PublishRows{ready});
   __syncthreads();
 
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
@@ -75,15 +80,15 @@ __global__ void __launch_bounds__(FT, 1)
 template <typename T, bool BPACK, int BNT>
 cudaError_t launch_t(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                      const RotateQuantArgs& rq, const GemmArgs& g, uint32_t* ready,
-                     int use_tma_store, int rq_stages, size_t smem, int grid, cudaStream_t st) {
+                     int use_tma_store, size_t smem, int grid, cudaStream_t st) {
   uint32_t* tile_counter = ready + (g.M + BM - 1) / BM;
   auto k = fused_linear_kernel<T, BPACK, BNT>;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, FT, nullptr);
   if (e != cudaSuccess) return e;
-  k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store,
-                             rq_stages);
+  k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store);
   return cudaGetLastError();
 }
+
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
@@ -108,19 +113,17 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   const int bn = BN;
   const size_t gemm_bytes = bpack ? Cfg<false, true>::BYTES : Cfg<false, false>::BYTES;
   const size_t limit = 227u * 1024u - 2048u;  // dynamic + static shared memory
-  // Rotate-quant phase: as many rows per tile as 512 threads cover, then as
-  // many raw stages (2..4) as fit next to them.
+  // Rotate-quant phase: as many rows per tile as 512 threads cover and one
+  // raw stage holds.
   RotateQuantArgs rq = rq_in;
   rq.logb = logb;
   rq.e4m3 = 1;  // the workspace holds the codes in the GEMM's operand layout
   const int segs = rq.K / 32;
-  int R = std::max(1, FT / segs);
-  int stages = rq::kMaxStages;
-  while (stages > 2 && rq::smem_bytes(rq.K, R, stages) > limit) --stages;
-  while (R > 1 && rq::smem_bytes(rq.K, R, stages) > limit) --R;
-  if (rq::smem_bytes(rq.K, R, stages) > limit || R * segs > FT) return cudaErrorInvalidValue;
+  const int R = std::max(1, std::min(FT / segs, kRqStride / (2 * rq.K)));
+  const size_t rq_bytes = rq::smem_bytes(R, kRqStride, kRqStages);
+  if (rq_bytes > limit || R * segs > FT) return cudaErrorInvalidValue;
   rq.rows_per_tile = R;
-  const size_t smem = std::max(gemm_bytes, rq::smem_bytes(rq.K, R, stages)) + 1024;
+  const size_t smem = std::max(gemm_bytes, rq_bytes) + 1024;
 
   const int tiles_m = (g.M + BM - 1) / BM;
   cudaError_t e =
@@ -140,13 +143,13 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   const int grid = sms;
   if (dtype == CLQ_F16)
     return bpack ? launch_t<__half, true, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                              stages, smem, grid, st)
+                                              smem, grid, st)
                  : launch_t<__half, false, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                               stages, smem, grid, st);
+                                               smem, grid, st);
   return bpack ? launch_t<__nv_bfloat16, true, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                                   stages, smem, grid, st)
+                                                   smem, grid, st)
                : launch_t<__nv_bfloat16, false, BN>(mapA, mapB, mapY, rq, g, ready,
-                                                    use_tma_store, stages, smem, grid, st);
+                                                    use_tma_store, smem, grid, st);
 }
 
 }  // namespace clq

@@ -1,18 +1,11 @@
-// Standalone rotate-quantize kernel (activations online, weights offline)
-// and the outlier-score kernel.  The tile loop itself lives in rq_device.cuh.
-#include "rq_device.cuh"
+// Rotate-quantize launch configuration and dispatch (the kernels are in
+// rotate_quant_f16.cu / rotate_quant_bf16.cu, the tile loop in
+// rq_device.cuh) and the outlier-score kernel.
+#include "rq_launch.cuh"
 
 namespace clq {
 
 namespace {
-
-constexpr int kStages = rq::kMaxStages;  // raw tiles in flight per CTA
-
-template <typename T, int LOGB, bool CLIP>
-__global__ void __maxnreg__(96) rotate_quant_kernel(RotateQuantArgs a) {
-  extern __shared__ __align__(16) uint8_t smem[];
-  rq::run<T, LOGB, CLIP>(a, smem, kStages, nullptr, rq::NoPublish());
-}
 
 // Outlier score (Sec. 3.3): S = fp32 batch mean (sequential sum over the
 // batch, then / B), score[k] = max_t |S[t][k]|.  Threads own channels;
@@ -37,63 +30,44 @@ __global__ void outlier_scores_kernel(const uint16_t* calib, int B, int Tn, int 
   atomicMax(reinterpret_cast<unsigned*>(scores) + k, __float_as_uint(best));
 }
 
-template <typename T, int LOGB, bool CLIP>
-cudaError_t launch_rq_t(const RotateQuantArgs& a, int threads, size_t smem, int sms,
-                        cudaStream_t st) {
-  auto kern = rotate_quant_kernel<T, LOGB, CLIP>;
-  int per_sm = 0;
-  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(kern), smem, threads, &per_sm);
-  if (e != cudaSuccess) return e;
-  if (per_sm < 1) return cudaErrorInvalidConfiguration;
-  const int ntiles = (a.M + a.rows_per_tile - 1) / a.rows_per_tile;
-  const int g = std::min(ntiles, sms * per_sm);
-  kern<<<g, threads, smem, st>>>(a);
-  return cudaGetLastError();
-}
-
-template <typename T, bool CLIP>
-cudaError_t launch_rq_b(const RotateQuantArgs& a, int logb, int threads, size_t smem, int sms,
-                        cudaStream_t st) {
-  switch (logb) {
-    case 0: return launch_rq_t<T, 0, CLIP>(a, threads, smem, sms, st);
-    case 1: return launch_rq_t<T, 1, CLIP>(a, threads, smem, sms, st);
-    case 2: return launch_rq_t<T, 2, CLIP>(a, threads, smem, sms, st);
-    case 3: return launch_rq_t<T, 3, CLIP>(a, threads, smem, sms, st);
-    case 4: return launch_rq_t<T, 4, CLIP>(a, threads, smem, sms, st);
-    case 5: return launch_rq_t<T, 5, CLIP>(a, threads, smem, sms, st);
-    case 6: return launch_rq_t<T, 6, CLIP>(a, threads, smem, sms, st);
-    case 7: return launch_rq_t<T, 7, CLIP>(a, threads, smem, sms, st);
-    case 8: return launch_rq_t<T, 8, CLIP>(a, threads, smem, sms, st);
-    default: return cudaErrorInvalidValue;
-  }
-}
-
 }  // namespace
 
 // Rows per tile: the CTA gets one thread per 32-element segment of each of
-// its rows.  Prefer thread counts that fill whole warps (padding lanes do no
-// useful work) and lie in [192, 384], which keeps two CTAs per SM, and keep
-// the shared-memory footprint (S + 1 row buffers) under 113 KB.
-void rotate_quant_config(int K, int* rows_per_tile, int* threads, size_t* smem) {
+// its rows, R rows fitting one raw stage (2 R K bytes).  At 128 registers a
+// thread an SM holds 16 warps.  R is chosen by a cost model fitted to timings
+// on GB300 (M up to 65536 tokens): a CTA takes about max(1.2, 0.1 + 0.121 W)
+// us per tile when W warps share the SM (a latency floor, then issue-bound),
+// every CTA walks ceil(tiles / CTAs) tiles, and the first tile's arrival adds
+// about 0.7 us per 2304-byte row.  Few rows per tile win when M is small (more
+// CTAs share the work), many when M is large.
+void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads,
+                         size_t* smem) {
   const int segs = K >> 5;
+  const bool large = rq::large_rows(K);
+  const int stride = large ? rq::kStrideLarge : rq::kStrideSmall;
+  const int stages = large ? rq::kStagesLarge : rq::kStagesSmall;
   int best_r = 1;
-  double best_score = -1.0;
-  for (int r = 1; r * segs <= 512; ++r) {
-    if (r > 1 && rq::smem_bytes(K, r, kStages) > 113u * 1024u) break;
-    const int t = r * segs;
-    const int t32 = (t + 31) & ~31;
-    const double fill = static_cast<double>(t) / t32;
-    const double size_term =
-        t32 < 192 ? t32 / 384.0 : (t32 <= 384 ? 1.0 + t32 / 4096.0 : 0.5);
-    const double score = fill * 4.0 + size_term;
-    if (score > best_score + 1e-9) {
-      best_score = score;
+  double best_cost = 1e300;
+  for (int r = 1; r * segs <= 512 && 2 * r * K <= stride; ++r) {
+    const int warps = (r * segs + 31) / 32;
+    const size_t bytes = rq::smem_bytes(r, stride, stages);
+    const int by_warps = (65536 / (32 * rq::kMaxRegs)) / warps;
+    const int by_smem = static_cast<int>((227u * 1024u) / (bytes + 1024u));
+    const int ctas = std::min(by_warps, by_smem);
+    if (ctas < 1) continue;
+    const long tiles = (static_cast<long>(M) + r - 1) / r;
+    const long total = static_cast<long>(ctas) * std::max(sms, 1);
+    const long rounds = (tiles + total - 1) / total;
+    const double cost =
+        rounds * std::max(1.2, 0.1 + 0.121 * ctas * warps) + 0.7 * r * (2.0 * K) / 2304.0;
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
       best_r = r;
     }
   }
   *rows_per_tile = best_r;
   *threads = ((best_r * segs) + 31) & ~31;
-  *smem = rq::smem_bytes(K, best_r, kStages);
+  *smem = rq::smem_bytes(best_r, stride, stages);
 }
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
@@ -101,15 +75,11 @@ cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
   RotateQuantArgs args = a;
   int threads = 0;
   size_t smem = 0;
-  rotate_quant_config(a.K, &args.rows_per_tile, &threads, &smem);
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
-  const bool clip = a.clip != nullptr;
-  if (dtype == CLQ_F16)
-    return clip ? launch_rq_b<__half, true>(args, logb, threads, smem, sms, st)
-                : launch_rq_b<__half, false>(args, logb, threads, smem, sms, st);
-  return clip ? launch_rq_b<__nv_bfloat16, true>(args, logb, threads, smem, sms, st)
-              : launch_rq_b<__nv_bfloat16, false>(args, logb, threads, smem, sms, st);
+  rotate_quant_config(a.M, a.K, sms, &args.rows_per_tile, &threads, &smem);
+  if (dtype == CLQ_F16) return launch_rotate_quant_f16(args, logb, threads, smem, sms, st);
+  return launch_rotate_quant_bf16(args, logb, threads, smem, sms, st);
 }
 
 cudaError_t launch_outlier_scores(const void* calib, int dtype, int B, int T, int K,

@@ -35,6 +35,9 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT>::THREADS), 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars.tmem_slot;
+  // Barriers and TMEM are set up; global inputs are read only from here on.
+  pdl_wait();
+  pdl_launch_dependents();
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
   pipeline<OutT, APACK, BPACK, BNT>(maps, g, smem, &bars, tmem, nullptr);
   tc_fence_before();
@@ -149,8 +152,7 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB,
   constexpr int threads = Cfg<APACK, BPACK, BNT>::THREADS;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, threads, nullptr);
   if (e != cudaSuccess) return e;
-  k<<<grid, threads, smem, st>>>(mapA, mapB, mapY, g, use_tma_store);
-  return cudaGetLastError();
+  return launch_pdl(k, grid, threads, smem, st, mapA, mapB, mapY, g, use_tma_store);
 }
 
 template <typename OutT>
