@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--impl", default="clq", choices=["clq", "reference"])
     p.add_argument("--workload", default="pixart_1024")
     p.add_argument("--fused", action="store_true")
+    p.add_argument("--sweep", action="store_true",
+                   help="time the 100-cell M x (K, N) x b grid, one JSON line per cell")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--layer", default=None,
@@ -251,11 +253,135 @@ def config_dict(cfg, args):
             "l2": "inputs rotated over sets totalling > 2x L2 (129 MB)"}
 
 
+# ------------------------------------------------------------------ sweep ---
+SWEEP_M = (256, 1024, 4096, 16384, 65536)
+SWEEP_KN = ((1152, 1152), (1152, 4608), (4608, 1152), (3072, 12288), (12288, 3072))
+SWEEP_B = (32, 64, 128, 256)
+
+
+def run_sweep(args):
+    """The 100-cell grid: M x (K, N) x b, each valid cell timed as
+    rotate-quant alone, rotate-quant + GEMM, the fused kernel and fp16 cuBLAS
+    (torch.addmm, independent of b), with inputs of the 256-token case's
+    distribution (N(0, 1), 8 channels x 40) generated on the device from a
+    fixed seed and rotated over sets larger than L2.  One JSON line per cell."""
+    import torch
+    from paper_2509_24416_gb300 import clq
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    clq.load()
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    gen = torch.Generator(device=dev)
+
+    def timed(fn, est_us):
+        reps = int(min(50, max(5, 200000.0 / max(est_us, 1.0))))
+        for k in range(3):
+            fn(k)
+        torch.cuda.synchronize()
+        a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for k in range(reps):
+            fn(k)
+        z.record(stream)
+        torch.cuda.synchronize()
+        return 1e3 * a.elapsed_time(z) / reps
+
+    for (K, N) in SWEEP_KN:
+        gen.manual_seed(1)
+        W = (torch.randn(N, K, device=dev, generator=gen) * 0.02).half()
+        bias = (torch.randn(N, device=dev, generator=gen) * 0.01).half()
+        # outlier scores without ties (a calibration mean never ties exactly):
+        # U(0, 1) for ordinary channels, 40 for the 8 outlier channels
+        cg = torch.Generator().manual_seed(3)
+        scores = torch.rand(K, generator=cg)
+        scores[torch.randperm(K, generator=cg)[:8]] = 40.0
+        perm = clq.build_permutation(scores).to(dev)
+        prepared = {b: clq.PreparedLinear.from_weight(W, perm, b, bias=bias)
+                    for b in SWEEP_B if K % b == 0}
+        for M in SWEEP_M:
+            xbytes = M * K * 2
+            nsets = max(2, math.ceil(2 * L2_BYTES / xbytes) + 1)
+            gen.manual_seed(0)
+            outl = (scores > 2).to(dev)
+            xs = []
+            for _ in range(nsets):
+                x = torch.randn(M, K, device=dev, generator=gen)
+                x[:, outl] *= 40.0
+                xs.append(x.half())
+                del x
+            Y = torch.empty((M, N), dtype=torch.float16, device=dev)
+            xq = torch.empty((M, K), dtype=torch.uint8, device=dev)
+            s_x = torch.empty(M, dtype=torch.float32, device=dev)
+            ws = clq.fused_workspace(M, K, dev)
+            ops = 2.0 * M * N * K
+            cub_us = timed(lambda k: torch.addmm(bias, xs[k % nsets], W.t(), out=Y),
+                           ops / 1.5e6)
+            for b in SWEEP_B:
+                cell = {"M": M, "K": K, "N": N, "b": b}
+                if K % b:
+                    cell.update({"valid": False, "reason": "K % b != 0"})
+                    print(json.dumps(cell), flush=True)
+                    continue
+                lay = prepared[b]
+
+                def rq(k):
+                    st = clq.clq_rotate_quant_act(xs[k % nsets].data_ptr(), clq.CLQ_F16, M, K, K,
+                                                  perm.data_ptr(), b, clq.CLQ_CODES_E4M3,
+                                                  xq.data_ptr(), s_x.data_ptr(), None, sp)
+                    if st:
+                        raise clq.ClqError(st, "clq_rotate_quant_act")
+
+                def sep(k):
+                    rq(k)
+                    st = clq.clq_w4a4_linear(xq.data_ptr(), clq.CLQ_CODES_E4M3, s_x.data_ptr(),
+                                             lay.We.data_ptr(), clq.CLQ_CODES_E4M3,
+                                             lay.s_w.data_ptr(), lay.bias.data_ptr(), M, N, K, b,
+                                             clq.CLQ_F16, Y.data_ptr(), None, sp)
+                    if st:
+                        raise clq.ClqError(st, "clq_w4a4_linear")
+
+                def fused(k):
+                    st = clq.clq_fused_linear(xs[k % nsets].data_ptr(), clq.CLQ_F16, M, K, K,
+                                              perm.data_ptr(), b, lay.We.data_ptr(),
+                                              clq.CLQ_CODES_E4M3, lay.s_w.data_ptr(),
+                                              lay.bias.data_ptr(), N, Y.data_ptr(),
+                                              ws.data_ptr(), ws.numel(), sp)
+                    if st:
+                        raise clq.ClqError(st, "clq_fused_linear")
+
+                rq_us = timed(rq, xbytes / 3e6)
+                sep_us = timed(sep, ops / 2.5e6 + rq_us)
+                fu_us = timed(fused, ops / 2.5e6 + rq_us)
+                cell.update({
+                    "valid": True,
+                    "rotate_quant_us": round(rq_us, 2),
+                    "rotate_quant_GBps": round(M * (3.0 * K + 4) / (rq_us * 1e-6) / 1e9, 1),
+                    "separate_us": round(sep_us, 2),
+                    "separate_TOPS": round(ops / (sep_us * 1e-6) / 1e12, 1),
+                    "fused_us": round(fu_us, 2),
+                    "fused_TOPS": round(ops / (fu_us * 1e-6) / 1e12, 1),
+                    "fp16_cublas_us": round(cub_us, 2),
+                    "fp16_cublas_TOPS": round(ops / (cub_us * 1e-6) / 1e12, 1),
+                    "speedup_separate_vs_cublas": round(cub_us / sep_us, 3),
+                    "speedup_fused_vs_cublas": round(cub_us / fu_us, 3),
+                })
+                print(json.dumps(cell), flush=True)
+            del xs, Y, xq, s_x, ws
+            torch.cuda.empty_cache()
+    status = clq.device_status()
+    if status != 0:
+        raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
+
+
 # --------------------------------------------------------------- GPU arm ---
 def main():
     args = parse()
     if args.impl == "reference":
         reference_arm(args)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
     import torch
     import torch.distributed as dist
@@ -281,7 +407,7 @@ def main():
     M = cfg["M"]
 
     # ---- offline: calibration, swap vectors, prepared weights (untimed) ----
-    layers, xs_host = [], []
+    layers, xs_host, w_dense = [], [], []
     all_names = [l[0] for l in synth.WORKLOADS[args.workload]["layers"]]
     for lname, _, _ in cfg["layers"]:
         li = all_names.index(lname)
@@ -292,6 +418,7 @@ def main():
                                              bias=d["bias"].to(dev))
         layers.append((d["name"], d["K"], d["N"], lay))
         xs_host.append(d["X"])
+        w_dense.append((d["W"].to(dev), d["bias"].to(dev)))  # fp16 cuBLAS comparator
     set_bytes = sum(x.numel() * 2 for x in xs_host)
     nsets = max(2, math.ceil(2 * L2_BYTES / set_bytes) + 1)
     xsets = [[x.to(dev) for x in xs_host] for _ in range(nsets)]
@@ -303,15 +430,16 @@ def main():
     sp = stream.cuda_stream
     nlay = len(layers)
 
-    def step(si, ev=None):
+    def step(si, ev=None, fused=None):
+        fused = args.fused if fused is None else fused
         xs = xsets[si % nsets]
         for i, (_, K, N, lay) in enumerate(layers):
             if ev is not None:
                 ev[4 * i].record(stream)
-                if args.fused:  # one kernel: its time is the "gemm" interval
+                if fused:  # one kernel: its time is the "gemm" interval
                     ev[4 * i + 1].record(stream)
                     ev[4 * i + 2].record(stream)
-            if args.fused:
+            if fused:
                 st = clq.clq_fused_linear(xs[i].data_ptr(), clq._dt(xs[i]), M, K, K,
                                           lay.perm.data_ptr(), b, lay.We.data_ptr(),
                                           clq.CLQ_CODES_E4M3, lay.s_w.data_ptr(),
@@ -386,6 +514,30 @@ def main():
         step(k, evs[k])
     torch.cuda.synchronize()
     clocks = sampler.stop()
+
+    # ---- context (not part of value): the other path, fp16 cuBLAS on the
+    # same layer shapes and rotated inputs, measured peak rates ----
+    def time_steps(fn, n):
+        for k in range(3):
+            fn(k)
+        torch.cuda.synchronize()
+        a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for k in range(n):
+            fn(k)
+        z.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(z) / n
+
+    other_ms = time_steps(lambda k: step(k, fused=not args.fused), args.steps)
+
+    def cublas_step(si):
+        xs = xsets[si % nsets]
+        for i, (w, bias) in enumerate(w_dense):
+            torch.addmm(bias, xs[i], w.t(), out=ys[i])
+
+    cublas_ms = time_steps(cublas_step, args.steps)
+    measured = clq.measure_peaks()
     status = clq.device_status()
     if status != 0:
         raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
@@ -428,6 +580,8 @@ def main():
     rq_bytes_all = sum(M * (3.0 * K + 4) for K in K_list)
     roofline = {"kernel": gemm_kernel, "bound": "tensor", "achieved": round(achieved, 1),
                 "peak": fp8_peak, "unit": "TFLOP/s", "frac": round(achieved / fp8_peak, 4),
+                "frac_of_measured_tcgen05_e4m3": round(achieved / measured["tcgen05_e4m3_tflops"], 4),
+                "frac_of_int8_mma_sync": round(achieved / measured["mma_sync_s8_tops"], 4),
                 "traffic": recorded_traffic(gemm_kernel, args.workload),
                 "peak_note": "E4M3 kind::f8f6f4 dense = 2 x bf16 %s (%s)" % (bf16_peak, peak_src)}
     rq_roof = None
@@ -482,6 +636,15 @@ def main():
             "config": config_dict(cfg, args), "roofline": roofline,
             "roofline_rotate_quant": rq_roof, "per_layer": per_layer,
             "cpu_baseline": cpu, "e2e": e2e,
+            "comparators": {
+                "fp16_cublas_tops": round(ops_step * world / (cublas_ms * 1e-3) / 1e12, 1),
+                "speedup_vs_fp16_cublas": round(cublas_ms / (total_ms / args.steps), 3),
+                ("separate" if args.fused else "fused") + "_tops":
+                    round(ops_step * world / (other_ms * 1e-3) / 1e12, 1),
+                "fused_over_separate_time": round(
+                    (total_ms / args.steps) / other_ms if args.fused
+                    else other_ms / (total_ms / args.steps), 3)},
+            "measured_peaks": measured,
             "gpu_launches": (1 if args.fused else 2) * nlay * args.steps,
             "clocks": clocks,
         }

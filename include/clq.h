@@ -235,6 +235,27 @@ clq_status clq_get_device_status(void* stream, int32_t* out);
  */
 clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream);
 
+/*
+ * Peak-rate microbenchmarks (measurement only; the paper has no counterpart:
+ * they give the measured denominators next to the GEMM and rotate-quant
+ * rates).  Each call launches on `stream` and returns at once; the caller
+ * times the launch with CUDA events on that stream and divides *ops by the
+ * elapsed time.  *ops receives the multiply-accumulates (or bytes) the
+ * launch performs.  No inputs are read except `buf`.
+ *
+ * clq_peak_tcgen05_e4m3: tcgen05.mma kind::f8f6f4 (E4M3 x E4M3, fp32
+ *   accumulate, the MMA of clq_w4a4_linear), one CTA per SM issuing `iters`
+ *   K = 128 steps of 128 x 256 tiles from shared memory (1 .. 1e6).
+ * clq_peak_mma_sync: warp-level mma.sync, kind 0 = s8 m16n8k32 (the INT8
+ *   tensor path of sm_103a), 1 = s4 m16n8k64, 2 = e4m3 m16n8k32; `iters`
+ *   (1 .. 1e6) rounds of 4 independent MMAs per warp, 32 warps per SM.
+ * clq_peak_hbm_read: reads `bytes` (a multiple of 16, buf 16-byte aligned)
+ *   once; *ops = bytes.
+ */
+clq_status clq_peak_tcgen05_e4m3(int32_t iters, int64_t* ops, void* stream);
+clq_status clq_peak_mma_sync(int32_t kind, int32_t iters, int64_t* ops, void* stream);
+clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

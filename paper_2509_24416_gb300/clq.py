@@ -30,7 +30,8 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_rotate_quant_act", "clq_expand_weights", "clq_w4a4_linear",
            "clq_fused_linear_workspace_size", "clq_fused_linear",
            "clq_fused_linear_noalloc", "clq_get_device_status",
-           "clq_selftest_bounded_wait")
+           "clq_selftest_bounded_wait", "clq_peak_tcgen05_e4m3",
+           "clq_peak_mma_sync", "clq_peak_hbm_read")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -55,6 +56,9 @@ _SIGS = {
                                       _P, _I, _P, _P]),
     "clq_get_device_status": (_I, [_P, _P]),
     "clq_selftest_bounded_wait": (_I, [ctypes.c_int64, _P]),
+    "clq_peak_tcgen05_e4m3": (_I, [_I, _P, _P]),
+    "clq_peak_mma_sync": (_I, [_I, _I, _P, _P]),
+    "clq_peak_hbm_read": (_I, [_P, ctypes.c_uint64, _P, _P]),
 }
 
 
@@ -142,6 +146,18 @@ def clq_get_device_status(stream, out):
 
 def clq_selftest_bounded_wait(timeout_ns, stream):
     return load().clq_selftest_bounded_wait(timeout_ns, stream)
+
+
+def clq_peak_tcgen05_e4m3(iters, ops, stream):
+    return load().clq_peak_tcgen05_e4m3(iters, ops, stream)
+
+
+def clq_peak_mma_sync(kind, iters, ops, stream):
+    return load().clq_peak_mma_sync(kind, iters, ops, stream)
+
+
+def clq_peak_hbm_read(buf, nbytes, ops, stream):
+    return load().clq_peak_hbm_read(buf, nbytes, ops, stream)
 
 
 # ----------------------------------------------------------- tensor helpers --
@@ -345,3 +361,42 @@ class PreparedLinear:
                                    stream=stream)
         return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, X.shape[1],
                            self.bias, out_dtype=X.dtype, stream=stream)
+
+
+def measure_peaks(stream=None, reps=5):
+    """Measured peak rates on the current device (best of `reps`, CUDA events
+    on `stream` around each microbenchmark launch): tcgen05 E4M3 and
+    mma.sync s8 / s4 / e4m3 in TFLOP/s (2 ops per multiply-accumulate) and
+    the HBM read bandwidth in GB/s."""
+    s = torch.cuda.current_stream() if stream is None else stream
+    sp = s.cuda_stream
+    dev = torch.device("cuda", torch.cuda.current_device())
+    buf = torch.empty(1 << 31, dtype=torch.uint8, device=dev)
+    ops = ctypes.c_int64(0)
+
+    def timed(launch):
+        best = None
+        for r in range(reps + 1):
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            launch()
+            z.record(s)
+            z.synchronize()
+            if r > 0:  # the first launch is a warm-up
+                t = a.elapsed_time(z) * 1e-3
+                best = t if best is None else min(best, t)
+        return ops.value / best
+
+    out = {}
+    out["tcgen05_e4m3_tflops"] = 2e-12 * timed(lambda: _check(
+        clq_peak_tcgen05_e4m3(20000, ctypes.byref(ops), sp), "clq_peak_tcgen05_e4m3"))
+    for kind, name in ((0, "mma_sync_s8_tops"), (1, "mma_sync_s4_tops"),
+                       (2, "mma_sync_e4m3_tflops")):
+        out[name] = 2e-12 * timed(lambda: _check(
+            clq_peak_mma_sync(kind, 4000, ctypes.byref(ops), sp), "clq_peak_mma_sync"))
+    out["hbm_read_gbs"] = 1e-9 * timed(lambda: _check(
+        clq_peak_hbm_read(buf.data_ptr(), buf.numel(), ctypes.byref(ops), sp),
+        "clq_peak_hbm_read"))
+    del buf
+    return {k: round(v, 1) for k, v in out.items()}

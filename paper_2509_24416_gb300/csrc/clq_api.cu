@@ -310,4 +310,40 @@ clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream) {
                                              static_cast<cudaStream_t>(stream)));
 }
 
+clq_status clq_peak_tcgen05_e4m3(int32_t iters, int64_t* ops, void* stream) {
+  if (ops == nullptr || iters < 1 || iters > 1000000) return CLQ_ERR_INVALID_ARG;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  long long n = 0;
+  st = from_cuda(clq::launch_peak_tcgen05(iters, status, static_cast<cudaStream_t>(stream), &n));
+  *ops = n;
+  return st;
+}
+
+clq_status clq_peak_mma_sync(int32_t kind, int32_t iters, int64_t* ops, void* stream) {
+  if (ops == nullptr || kind < 0 || kind > 2 || iters < 1 || iters > 1000000)
+    return CLQ_ERR_INVALID_ARG;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  long long n = 0;
+  st = from_cuda(
+      clq::launch_peak_mma_sync(kind, iters, status, static_cast<cudaStream_t>(stream), &n));
+  *ops = n;
+  return st;
+}
+
+clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void* stream) {
+  if (ops == nullptr || buf == nullptr || bytes == 0 || bytes % 16 != 0)
+    return CLQ_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(buf) % 16 != 0) return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  st = from_cuda(clq::launch_peak_hbm_read(buf, bytes, status, static_cast<cudaStream_t>(stream)));
+  *ops = static_cast<int64_t>(bytes);
+  return st;
+}
+
 }  // extern "C"

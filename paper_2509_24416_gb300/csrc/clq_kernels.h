@@ -76,6 +76,11 @@ int sm_count();  // cached per device
 // TMA map of an INT4 code array (rows x K) in layout `codes`, box_rows rows.
 bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows, int K,
                       int box_rows);
+// Peak-rate microbenchmarks (peaks.cu); *macs / *ops receive the work done.
+cudaError_t launch_peak_tcgen05(int iters, int32_t* status, cudaStream_t st, long long* macs);
+cudaError_t launch_peak_mma_sync(int kind, int iters, int32_t* sink, cudaStream_t st,
+                                 long long* macs);
+cudaError_t launch_peak_hbm_read(const void* buf, size_t bytes, int32_t* sink, cudaStream_t st);
 // Raise `func`'s dynamic shared-memory limit to the device maximum once per
 // device, and (per_sm != null) return its occupancy for (threads, smem),
 // cached, so that launches make no per-call attribute queries.

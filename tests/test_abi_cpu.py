@@ -110,6 +110,17 @@ def test_fused_and_prepare_host_validation(lib):
     assert clq.clq_get_device_status(None, None) == 1
 
 
+def test_peak_microbenchmark_host_validation(lib):
+    ops = ctypes.c_int64(0)
+    assert clq.clq_peak_tcgen05_e4m3(0, ctypes.byref(ops), None) == 1      # iters < 1
+    assert clq.clq_peak_tcgen05_e4m3(10, None, None) == 1                  # null ops
+    assert clq.clq_peak_mma_sync(3, 10, ctypes.byref(ops), None) == 1      # bad kind
+    assert clq.clq_peak_mma_sync(0, 2000000, ctypes.byref(ops), None) == 1  # iters > 1e6
+    assert clq.clq_peak_hbm_read(P, 100, ctypes.byref(ops), None) == 1     # bytes % 16
+    assert clq.clq_peak_hbm_read(P + 4, 64, ctypes.byref(ops), None) == 3  # alignment
+    assert clq.clq_peak_hbm_read(None, 64, ctypes.byref(ops), None) == 1
+
+
 @pytest.mark.parametrize("K,seed", [(1, 0), (2, 1), (7, 2), (64, 3),
                                     (1152, 4), (4608, 5)])
 def test_build_permutation_matches_oracle(lib, K, seed):
