@@ -82,6 +82,21 @@ KERNEL_SOURCES = {
 }
 
 
+def job_throughput(local_ms, ops_per_step, steps, world, device=None):
+    """Whole-job rate of a weak-scaling run: every rank processes its own
+    batch, so the job takes the slowest rank's time; returns (that time in
+    ms, all ranks' operations / that time in TOPS).  With world > 1 it needs
+    an initialised process group (nccl on GPUs, gloo in the CPU tests)."""
+    import torch
+    import torch.distributed as dist
+    ms = float(local_ms)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms, ops_per_step * steps * world / (ms * 1e-3) / 1e12
+
+
 def kernel_source_sha(kernel):
     import glob
     csrc = os.path.join(ROOT, "paper_2509_24416_gb300", "csrc")
@@ -411,7 +426,8 @@ def main():
     all_names = [l[0] for l in synth.WORKLOADS[args.workload]["layers"]]
     for lname, _, _ in cfg["layers"]:
         li = all_names.index(lname)
-        d = synth.layer_inputs(dict(synth.WORKLOADS[args.workload], M=cfg["M"]), li)
+        d = synth.layer_inputs(dict(synth.WORKLOADS[args.workload], M=cfg["M"]), li,
+                               batch=rank)  # each rank its own token batch
         calib = torch.from_numpy(d["calib"]).to(td).to(dev)
         perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
         lay = clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b,
@@ -548,13 +564,8 @@ def main():
         for i in range(nlay):
             rq_ms[i] += e[4 * i].elapsed_time(e[4 * i + 1])
             gm_ms[i] += e[4 * i + 2].elapsed_time(e[4 * i + 3])
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-
     ops_step = sum(layer_ops(cfg))
-    value = ops_step * args.steps * world / (total_ms * 1e-3) / 1e12
+    total_ms, value = job_throughput(total_ms, ops_step, args.steps, world, dev)
     hbm_peak, bf16_peak, peak_src = peaks()
     fp8_peak = 2.0 * bf16_peak  # E4M3 dense rate = 2x bf16 (nominal ratio)
     K_list = [K for (_, K, _, _) in layers]

@@ -112,9 +112,12 @@ def n_outliers(cfg, K):
     return int(round(cfg["out_frac"] * K))
 
 
-def layer_inputs(cfg, li, M=None, calib_tokens=256, calib_batch=4):
+def layer_inputs(cfg, li, M=None, calib_tokens=256, calib_batch=4, batch=0):
     """All seeded inputs of layer ``li`` of a workload, as numpy fp32 holding
     values already rounded to the workload dtype, plus the torch tensors.
+    ``batch`` selects another token batch of the same distribution (the
+    activations' seed moves; weights, bias and calibration do not), so that
+    ranks of a multi-GPU run each process their own batch.
 
     Returns a dict with X, W, bias (torch, CPU, workload dtype), the exact
     fp32 copies X32, W32, bias32, and the calibration batch calib [B, T, K]
@@ -129,7 +132,7 @@ def layer_inputs(cfg, li, M=None, calib_tokens=256, calib_batch=4):
                                         if cfg["out_lo"] == cfg["out_hi"]
                                         else None))
     dt = cfg["dtype"]
-    X = to_torch(activations(M, K, ch, layer_seed(SEED_X, li), gelu,
+    X = to_torch(activations(M, K, ch, layer_seed(SEED_X, li) + 100003 * int(batch), gelu,
                              min(cfg["text_rows"], M), cfg["text_scale"]), dt)
     W = to_torch(normal((N, K), cfg["w_std"], layer_seed(SEED_W, li)), dt)
     bias = to_torch(normal((N,), 0.01, layer_seed(SEED_BIAS, li)), dt)
