@@ -353,14 +353,81 @@ class PreparedLinear:
     def from_state_dict(cls, d):
         return cls(d["Wq"], d["s_w"], d["perm"], int(d["b"]), d.get("bias"))
 
-    def __call__(self, X, fused=False, workspace=None, stream=None):
+    def __call__(self, X, fused=False, workspace=None, stream=None, Y=None,
+                 Xq=None, s_x=None):
+        """Y = X W^T + bias through the W4A4 path.  Y, and the activation
+        codes / scales of the separate path (Xq [M, K] uint8, s_x [M] fp32),
+        may be passed in to avoid allocations."""
         if fused:
             return fused_linear(X, self.perm, self.b, self.We, self.s_w,
-                                self.bias, workspace=workspace, stream=stream)
+                                self.bias, Y=Y, workspace=workspace, stream=stream)
         Xq, s_x = rotate_quant_act(X, self.perm, self.b, CLQ_CODES_E4M3,
-                                   stream=stream)
+                                   Xq=Xq, s_x=s_x, stream=stream)
         return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, X.shape[1],
-                           self.bias, out_dtype=X.dtype, stream=stream)
+                           self.bias, out_dtype=X.dtype, Y=Y, stream=stream)
+
+
+class HostPipeline:
+    """Runs prepared layers on host inputs into host outputs with the three
+    kinds of work on three CUDA streams, so that they overlap: while layer i
+    computes, layer i + 1's input travels to the device and layer i - 1's
+    output travels back.  All device buffers (inputs, codes, scales,
+    workspaces, outputs) are allocated once here; host buffers should be
+    pinned (`torch.Tensor.pin_memory`) for the copies to be asynchronous.
+
+    `layers` is a list of (PreparedLinear, M, K, N).  `run` enqueues one pass
+    and returns at once; a later `run` waits on the device, per layer, for the
+    previous pass to have released that layer's buffers.  `join(stream)`
+    makes `stream` wait for everything enqueued so far."""
+
+    def __init__(self, layers, dtype, device, fused=False):
+        self.layers = layers
+        self.fused = fused
+        dev = torch.device(device)
+        self.xd = [torch.empty((M, K), dtype=dtype, device=dev) for (_, M, K, _) in layers]
+        self.yd = [torch.empty((M, N), dtype=dtype, device=dev) for (_, M, _, N) in layers]
+        self.xq = [torch.empty((M, K), dtype=torch.uint8, device=dev)
+                   for (_, M, K, _) in layers]
+        self.sx = [torch.empty(M, dtype=torch.float32, device=dev) for (_, M, _, _) in layers]
+        self.ws = [fused_workspace(M, K, dev) if fused else None for (_, M, K, _) in layers]
+        self.s_in = torch.cuda.Stream(device=dev)
+        self.s_comp = torch.cuda.Stream(device=dev)
+        self.s_out = torch.cuda.Stream(device=dev)
+        n = len(layers)
+        self.in_done = [torch.cuda.Event() for _ in range(n)]
+        self.comp_done = [torch.cuda.Event() for _ in range(n)]
+        self.out_done = [torch.cuda.Event() for _ in range(n)]
+        self.started = False
+
+    def run(self, xh, yh, after=None):
+        """One pass: xh[i] (host [M, K]) -> yh[i] (host [M, N]).  `after`: an
+        event that every stream waits on first (for timing)."""
+        for s in (self.s_in, self.s_comp, self.s_out):
+            if after is not None:
+                s.wait_event(after)
+        for i, (lay, M, K, N) in enumerate(self.layers):
+            with torch.cuda.stream(self.s_in):
+                if self.started:  # the previous pass has consumed xd[i]
+                    self.s_in.wait_event(self.comp_done[i])
+                self.xd[i].copy_(xh[i], non_blocking=True)
+                self.in_done[i].record(self.s_in)
+            with torch.cuda.stream(self.s_comp):
+                self.s_comp.wait_event(self.in_done[i])
+                if self.started:  # the previous pass has read yd[i] back
+                    self.s_comp.wait_event(self.out_done[i])
+                lay(self.xd[i], fused=self.fused, workspace=self.ws[i], stream=self.s_comp,
+                    Y=self.yd[i], Xq=self.xq[i], s_x=self.sx[i])
+                self.comp_done[i].record(self.s_comp)
+            with torch.cuda.stream(self.s_out):
+                self.s_out.wait_event(self.comp_done[i])
+                yh[i].copy_(self.yd[i], non_blocking=True)
+                self.out_done[i].record(self.s_out)
+        self.started = True
+
+    def join(self, stream=None):
+        s = torch.cuda.current_stream() if stream is None else stream
+        for e in self.out_done + self.comp_done + self.in_done:
+            s.wait_event(e)
 
 
 def measure_peaks(stream=None, reps=5):
