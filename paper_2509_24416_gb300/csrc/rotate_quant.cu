@@ -38,14 +38,14 @@ __global__ void outlier_scores_kernel(const uint16_t* calib, int B, int Tn, int 
 // on GB300 (M up to 65536 tokens): a CTA takes about max(1.2, 0.1 + 0.121 W)
 // us per tile when W warps share the SM (a latency floor, then issue-bound),
 // every CTA walks ceil(tiles / CTAs) tiles, and the first tile's arrival adds
-// about 0.7 us per 2304-byte row.  Few rows per tile win when M is small (more
-// CTAs share the work), many when M is large.
+// about 0.7 us per 2304-byte row; a lone CTA per SM pays 1.35x per tile.  Few
+// rows per tile win when M is small (more CTAs share the work), many when M
+// is large.
 void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads,
                          size_t* smem) {
   const int segs = K >> 5;
-  const bool large = rq::large_rows(K);
-  const int stride = large ? rq::kStrideLarge : rq::kStrideSmall;
-  const int stages = large ? rq::kStagesLarge : rq::kStagesSmall;
+  const int stride = rq::kStride;
+  const int stages = rq::kStages;
   int best_r = 1;
   double best_cost = 1e300;
   for (int r = 1; r * segs <= 512 && 2 * r * K <= stride; ++r) {
@@ -58,8 +58,11 @@ void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads
     const long tiles = (static_cast<long>(M) + r - 1) / r;
     const long total = static_cast<long>(ctas) * std::max(sms, 1);
     const long rounds = (tiles + total - 1) / total;
-    const double cost =
-        rounds * std::max(1.2, 0.1 + 0.121 * ctas * warps) + 0.7 * r * (2.0 * K) / 2304.0;
+    // A lone CTA per SM has no second CTA to run through its barrier stalls
+    // (measured: 1.35x per tile at K = 4608).
+    const double alone = ctas == 1 ? 1.35 : 1.0;
+    const double cost = rounds * alone * std::max(1.2, 0.1 + 0.121 * ctas * warps) +
+                        0.7 * r * (2.0 * K) / 2304.0;
     if (cost < best_cost - 1e-9) {
       best_cost = cost;
       best_r = r;

@@ -40,9 +40,7 @@ cudaError_t launch_geom(const RotateQuantArgs& a, int threads, size_t smem, int 
 template <typename T, int LOGB, bool CLIP>
 cudaError_t launch_b(const RotateQuantArgs& a, int threads, size_t smem, int sms,
                      cudaStream_t st) {
-  if (large_rows(a.K))
-    return launch_geom<T, LOGB, CLIP, kStrideLarge, kStagesLarge>(a, threads, smem, sms, st);
-  return launch_geom<T, LOGB, CLIP, kStrideSmall, kStagesSmall>(a, threads, smem, sms, st);
+  return launch_geom<T, LOGB, CLIP, kStride, kStages>(a, threads, smem, sms, st);
 }
 
 // log2(b) is a compile-time constant for b >= 16 on the activation path;
