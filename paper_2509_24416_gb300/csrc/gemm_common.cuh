@@ -200,7 +200,7 @@ __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, in
                                               const float* col_scale, const float* col_bias,
                                               uint8_t* staging, const CUtensorMap* mapY,
                                               void* Y, int32_t* acc_dbg, int& store_count) {
-  static_assert(NCOL % (2 * EPI_COLS) == 0, "column share must be an even number of blocks");
+  static_assert(NCOL % EPI_COLS == 0, "column share must be whole 32-column blocks");
   const uint32_t lane_base = tmem_acc + (static_cast<uint32_t>(quarter * 32) << 16);
   if (n0 + col0 >= N) return;
   if (!PREFETCH) {
@@ -220,7 +220,7 @@ __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, in
   for (int c = col0; c < col0 + NCOL; c += 2 * EPI_COLS) {
     // ra holds block c (issued earlier); warp-uniform conditions throughout.
     tmem_ld_wait_tie(ra);
-    const bool more1 = n0 + c + EPI_COLS < N;
+    const bool more1 = c + EPI_COLS < col0 + NCOL && n0 + c + EPI_COLS < N;
     if (more1) tmem_ld32(lane_base + c + EPI_COLS, rb);
     epilogue_block<OutT, NBUF>(ra, c, quarter, lane, m0, n0, M, N, sx, col_scale, col_bias,
                                staging, mapY, Y, acc_dbg, store_count);

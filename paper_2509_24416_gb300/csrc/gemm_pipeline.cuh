@@ -46,7 +46,7 @@ constexpr int WARP_UNPACK0 = 6;
 constexpr int MIN_THREADS = (WARP_UNPACK0 + NUM_UNPACK / 32) * 32;  // 448
 constexpr int MAX_STAGES = 6;
 
-// Tile BM x BNT (the kernels use BNT = 256).
+// Tile BM x BNT (BNT = 256, or 192 for E4M3 operands where N splits better).
 template <bool APACK, bool BPACK, int BNT = BN>
 struct Cfg {
   static constexpr bool UNPACK = APACK || BPACK;
@@ -59,7 +59,7 @@ struct Cfg {
   static constexpr int BP = BNT * BKP;   // packed B stage
   static constexpr int STAGE = A_U + BU + (APACK ? A_P : 0) + (BPACK ? BP : 0);
   static constexpr int FIXED = EPI_TOTAL + 4 * BNT * 4;
-  static constexpr int S0 = (212 * 1024 - FIXED) / STAGE;
+  static constexpr int S0 = (222 * 1024 - FIXED) / STAGE;
   static constexpr int S = S0 > MAX_STAGES ? MAX_STAGES : S0;  // pipeline stages
   static constexpr size_t OFF_UA = 0;                           // E4M3 operands
   static constexpr size_t OFF_UB = OFF_UA + S * A_U;
@@ -69,7 +69,9 @@ struct Cfg {
   static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;        // [2][2][BNT] floats
   static constexpr size_t BYTES = OFF_COL + 4 * BNT * sizeof(float);
   static constexpr uint32_t TX = (APACK ? A_P : A_U) + (BPACK ? BP : BU);
-  static constexpr uint32_t TMEM = 2 * BNT;                     // two accumulators
+  // two accumulators of BNT columns, 2 * BNT rounded up to the power of two
+  // tcgen05.alloc takes
+  static constexpr uint32_t TMEM = 2 * BNT <= 256 ? 256u : 512u;
   static_assert(S >= 2, "pipeline needs two stages");
 };
 

@@ -158,7 +158,7 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB,
 template <typename OutT>
 cudaError_t launch_gemm_dt(const CUtensorMap& mapA, const CUtensorMap& mapB,
                            const CUtensorMap& mapY, const GemmArgs& g, bool apack, bool bpack,
-                           int use_tma_store, int grid, cudaStream_t st) {
+                           int bn, int use_tma_store, int grid, cudaStream_t st) {
   if (apack)
     return bpack ? launch_gemm_t<OutT, true, true, BN>(mapA, mapB, mapY, g, use_tma_store, grid,
                                                        st)
@@ -166,6 +166,8 @@ cudaError_t launch_gemm_dt(const CUtensorMap& mapA, const CUtensorMap& mapB,
                                                         st);
   if (bpack)
     return launch_gemm_t<OutT, false, true, BN>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+  if (bn == 192)
+    return launch_gemm_t<OutT, false, false, 192>(mapA, mapB, mapY, g, use_tma_store, grid, st);
   return launch_gemm_t<OutT, false, false, BN>(mapA, mapB, mapY, g, use_tma_store, grid, st);
 }
 
@@ -189,10 +191,20 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   if (sms <= 0) return cudaErrorInvalidDevice;
   const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
   const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
-  // 256-wide tiles: measured faster than 128-wide ones even where 128 fills
-  // the last wave of tiles better (the narrower tile moves more operand bytes
-  // through shared memory per multiply-add).
-  const int bn = BN;
+  // Tile width: an SM's intake from L2 bounds the kernel, so a tile costs
+  // about its operand bytes per K step (A 16 KB + B BN/8 KB), and the CTAs
+  // walk ceil(tiles / SMs) rounds.  256 wins unless 192 splits N into whole
+  // tiles with no more rounds (N = 1152: 6 x 192 instead of 4.5 x 256).  128
+  // measured slower everywhere.
+  int bn = BN;
+  if (!apack && !bpack) {
+    const long mt = (g.M + BM - 1) / BM;
+    auto cost = [&](int w) {
+      const long rounds = (mt * ((g.N + w - 1) / w) + sms - 1) / sms;
+      return rounds * (16.0 + w / 8.0);
+    };
+    if (cost(192) < cost(256)) bn = 192;
+  }
   CUtensorMap mapA, mapB, mapY;
   if (!encode_codes_map(&mapA, Xq, x_codes, g.M, g.K, BM) ||
       !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn))
@@ -206,9 +218,9 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   const int tiles = ((g.M + BM - 1) / BM) * ((g.N + bn - 1) / bn);
   const int grid = std::min(tiles, sms);
   if (out_dtype == CLQ_F16)
-    return launch_gemm_dt<__half>(mapA, mapB, mapY, g, apack, bpack, use_tma_store, grid,
+    return launch_gemm_dt<__half>(mapA, mapB, mapY, g, apack, bpack, bn, use_tma_store, grid,
                                   st);
-  return launch_gemm_dt<__nv_bfloat16>(mapA, mapB, mapY, g, apack, bpack, use_tma_store,
+  return launch_gemm_dt<__nv_bfloat16>(mapA, mapB, mapY, g, apack, bpack, bn, use_tma_store,
                                        grid, st);
 }
 
