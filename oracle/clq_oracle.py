@@ -10,7 +10,8 @@ paper's order, in plain numpy, slowly and without blocking or fusion:
 
 * Sec. 3.3 "Data Preparing": batch mean S of the calibration activations.
 * Sec. 3.3 "Outlier Detection": per-channel absolute maximum of S as the
-  outlier score; the top 50% of channels are moved to the left side.
+  outlier score (Sec. 4.4's alternative metrics too); the top 50% of
+  channels are moved to the left side.
 * Sec. 3.3 "Orthogonal Smoothing" / "Overhead Analysis": G = S_swap H with H a
   block-diagonal +-1 Hadamard matrix; G is absorbed into the weights before
   quantization; the activations are rotated online; only the index vector s
@@ -48,6 +49,11 @@ Readings of the paper that this file fixes (the paper leaves them open):
    precision the GPU path uses, because it decides an integer permutation.
 7. Packing.  Byte j of a packed row holds code 2j in its low nibble and code
    2j+1 in its high nibble, as 4-bit two's complement.
+8. Outlier-metric variants.  Sec. 4.4 names percentile (1 %, 99 %), top-k
+   mean (k = 1 %), range and peak-average ratio without formulas; read as
+   in outlier_scores() (percentile: max(|P1|, |P99|) with linear
+   interpolation; k = max(1, round-half-up(T / 100)); PAR = peak / mean of
+   |S|), each in fp32 in a fixed order.
 """
 
 import numpy as np
@@ -74,13 +80,13 @@ def hadamard_sylvester(b):
     return np.where(parity == 1, -1, 1).astype(np.int64)
 
 
-def outlier_scores(calib):
-    """Outlier score per channel from calibration activations [B, T, K].
+OUTLIER_METRICS = ("absmax", "percentile", "topk_mean", "range", "par")
+PERCENTILE_PAIR = (0.01, 0.99)  # Sec. 4.4 "Choice of Outlier Metric": (1 %, 99 %)
 
-    Sec. 3.3 "Data Preparing": S = mean of X over the batch axis (fp32,
-    summed over b in order, then divided by B).  "Outlier Detection": the
-    score of channel c is max over tokens of |S[:, c]|.
-    """
+
+def batch_mean(calib):
+    """Sec. 3.3 "Data Preparing": S = mean of X [B, T, K] over the batch axis
+    (fp32, summed over b in order, then divided by B)."""
     calib = np.asarray(calib, dtype=np.float32)
     if calib.ndim != 3:
         raise ValueError("calibration data must be [B, T, K]")
@@ -88,8 +94,77 @@ def outlier_scores(calib):
     total = np.zeros(calib.shape[1:], dtype=np.float32)
     for bi in range(B):
         total = total + calib[bi]
-    mean = total / np.float32(B)
-    return np.max(np.abs(mean), axis=0).astype(np.float32)
+    return total / np.float32(B)
+
+
+def topk_count(T):
+    """k of the top-k mean: 1 % of the tokens (Sec. 4.4), rounded half up,
+    at least 1 (reading 8)."""
+    return max(1, (int(T) + 50) // 100)
+
+
+def _percentile_fp32(sorted_col, q):
+    """Linear interpolation between order statistics, every step in fp32:
+    pos = q * (T - 1), lo = floor(pos), v = v[lo] + (pos - lo) * (v[lo+1] - v[lo])
+    (reading 8)."""
+    T = sorted_col.shape[0]
+    pos = np.float32(q) * np.float32(T - 1)
+    lo = int(np.floor(pos))
+    hi = min(lo + 1, T - 1)
+    frac = np.float32(pos - np.float32(lo))
+    d = np.float32(sorted_col[hi] - sorted_col[lo])
+    return np.float32(sorted_col[lo] + np.float32(frac * d))
+
+
+def outlier_scores(calib, metric="absmax"):
+    """Outlier score per channel from calibration activations [B, T, K].
+
+    Sec. 3.3 "Outlier Detection": the score of channel c is max over tokens
+    of |S[:, c]| (the method's choice).  Sec. 4.4 "Choice of Outlier Metric"
+    names four alternatives, read here (reading 8) as, per channel of S:
+      percentile: max(|P1|, |P99|), P linear-interpolated order statistics;
+      topk_mean:  the mean of the k = topk_count(T) largest |S[t, c]|, summed
+                  from the largest down in fp32;
+      range:      max_t S - min_t S;
+      par:        peak-to-average ratio max_t |S| / (sum_t |S| / T), the sum
+                  taken over t in order in fp32; 0 for an all-zero channel.
+    All arithmetic in fp32 in the stated order: the scores decide an integer
+    permutation, and the GPU takes the same steps.
+    """
+    if metric not in OUTLIER_METRICS:
+        raise ValueError("unknown outlier metric %r" % (metric,))
+    S = batch_mean(calib)
+    T, K = S.shape
+    A = np.abs(S)
+    if metric == "absmax":
+        return np.max(A, axis=0).astype(np.float32)
+    if metric == "range":
+        return (np.max(S, axis=0) - np.min(S, axis=0)).astype(np.float32)
+    if metric == "par":
+        total = np.zeros(K, dtype=np.float32)
+        for t in range(T):
+            total = total + A[t]
+        mean = total / np.float32(T)
+        peak = np.max(A, axis=0)
+        out = np.zeros(K, dtype=np.float32)
+        nz = mean > 0
+        out[nz] = (peak[nz] / mean[nz]).astype(np.float32)
+        return out
+    if metric == "percentile":
+        Ss = np.sort(S, axis=0)
+        out = np.empty(K, dtype=np.float32)
+        for c in range(K):
+            lo = _percentile_fp32(Ss[:, c], PERCENTILE_PAIR[0])
+            hi = _percentile_fp32(Ss[:, c], PERCENTILE_PAIR[1])
+            out[c] = max(abs(lo), abs(hi))
+        return out
+    # topk_mean
+    k = topk_count(T)
+    As = -np.sort(-A, axis=0)  # descending per channel
+    total = np.zeros(K, dtype=np.float32)
+    for t in range(k):
+        total = total + As[t]
+    return (total / np.float32(k)).astype(np.float32)
 
 
 def build_permutation(scores):

@@ -361,3 +361,93 @@ def test_planted_mistake_is_caught(monkeypatch, name, fn):
 
 def test_package_reexports():
     assert oracle.QMAX == 7 and oracle.hadamard_sylvester is not None
+
+
+# ---------------------------------------------- outlier-metric variants --
+def test_outlier_metrics_hand_example():
+    # B = 1, so S is the data itself; column 0 = [1, -3, 2, 0.5, -0.5]
+    col = np.array([1.0, -3.0, 2.0, 0.5, -0.5], np.float32)
+    cal = np.stack([col, col * 0, -col], axis=1)[None]          # [1, 5, 3]
+    assert np.array_equal(orc.outlier_scores(cal, "absmax"), [3, 0, 3])
+    assert np.array_equal(orc.outlier_scores(cal, "range"), [5, 0, 5])
+    assert np.array_equal(orc.outlier_scores(cal, "topk_mean"), [3, 0, 3])  # k = 1
+    par = orc.outlier_scores(cal, "par")
+    assert par[1] == 0 and abs(par[0] - 3 / 1.4) < 1e-6 and par[0] == par[2]
+    # sorted col: [-3, -0.5, 0.5, 1, 2]; P1 at 0.04 -> -2.9, P99 at 3.96 -> 1.96
+    pct = orc.outlier_scores(cal, "percentile")
+    assert abs(pct[0] - 2.9) < 1e-6 and pct[1] == 0
+    # column 2 is -column 0: P1 -> -1.96, P99 -> 2.9
+    assert abs(pct[2] - 2.9) < 1e-6
+
+
+@pytest.mark.parametrize("metric", ["percentile", "topk_mean", "range", "par"])
+def test_outlier_metrics_against_independent_definitions(metric):
+    rng = np.random.default_rng(11)
+    cal = rng.standard_normal((3, 257, 9)).astype(np.float32)
+    cal[:, 5, 2] += 40.0          # one spike
+    cal[:, :, 7] = 0.0            # an all-zero channel
+    got = orc.outlier_scores(cal, metric).astype(np.float64)
+    S = orc.batch_mean(cal).astype(np.float64)
+    A = np.abs(S)
+    if metric == "percentile":
+        ref = np.maximum(np.abs(np.percentile(S, 1, axis=0, method="linear")),
+                         np.abs(np.percentile(S, 99, axis=0, method="linear")))
+    elif metric == "topk_mean":
+        k = 3                      # round-half-up(257 / 100)
+        assert orc.topk_count(257) == k and orc.topk_count(5) == 1
+        assert orc.topk_count(150) == 2 and orc.topk_count(149) == 1
+        ref = np.array([np.mean(sorted(A[:, c], reverse=True)[:k]) for c in range(9)])
+    elif metric == "range":
+        ref = S.max(axis=0) - S.min(axis=0)
+    else:
+        mean = A.mean(axis=0)
+        ref = np.where(mean > 0, A.max(axis=0) / np.where(mean > 0, mean, 1), 0)
+    assert np.all(np.abs(got - ref) <= 2e-6 * np.maximum(np.abs(ref), 1e-30)), (got, ref)
+    assert got[7] == 0
+
+
+@pytest.mark.parametrize("metric", ["absmax", "percentile", "topk_mean", "range", "par"])
+def test_outlier_metrics_invariances(metric):
+    rng = np.random.default_rng(12)
+    cal = rng.standard_normal((4, 64, 6)).astype(np.float32)
+    s = orc.outlier_scores(cal, metric)
+    # token order: exact for order statistics and extremes, 1e-6 for sums
+    rev = orc.outlier_scores(cal[:, ::-1, :], metric)
+    assert np.allclose(rev, s, rtol=1e-6, atol=0)
+    # scaling a channel by 4 is exact: scores scale by 4, PAR is unchanged
+    cal2 = cal.copy()
+    cal2[:, :, 3] *= 4
+    s2 = orc.outlier_scores(cal2, metric)
+    assert s2[3] == (s[3] if metric == "par" else 4 * s[3])
+    assert np.array_equal(np.delete(s2, 3), np.delete(s, 3))
+    # every metric gives a valid swap vector
+    perm = orc.build_permutation(s)
+    assert np.array_equal(np.sort(perm), np.arange(6))
+
+
+def test_outlier_metric_planted_mistakes_are_caught(monkeypatch):
+    col = np.array([1.0, -3.0, 2.0, 0.5, -0.5], np.float32)
+    cal = np.stack([col, -col], axis=1)[None]
+    good_pct = orc.outlier_scores(cal, "percentile")
+    # nearest-rank instead of linear interpolation
+    monkeypatch.setattr(orc, "_percentile_fp32",
+                        lambda v, q: np.float32(v[int(round(q * (v.shape[0] - 1)))]))
+    assert not np.allclose(orc.outlier_scores(cal, "percentile"), good_pct)
+    monkeypatch.undo()
+    # range over magnitudes, PAR over the median: the hand values catch both
+    real = orc.outlier_scores
+
+    def wrong(calib, metric="absmax"):
+        S = orc.batch_mean(calib)
+        if metric == "range":
+            return (np.abs(S).max(axis=0) - np.abs(S).min(axis=0)).astype(np.float32)
+        if metric == "par":
+            return (np.abs(S).max(axis=0) / np.median(np.abs(S), axis=0)).astype(np.float32)
+        return real(calib, metric)
+
+    monkeypatch.setattr(orc, "outlier_scores", wrong)
+    assert orc.outlier_scores(cal, "range")[0] != 5
+    assert abs(orc.outlier_scores(cal, "par")[0] - 3 / 1.4) > 1e-3
+    monkeypatch.undo()
+    with pytest.raises(ValueError):
+        orc.outlier_scores(cal, "variance")
