@@ -100,6 +100,39 @@ clq_status clq_outlier_scores(const void* calib, clq_dtype dtype, int32_t B,
                               void* stream);
 
 /*
+ * Outlier metrics of Sec. 4.4 ("Choice of Outlier Metric"), which names them
+ * and their parameters but no formulas; this library reads them as below,
+ * every step in fp32 in a fixed order (the scores decide an integer
+ * permutation):
+ *   CLQ_METRIC_ABSMAX      max_t |S| (Sec. 3.3, as clq_outlier_scores);
+ *   CLQ_METRIC_PERCENTILE  max(|P(1 %)|, |P(99 %)|) of S, P by linear
+ *                          interpolation between order statistics:
+ *                          pos = q (T - 1), v[lo] + (pos - lo)(v[lo + 1] - v[lo]);
+ *   CLQ_METRIC_TOPK_MEAN   mean of the k largest |S|, k = max(1, (T + 50) / 100)
+ *                          (1 % of the tokens), summed from the largest down;
+ *   CLQ_METRIC_RANGE       max_t S - min_t S;
+ *   CLQ_METRIC_PAR         peak-to-average ratio max_t |S| / (sum_t |S| / T),
+ *                          the sum over t in order; 0 for an all-zero channel.
+ */
+typedef enum clq_outlier_metric {
+  CLQ_METRIC_ABSMAX = 0,
+  CLQ_METRIC_PERCENTILE = 1,
+  CLQ_METRIC_TOPK_MEAN = 2,
+  CLQ_METRIC_RANGE = 3,
+  CLQ_METRIC_PAR = 4
+} clq_outlier_metric;
+
+/*
+ * Outlier score per input channel under `metric` (see above), from the batch
+ * mean S of calib[B][T][K] (device, dtype `dtype`, contiguous) into scores
+ * (device fp32 [K]).  Requires B, K >= 1 and 1 <= T <= 16384
+ * (CLQ_ERR_SHAPE beyond).  Offline; not on the timed path.
+ */
+clq_status clq_outlier_scores_metric(const void* calib, clq_dtype dtype, int32_t B, int32_t T,
+                                     int32_t K, clq_outlier_metric metric, float* scores,
+                                     void* stream);
+
+/*
  * Column-swap vector from outlier scores (Sec. 3.3, "Outlier Detection"):
  * rank channels by score descending (ties to the lower index); the first
  * K/2 (rounded down) form the high-peak set, placed left, the rest right,

@@ -30,7 +30,8 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_rotate_quant_act", "clq_expand_weights", "clq_w4a4_linear",
            "clq_fused_linear_workspace_size", "clq_fused_linear",
            "clq_fused_linear_noalloc", "clq_get_device_status",
-           "clq_selftest_bounded_wait", "clq_peak_tcgen05_e4m3",
+           "clq_selftest_bounded_wait", "clq_outlier_scores_metric",
+           "clq_peak_tcgen05_e4m3",
            "clq_peak_mma_sync", "clq_peak_hbm_read")
 
 _lib = None
@@ -41,6 +42,7 @@ _SIGS = {
     "clq_status_string": (ctypes.c_char_p, [_I]),
     "clq_version": (_I, []),
     "clq_outlier_scores": (_I, [_P, _I, _I, _I, _I, _P, _P]),
+    "clq_outlier_scores_metric": (_I, [_P, _I, _I, _I, _I, _I, _P, _P]),
     "clq_build_permutation": (_I, [_P, _I, _P]),
     "clq_prepare_weights": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _P, _P, _P,
                                  _P]),
@@ -148,6 +150,10 @@ def clq_selftest_bounded_wait(timeout_ns, stream):
     return load().clq_selftest_bounded_wait(timeout_ns, stream)
 
 
+def clq_outlier_scores_metric(calib, dtype, B, T, K, metric, scores, stream):
+    return load().clq_outlier_scores_metric(calib, dtype, B, T, K, metric, scores, stream)
+
+
 def clq_peak_tcgen05_e4m3(iters, ops, stream):
     return load().clq_peak_tcgen05_e4m3(iters, ops, stream)
 
@@ -189,13 +195,24 @@ def _row_major(t, name):
                          % name)
 
 
-def outlier_scores(calib, stream=None):
-    """calib [B, T, K] fp16/bf16 on the GPU -> fp32 scores [K]."""
+OUTLIER_METRICS = {"absmax": 0, "percentile": 1, "topk_mean": 2, "range": 3, "par": 4}
+
+
+def outlier_scores(calib, metric="absmax", stream=None):
+    """calib [B, T, K] fp16/bf16 on the GPU -> fp32 scores [K] under `metric`
+    (one of OUTLIER_METRICS; "absmax" is the method's, Sec. 3.3)."""
     calib = calib.contiguous()
     B, T, K = calib.shape
     scores = torch.empty(K, dtype=torch.float32, device=calib.device)
-    _check(clq_outlier_scores(_ptr(calib), _dt(calib), B, T, K, _ptr(scores),
-                              _stream(stream)), "clq_outlier_scores")
+    if metric == "absmax":
+        _check(clq_outlier_scores(_ptr(calib), _dt(calib), B, T, K, _ptr(scores),
+                                  _stream(stream)), "clq_outlier_scores")
+    else:
+        if metric not in OUTLIER_METRICS:
+            raise ValueError("unknown outlier metric %r" % (metric,))
+        _check(clq_outlier_scores_metric(_ptr(calib), _dt(calib), B, T, K,
+                                         OUTLIER_METRICS[metric], _ptr(scores),
+                                         _stream(stream)), "clq_outlier_scores_metric")
     return scores
 
 

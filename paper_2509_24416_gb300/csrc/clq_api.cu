@@ -192,6 +192,22 @@ clq_status clq_outlier_scores(const void* calib, clq_dtype dtype, int32_t B, int
       clq::launch_outlier_scores(calib, dtype, B, T, K, scores, static_cast<cudaStream_t>(stream)));
 }
 
+clq_status clq_outlier_scores_metric(const void* calib, clq_dtype dtype, int32_t B, int32_t T,
+                                     int32_t K, clq_outlier_metric metric, float* scores,
+                                     void* stream) {
+  if (!valid_dtype(dtype) || B < 1 || T < 1 || K < 1) return CLQ_ERR_INVALID_ARG;
+  if (static_cast<int>(metric) < CLQ_METRIC_ABSMAX || static_cast<int>(metric) > CLQ_METRIC_PAR)
+    return CLQ_ERR_INVALID_ARG;
+  if (T > 16384) return CLQ_ERR_SHAPE;
+  if (calib == nullptr || scores == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(calib, 2) || !aligned(scores, 4)) return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  return from_cuda(clq::launch_outlier_metric(calib, dtype, B, T, K, static_cast<int>(metric),
+                                              scores, static_cast<cudaStream_t>(stream)));
+}
+
 clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N, int32_t K, int32_t ldw,
                                const int32_t* perm, int32_t b, const float* clip, uint8_t* Wq,
                                float* s_w, float* w_rot_dbg, void* stream) {

@@ -30,6 +30,8 @@ void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads
                          size_t* smem);
 cudaError_t launch_outlier_scores(const void* calib, int dtype, int B, int T, int K,
                                   float* scores, cudaStream_t st);
+cudaError_t launch_outlier_metric(const void* calib, int dtype, int B, int T, int K, int metric,
+                                  float* scores, cudaStream_t st);
 
 struct GemmArgs {
   const float* s_x;   // [M]

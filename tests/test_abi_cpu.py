@@ -110,6 +110,16 @@ def test_fused_and_prepare_host_validation(lib):
     assert clq.clq_get_device_status(None, None) == 1
 
 
+def test_outlier_metric_host_validation(lib):
+    assert clq.clq_outlier_scores_metric(P, 0, 2, 8, 4, 5, P, None) == 1      # metric
+    assert clq.clq_outlier_scores_metric(P, 0, 2, 8, 4, -1, P, None) == 1
+    assert clq.clq_outlier_scores_metric(P, 0, 2, 16385, 4, 1, P, None) == 2  # T limit
+    assert clq.clq_outlier_scores_metric(P, 2, 2, 8, 4, 1, P, None) == 1      # dtype
+    assert clq.clq_outlier_scores_metric(None, 0, 2, 8, 4, 1, P, None) == 1
+    assert clq.clq_outlier_scores_metric(P + 1, 0, 2, 8, 4, 1, P, None) == 3  # alignment
+    assert clq.clq_outlier_scores_metric(P, 0, 0, 8, 4, 1, P, None) == 1      # B < 1
+
+
 def test_peak_microbenchmark_host_validation(lib):
     ops = ctypes.c_int64(0)
     assert clq.clq_peak_tcgen05_e4m3(0, ctypes.byref(ops), None) == 1      # iters < 1
