@@ -54,11 +54,23 @@ Readings of the paper that this file fixes (the paper leaves them open):
    in outlier_scores() (percentile: max(|P1|, |P99|) with linear
    interpolation; k = max(1, round-half-up(T / 100)); PAR = peak / mean of
    |S|), each in fp32 in a fixed order.
+9. Bit widths.  The paper runs W4A4, W4A8 and W8A8 (Sec. 4.1); the grid of
+   reading 5 generalizes to n bits as qmax = 2^(n-1) - 1 (7 or 127): codes in
+   [-qmax, qmax], s = r / qmax, code -2^(n-1) unused.  The product of n-bit
+   codes is the same exact integer sum, dequantized by the same epilogue.
 """
 
 import numpy as np
 
 QMAX = 7  # 2^(n-1) - 1 for n = 4 bits (symmetric reading of Eq. 1)
+BIT_WIDTHS = (4, 8)  # Sec. 4.1: W4A4, W4A8, W8A8
+
+
+def qmax_for_bits(bits):
+    """Largest code of the symmetric n-bit grid, 2^(n-1) - 1 (reading 9)."""
+    if bits not in BIT_WIDTHS:
+        raise ValueError("bit width must be 4 or 8")
+    return 2 ** (bits - 1) - 1
 
 
 # ---------------------------------------------------------------- Sec. 3.3 --
@@ -204,23 +216,26 @@ def rotate(X, perm, b):
 
 
 # ------------------------------------------------------------ Sec. 3.1 Eq.1 --
-def quantize_symmetric(V, clip=None):
-    """Per-row symmetric INT4 quantization of fp32 rows (Eq. 1, reading 5).
+def quantize_symmetric(V, clip=None, bits=4):
+    """Per-row symmetric n-bit quantization of fp32 rows (Eq. 1, readings 5
+    and 9).
 
-    Returns (codes int8 [R, K] in [-7, 7], scales fp32 [R]).  ``clip`` (one
-    fp32 bound per row, > 0) replaces the row's absolute maximum by
-    min(absmax, clip); values beyond it saturate at +-7.
+    Returns (codes int8 [R, K] in [-qmax, qmax], scales fp32 [R]), qmax = 7
+    for 4 bits and 127 for 8.  ``clip`` (one fp32 bound per row, > 0)
+    replaces the row's absolute maximum by min(absmax, clip); values beyond
+    it saturate at +-qmax.
     """
+    qmax = qmax_for_bits(bits)
     V = np.asarray(V, dtype=np.float32)
     amax = np.max(np.abs(V), axis=1).astype(np.float32)
     if clip is not None:
         amax = np.minimum(amax, np.asarray(clip, dtype=np.float32))
-    scale = (amax / np.float32(QMAX)).astype(np.float32)
+    scale = (amax / np.float32(qmax)).astype(np.float32)
     codes = np.zeros(V.shape, dtype=np.int8)
     nz = scale > 0
     if np.any(nz):
         ratio = (V[nz] / scale[nz][:, None]).astype(np.float32)
-        codes[nz] = np.clip(np.rint(ratio), -QMAX, QMAX).astype(np.int8)
+        codes[nz] = np.clip(np.rint(ratio), -qmax, qmax).astype(np.int8)
     scale = np.where(nz, scale, np.float32(0)).astype(np.float32)
     return codes, scale
 
@@ -248,27 +263,29 @@ def unpack_int4(packed):
     return out
 
 
-def rotate_quant_act(X, perm, b):
+def rotate_quant_act(X, perm, b, bits=4):
     """Online activation path: gather by s, block Hadamard, dynamic per-token
     scale, codes, pack (Sec. 3.1 dynamic quantization + Sec. 3.3).
 
-    Returns (Xq uint8 [M, K/2], s_x fp32 [M], x_rot fp32 [M, K], codes int8).
+    Returns (Xq, s_x fp32 [M], x_rot fp32 [M, K], codes int8 [M, K]); Xq is
+    the packed uint8 [M, K/2] for 4 bits and the codes themselves for 8.
     """
     x_rot = rotate(X, perm, b)
-    codes, s_x = quantize_symmetric(x_rot)
-    return pack_int4(codes), s_x, x_rot, codes
+    codes, s_x = quantize_symmetric(x_rot, bits=bits)
+    return (pack_int4(codes) if bits == 4 else codes), s_x, x_rot, codes
 
 
-def prepare_weights(W, perm, b, clip=None):
+def prepare_weights(W, perm, b, clip=None, bits=4):
     """Offline weight path: absorb G into W (W~ = W_p H_blk, Sec. 3.3
-    "Overhead Analysis"), then per-output-channel symmetric INT4.
+    "Overhead Analysis"), then per-output-channel symmetric n-bit codes.
 
-    W is [N, K] as in nn.Linear.  Returns (Wq uint8 [N, K/2], s_w fp32 [N],
-    w_rot fp32 [N, K], codes int8).
+    W is [N, K] as in nn.Linear.  Returns (Wq, s_w fp32 [N], w_rot fp32
+    [N, K], codes int8 [N, K]); Wq is packed uint8 [N, K/2] for 4 bits and
+    the codes themselves for 8.
     """
     w_rot = rotate(W, perm, b)
-    codes, s_w = quantize_symmetric(w_rot, clip)
-    return pack_int4(codes), s_w, w_rot, codes
+    codes, s_w = quantize_symmetric(w_rot, clip, bits=bits)
+    return (pack_int4(codes) if bits == 4 else codes), s_w, w_rot, codes
 
 
 # ------------------------------------------------------------ INT4 product --
@@ -297,6 +314,21 @@ def w4a4_linear(Xq, s_x, Wq, s_w, b, bias=None):
     """
     acc = int_gemm(unpack_int4(Xq), unpack_int4(Wq))
     return dequant_epilogue(acc, s_x, s_w, b, bias), acc
+
+
+def quant_linear(qx, s_x, qw, s_w, b, bias=None):
+    """Product of unpacked n-bit codes (any of W4A4, W4A8, W8A8) with the
+    dequant + bias epilogue.  Returns (y fp64 [M, N], acc int64 [M, N])."""
+    acc = int_gemm(qx, qw)
+    return dequant_epilogue(acc, s_x, s_w, b, bias), acc
+
+
+def obs_linear(X, perm, b, qw, s_w, bias=None, a_bits=4):
+    """The layer at any bit setting: rotate-quant of X to a_bits, then the
+    product with the prepared weight codes qw (int8 [N, K], any width)."""
+    _, s_x, _, qx = rotate_quant_act(X, perm, b, bits=a_bits)
+    y, _ = quant_linear(qx, s_x, qw, s_w, b, bias)
+    return y
 
 
 def fused_linear(X, perm, b, Wq, s_w, bias=None):

@@ -314,7 +314,7 @@ def _hadamard_sequency(b):
     return H[np.argsort([np.count_nonzero(np.diff(r)) for r in H])]
 
 
-def _quantize_half_away(V, clip=None):
+def _quantize_half_away(V, clip=None, bits=4):
     V = np.asarray(V, dtype=np.float32)
     amax = np.max(np.abs(V), axis=1).astype(np.float32)
     s = (amax / np.float32(7)).astype(np.float32)
@@ -451,3 +451,107 @@ def test_outlier_metric_planted_mistakes_are_caught(monkeypatch):
     monkeypatch.undo()
     with pytest.raises(ValueError):
         orc.outlier_scores(cal, "variance")
+
+
+# ------------------------------------------------ bit widths (W4A8, W8A8) --
+def test_8bit_hand_example():
+    """s = r / 127: a row with absolute maximum 127 has s = 1 and its codes
+    are the values rounded half to even; one with maximum 254 has s = 2."""
+    V = np.array([[127, -63.5, 0.5, 2.5, -1.5, 126.5, -127, 0],
+                  [254, 3, -5, 1, 253, -0.5, 0, -254]], dtype=np.float32)
+    codes, s = orc.quantize_symmetric(V, bits=8)
+    assert s.tolist() == [1.0, 2.0]
+    assert codes.tolist() == [[127, -64, 0, 2, -2, 126, -127, 0],
+                              [127, 2, -2, 0, 126, 0, 0, -127]]
+    c4, s4 = orc.quantize_symmetric(V[:1] * np.float32(7 / 127), bits=4)
+    assert c4.max() == 7 and c4.min() == -7
+
+
+def test_qmax_for_bits():
+    assert orc.qmax_for_bits(4) == 7 and orc.qmax_for_bits(8) == 127
+    with pytest.raises(ValueError):
+        orc.qmax_for_bits(6)
+
+
+def test_8bit_textbook_and_error_bound():
+    rng = np.random.default_rng(31)
+    X = (rng.standard_normal((12, 128)) * rng.uniform(0.1, 30, (12, 1)))
+    X = X.astype(np.float16)
+    X[4] = 0
+    perm = np.arange(128, dtype=np.int32)
+    xq, s_x, x_rot, codes = orc.rotate_quant_act(X, perm, 1, bits=8)
+    assert np.array_equal(xq, codes) and codes.dtype == np.int8
+    for i in range(12):   # independent scalar loop, qmax 127
+        v = X[i].astype(np.float32)
+        amax = max(abs(float(t)) for t in v)
+        sc = float(np.float32(np.float32(amax) / np.float32(127)))
+        assert s_x[i] == np.float32(sc)
+        for k in range(128):
+            if sc == 0:
+                assert codes[i, k] == 0
+                continue
+            q = round(float(np.float32(np.float32(v[k]) / np.float32(sc))))
+            assert codes[i, k] == max(-127, min(127, q))
+    _, s2, r2, c2 = orc.rotate_quant_act(X, _perm(128, 3), 32, bits=8)
+    assert c2.min() >= -127 and c2.max() <= 127
+    err = np.abs(r2.astype(np.float64) - c2 * s2[:, None].astype(np.float64))
+    assert np.all(err <= s2[:, None] * (0.5 + 1e-5))
+    hit = np.abs(c2[np.arange(12), np.argmax(np.abs(r2), axis=1)])
+    assert np.all(hit[s2 > 0] == 127)
+
+
+def test_8bit_linear_one_hot_closed_form():
+    """One-hot activation rows (b = 1, identity swap) times constant weight
+    rows: the codes are +-qmax on both sides, so y = x * w up to the fp32
+    rounding of the two scales, at every bit setting."""
+    K, N = 64, 5
+    X = np.zeros((3, K), dtype=np.float32)
+    X[0, 3], X[1, 40], X[2, 63] = 2.5, -7.0, 0.375
+    wv = np.array([0.5, -1.25, 3.0, -0.0625, 8.0], dtype=np.float32)
+    W = np.repeat(wv[:, None], K, axis=1)
+    perm = np.arange(K, dtype=np.int32)
+    for a_bits, w_bits in [(4, 4), (8, 4), (8, 8)]:
+        _, s_w, _, qw = orc.prepare_weights(W, perm, 1, bits=w_bits)
+        assert np.all(np.abs(qw) == orc.qmax_for_bits(w_bits))
+        y = orc.obs_linear(X, perm, 1, qw, s_w, a_bits=a_bits)
+        ref = X.sum(axis=1)[:, None].astype(np.float64) * wv[None, :]
+        assert np.allclose(y, ref, rtol=4e-7, atol=0)
+
+
+def test_quant_linear_bruteforce_8bit():
+    rng = np.random.default_rng(5)
+    qx = rng.integers(-127, 128, (4, 48))
+    qw = rng.integers(-7, 8, (3, 48))
+    s_x = rng.uniform(0.1, 1, 4).astype(np.float32)
+    s_w = rng.uniform(0.1, 1, 3).astype(np.float32)
+    y, acc = orc.quant_linear(qx, s_x, qw, s_w, 16)
+    for i in range(4):
+        for n in range(3):
+            a = sum(int(qx[i, k]) * int(qw[n, k]) for k in range(48))
+            assert acc[i, n] == a
+            assert y[i, n] == a * float(s_x[i]) * float(s_w[n]) / 16.0
+
+
+def test_more_bits_less_error():
+    """W8A8 < W4A8 < W4A4 in output error against the fp64 product (the
+    ordering Tab. 3 shows for every method)."""
+    rng = np.random.default_rng(17)
+    K, M, N, b = 256, 64, 96, 64
+    X = rng.standard_normal((M, K)).astype(np.float16)
+    W = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
+    ref = orc.linear_fp64(X, W)
+    perm = orc.build_permutation(orc.outlier_scores(X.astype(np.float32)[None]))
+    errs = []
+    for a_bits, w_bits in [(4, 4), (8, 4), (8, 8)]:
+        _, s_w, _, qw = orc.prepare_weights(W, perm, b, bits=w_bits)
+        y = orc.obs_linear(X, perm, b, qw, s_w, a_bits=a_bits)
+        errs.append(np.linalg.norm(y - ref) / np.linalg.norm(ref))
+    assert errs[2] < errs[1] < errs[0]
+
+
+@pytest.mark.parametrize("wrong", [lambda bits: 2 ** (bits - 1),
+                                   lambda bits: 2 ** bits - 1])
+def test_8bit_planted_grid_mistake_is_caught(monkeypatch, wrong):
+    monkeypatch.setattr(orc, "qmax_for_bits", wrong)
+    with pytest.raises(AssertionError):
+        test_8bit_hand_example()
