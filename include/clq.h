@@ -66,7 +66,8 @@ typedef int32_t clq_dtype;
 #define CLQ_BF16 1
 
 /*
- * Layout of an array of INT4 codes (activations or weights), `rows` x K:
+ * Layout of an array of codes (activations or weights), `rows` x K.  The
+ * 4-bit layouts:
  *  CLQ_CODES_INT4_PACKED  [rows][K/2] bytes, two codes per byte (code 2j in
  *                         the low nibble), 4-bit two's complement; the
  *                         storage format.
@@ -76,11 +77,19 @@ typedef int32_t clq_dtype;
  *                         tensor-core GEMM loads with TMA directly, without
  *                         expanding nibbles in every CTA.
  * The codes are the same INT4 values in both layouts and every call gives
- * identical results for either.
+ * identical results for either.  The 8-bit layout (the W4A8 and W8A8 bit
+ * settings of Sec. 4.1; codes q in [-127, 127], s = r / 127):
+ *  CLQ_CODES_E4M3_SPLIT   [rows][2][K] bytes: for each row, plane 0 holds the
+ *                         E4M3 encoding of 16 h and plane 1 that of l, where
+ *                         h = floor((q + 8) / 16) in [-8, 8] and
+ *                         l = q - 16 h in [-8, 7]; both are E4M3 values, so
+ *                         the tensor cores take q = 16 h + l as two MMAs
+ *                         into one accumulator.
  */
 typedef int32_t clq_codes;
 #define CLQ_CODES_INT4_PACKED 0
 #define CLQ_CODES_E4M3 1
+#define CLQ_CODES_E4M3_SPLIT 2
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char* clq_status_string(clq_status status);
@@ -158,13 +167,27 @@ clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N,
                                float* s_w, float* w_rot_dbg, void* stream);
 
 /*
+ * clq_prepare_weights in any code layout (`w_codes`): 4-bit codes (qmax 7)
+ * for CLQ_CODES_INT4_PACKED ([N][K/2]) or CLQ_CODES_E4M3 ([N][K]), 8-bit
+ * codes (qmax 127, the W8A8 setting) for CLQ_CODES_E4M3_SPLIT ([N][2][K]).
+ * The clip bound caps max_k |W~[n][k]| as above.
+ */
+clq_status clq_prepare_weights_codes(const void* W, clq_dtype dtype, int32_t N,
+                                     int32_t K, int32_t ldw,
+                                     const int32_t* perm, int32_t b,
+                                     const float* clip, clq_codes w_codes,
+                                     uint8_t* Wq, float* s_w, float* w_rot_dbg,
+                                     void* stream);
+
+/*
  * Online activation rotate + quantize (Sec. 3.1 dynamic quantization with
  * Sec. 3.3's online fast Hadamard): X~ = X_p H in fp32, s_x[i] =
- * max_k |X~[i][k]| / 7, Xq[i] = pack(clamp(rint(X~[i] / s_x[i]), -7, 7)).
+ * max_k |X~[i][k]| / qmax, codes clamp(rint(X~[i] / s_x[i]), -qmax, qmax),
+ * qmax = 7 for the 4-bit layouts and 127 for CLQ_CODES_E4M3_SPLIT.
  * One HBM pass over X.  X: device [M][ldx] of `dtype`.  perm: device int32
- * [K].  Xq: device uint8 codes in layout `x_codes` ([M][K/2] packed or
- * [M][K] E4M3).  s_x: device fp32 [M].  x_rot_dbg: device fp32 [M][K] or
- * NULL (receives X~).
+ * [K].  Xq: device uint8 codes in layout `x_codes` ([M][K/2] packed,
+ * [M][K] E4M3 or [M][2][K] split).  s_x: device fp32 [M].  x_rot_dbg:
+ * device fp32 [M][K] or NULL (receives X~).
  */
 clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M,
                                 int32_t K, int32_t ldx, const int32_t* perm,
@@ -198,6 +221,26 @@ clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes,
                            const void* bias, int32_t M, int32_t N, int32_t K,
                            int32_t b, clq_dtype out_dtype, void* Y,
                            int32_t* acc_dbg, void* stream);
+
+/*
+ * The product at any of the paper's bit settings (Sec. 4.1), with the same
+ * epilogue as clq_w4a4_linear: Y[i][n] = out_dtype(acc[i][n] * s_x[i] *
+ * s_w[n] / b + bias[n]), acc[i][n] = sum_k qx[i][k] * qw[n][k].
+ *  W4A4  x_codes and w_codes 4-bit layouts (as clq_w4a4_linear);
+ *  W4A8  x_codes CLQ_CODES_E4M3_SPLIT, w_codes CLQ_CODES_E4M3;
+ *  W8A8  both CLQ_CODES_E4M3_SPLIT.
+ * Other combinations return CLQ_ERR_UNSUPPORTED.  W4A4 and W4A8
+ * accumulators are exact integers for every K <= 16384; W8A8 accumulators
+ * are exact while every partial sum stays below 2^24 in magnitude (always
+ * for K <= 896) and carry fp32 rounding beyond.  acc_dbg (int32 [M][N] or
+ * NULL) receives the accumulators rounded to integers.  Arguments otherwise
+ * as for clq_w4a4_linear.
+ */
+clq_status clq_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x,
+                      const uint8_t* W, clq_codes w_codes, const float* s_w,
+                      const void* bias, int32_t M, int32_t N, int32_t K,
+                      int32_t b, clq_dtype out_dtype, void* Y,
+                      int32_t* acc_dbg, void* stream);
 
 /*
  * Bytes of device workspace clq_fused_linear needs for M tokens of K

@@ -20,7 +20,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libclq.so")
 
 CLQ_F16, CLQ_BF16 = 0, 1
-CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3 = 0, 1
+CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3, CLQ_CODES_E4M3_SPLIT = 0, 1, 2
 STATUS = {0: "CLQ_OK", 1: "CLQ_ERR_INVALID_ARG", 2: "CLQ_ERR_SHAPE",
           3: "CLQ_ERR_ALIGN", 4: "CLQ_ERR_UNSUPPORTED", 5: "CLQ_ERR_CUDA",
           6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX",
@@ -32,7 +32,8 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_fused_linear_noalloc", "clq_get_device_status",
            "clq_selftest_bounded_wait", "clq_outlier_scores_metric",
            "clq_peak_tcgen05_e4m3",
-           "clq_peak_mma_sync", "clq_peak_hbm_read")
+           "clq_peak_mma_sync", "clq_peak_hbm_read",
+           "clq_prepare_weights_codes", "clq_linear")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -61,6 +62,10 @@ _SIGS = {
     "clq_peak_tcgen05_e4m3": (_I, [_I, _P, _P]),
     "clq_peak_mma_sync": (_I, [_I, _I, _P, _P]),
     "clq_peak_hbm_read": (_I, [_P, ctypes.c_uint64, _P, _P]),
+    "clq_prepare_weights_codes": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I,
+                                       _P, _P, _P, _P]),
+    "clq_linear": (_I, [_P, _I, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P,
+                        _P, _P]),
 }
 
 
@@ -107,6 +112,19 @@ def clq_prepare_weights(W, dtype, N, K, ldw, perm, b, clip, Wq, s_w,
                         w_rot_dbg, stream):
     return load().clq_prepare_weights(W, dtype, N, K, ldw, perm, b, clip, Wq,
                                       s_w, w_rot_dbg, stream)
+
+
+def clq_prepare_weights_codes(W, dtype, N, K, ldw, perm, b, clip, w_codes,
+                              Wq, s_w, w_rot_dbg, stream):
+    return load().clq_prepare_weights_codes(W, dtype, N, K, ldw, perm, b,
+                                            clip, w_codes, Wq, s_w, w_rot_dbg,
+                                            stream)
+
+
+def clq_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b,
+               out_dtype, Y, acc_dbg, stream):
+    return load().clq_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N,
+                             K, b, out_dtype, Y, acc_dbg, stream)
 
 
 def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, x_codes, Xq, s_x,
@@ -226,31 +244,49 @@ def build_permutation(scores):
     return perm
 
 
-def prepare_weights(W, perm, b, clip=None, with_rot=False, stream=None):
-    """W [N, K] -> (Wq uint8 [N, K/2], s_w fp32 [N][, w_rot fp32 [N, K]])."""
+def codes_width(codes, K):
+    """Bytes per row of K codes in layout `codes`."""
+    return {CLQ_CODES_INT4_PACKED: K // 2, CLQ_CODES_E4M3: K,
+            CLQ_CODES_E4M3_SPLIT: 2 * K}[codes]
+
+
+def prepare_weights(W, perm, b, clip=None, with_rot=False, stream=None,
+                    codes=CLQ_CODES_INT4_PACKED):
+    """W [N, K] -> (Wq uint8 [N, width], s_w fp32 [N][, w_rot fp32 [N, K]]);
+    4-bit codes packed ([N, K/2], the default) or E4M3 ([N, K]), or 8-bit
+    codes as split planes ([N, 2K], CLQ_CODES_E4M3_SPLIT)."""
     _row_major(W, "W")
     N, K = W.shape
     dev = W.device
-    Wq = torch.empty((N, K // 2), dtype=torch.uint8, device=dev)
+    Wq = torch.empty((N, codes_width(codes, K)), dtype=torch.uint8, device=dev)
     s_w = torch.empty(N, dtype=torch.float32, device=dev)
     rot = (torch.empty((N, K), dtype=torch.float32, device=dev)
            if with_rot else None)
-    _check(clq_prepare_weights(_ptr(W), _dt(W), N, K, W.stride(0), _ptr(perm),
-                               b, _ptr(clip), _ptr(Wq), _ptr(s_w), _ptr(rot),
-                               _stream(stream)), "clq_prepare_weights")
+    if codes == CLQ_CODES_INT4_PACKED:
+        _check(clq_prepare_weights(_ptr(W), _dt(W), N, K, W.stride(0),
+                                   _ptr(perm), b, _ptr(clip), _ptr(Wq),
+                                   _ptr(s_w), _ptr(rot), _stream(stream)),
+               "clq_prepare_weights")
+    else:
+        _check(clq_prepare_weights_codes(_ptr(W), _dt(W), N, K, W.stride(0),
+                                         _ptr(perm), b, _ptr(clip), codes,
+                                         _ptr(Wq), _ptr(s_w), _ptr(rot),
+                                         _stream(stream)),
+               "clq_prepare_weights_codes")
     return (Wq, s_w, rot) if with_rot else (Wq, s_w)
 
 
 def rotate_quant_act(X, perm, b, codes=CLQ_CODES_INT4_PACKED, Xq=None, s_x=None,
                      with_rot=False, stream=None):
     """X [M, K] -> (Xq uint8, s_x fp32 [M][, x_rot fp32 [M, K]]); Xq is
-    [M, K/2] packed (CLQ_CODES_INT4_PACKED) or [M, K] E4M3 (CLQ_CODES_E4M3)."""
+    [M, K/2] packed (CLQ_CODES_INT4_PACKED), [M, K] E4M3 (CLQ_CODES_E4M3) or,
+    for 8-bit codes, [M, 2K] split planes (CLQ_CODES_E4M3_SPLIT)."""
     _row_major(X, "X")
     M, K = X.shape
     dev = X.device
     if Xq is None:
-        width = K if codes == CLQ_CODES_E4M3 else K // 2
-        Xq = torch.empty((M, width), dtype=torch.uint8, device=dev)
+        Xq = torch.empty((M, codes_width(codes, K)), dtype=torch.uint8,
+                         device=dev)
     if s_x is None:
         s_x = torch.empty(M, dtype=torch.float32, device=dev)
     rot = (torch.empty((M, K), dtype=torch.float32, device=dev)
@@ -277,7 +313,10 @@ def codes_layout(t, K):
         return CLQ_CODES_E4M3
     if 2 * t.shape[1] == K:
         return CLQ_CODES_INT4_PACKED
-    raise ValueError("codes must be [rows, K/2] packed or [rows, K] E4M3")
+    if t.shape[1] == 2 * K:
+        return CLQ_CODES_E4M3_SPLIT
+    raise ValueError("codes must be [rows, K/2] packed, [rows, K] E4M3 or "
+                     "[rows, 2K] split")
 
 
 def w4a4_linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
@@ -296,6 +335,25 @@ def w4a4_linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
                            codes_layout(W, K), _ptr(s_w), _ptr(bias), M, N, K,
                            b, _dt(Y), _ptr(Y), _ptr(acc), _stream(stream)),
            "clq_w4a4_linear")
+    return (Y, acc) if with_acc else Y
+
+
+def linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
+           Y=None, with_acc=False, stream=None):
+    """Codes x codes at any bit setting (W4A4, W4A8, W8A8; layouts inferred
+    from the widths) -> Y [M, N] (out_dtype)[, acc int32 [M, N]]."""
+    M = Xq.shape[0]
+    N = W.shape[0]
+    if Y is None:
+        Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
+    acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
+           if with_acc else None)
+    if bias is not None and bias.dtype != Y.dtype:
+        raise TypeError("bias must have the output dtype")
+    _check(clq_linear(_ptr(Xq), codes_layout(Xq, K), _ptr(s_x), _ptr(W),
+                      codes_layout(W, K), _ptr(s_w), _ptr(bias), M, N, K, b,
+                      _dt(Y), _ptr(Y), _ptr(acc), _stream(stream)),
+           "clq_linear")
     return (Y, acc) if with_acc else Y
 
 
@@ -340,48 +398,68 @@ class PreparedLinear:
     """A quantized linear layer: the prepared-weight package (Wq, s_w, perm,
     b, bias) of Sec. 3.3, where the swap vector is the only stored part of G.
 
-    Wq holds the packed INT4 codes (the storage format, 4 bits per weight);
-    We the same codes in the E4M3 execution layout the GEMM loads directly.
-    Activation codes are produced in the E4M3 layout too (they are transient,
-    so their container is chosen for the GEMM).
-    ``state_dict()`` keeps only the packed codes; ``from_state_dict()``
+    At W4A4 and W4A8, Wq holds the packed INT4 codes (the storage format,
+    4 bits per weight) and We the same codes in the E4M3 execution layout the
+    GEMM loads directly.  At W8A8, Wq holds the 8-bit codes as split planes
+    ([N, 2K], which is also the execution layout).  Activation codes are
+    produced in an execution layout too (they are transient): E4M3 for
+    4-bit, split planes for 8-bit activations (a_bits).
+    ``state_dict()`` keeps only the storage codes; ``from_state_dict()``
     expands them again.  Calling the object runs the separate rotate-quant
-    and GEMM kernels (``fused=False``) or the fused kernel.
+    and GEMM kernels (``fused=False``) or, at W4A4, the fused kernel.
     """
 
-    def __init__(self, Wq, s_w, perm, b, bias=None, We=None):
+    def __init__(self, Wq, s_w, perm, b, bias=None, We=None, a_bits=4):
         self.Wq, self.s_w, self.perm, self.b, self.bias = Wq, s_w, perm, b, bias
-        self.We = expand_weights(Wq) if We is None else We
+        K = perm.numel()
+        self.w_bits = 8 if Wq.shape[1] == 2 * K else 4
+        if a_bits not in (4, 8) or (self.w_bits == 8 and a_bits != 8):
+            raise ValueError("bit settings are W4A4, W4A8 and W8A8")
+        self.a_bits = a_bits
+        if self.w_bits == 8:
+            self.We = Wq
+        else:
+            self.We = expand_weights(Wq) if We is None else We
 
     @classmethod
-    def from_weight(cls, W, perm, b, bias=None, clip=None):
+    def from_weight(cls, W, perm, b, bias=None, clip=None, a_bits=4, w_bits=4):
         perm = perm.to(W.device, torch.int32).contiguous()
-        Wq, s_w = prepare_weights(W.contiguous(), perm, b, clip)
-        return cls(Wq, s_w, perm, b, bias)
+        codes = CLQ_CODES_E4M3_SPLIT if w_bits == 8 else CLQ_CODES_INT4_PACKED
+        Wq, s_w = prepare_weights(W.contiguous(), perm, b, clip, codes=codes)
+        return cls(Wq, s_w, perm, b, bias, a_bits=a_bits)
 
     def state_dict(self):
         d = dict(Wq=self.Wq, s_w=self.s_w, perm=self.perm,
-                 b=torch.tensor(self.b))
+                 b=torch.tensor(self.b), a_bits=torch.tensor(self.a_bits))
         if self.bias is not None:
             d["bias"] = self.bias
         return d
 
     @classmethod
     def from_state_dict(cls, d):
-        return cls(d["Wq"], d["s_w"], d["perm"], int(d["b"]), d.get("bias"))
+        a_bits = int(d["a_bits"]) if "a_bits" in d else 4
+        return cls(d["Wq"], d["s_w"], d["perm"], int(d["b"]), d.get("bias"),
+                   a_bits=a_bits)
 
     def __call__(self, X, fused=False, workspace=None, stream=None, Y=None,
                  Xq=None, s_x=None):
-        """Y = X W^T + bias through the W4A4 path.  Y, and the activation
-        codes / scales of the separate path (Xq [M, K] uint8, s_x [M] fp32),
-        may be passed in to avoid allocations."""
+        """Y = X W^T + bias at the layer's bit setting.  Y, and the activation
+        codes / scales of the separate path (Xq [M, K] uint8 for 4-bit, [M, 2K]
+        for 8-bit activations; s_x [M] fp32), may be passed in to avoid
+        allocations."""
         if fused:
+            if self.a_bits != 4:
+                raise ValueError("the fused kernel runs W4A4 only")
             return fused_linear(X, self.perm, self.b, self.We, self.s_w,
                                 self.bias, Y=Y, workspace=workspace, stream=stream)
-        Xq, s_x = rotate_quant_act(X, self.perm, self.b, CLQ_CODES_E4M3,
+        codes = CLQ_CODES_E4M3_SPLIT if self.a_bits == 8 else CLQ_CODES_E4M3
+        Xq, s_x = rotate_quant_act(X, self.perm, self.b, codes,
                                    Xq=Xq, s_x=s_x, stream=stream)
-        return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, X.shape[1],
-                           self.bias, out_dtype=X.dtype, Y=Y, stream=stream)
+        if self.a_bits == 4:
+            return w4a4_linear(Xq, s_x, self.We, self.s_w, self.b, X.shape[1],
+                               self.bias, out_dtype=X.dtype, Y=Y, stream=stream)
+        return linear(Xq, s_x, self.We, self.s_w, self.b, X.shape[1],
+                      self.bias, out_dtype=X.dtype, Y=Y, stream=stream)
 
 
 class HostPipeline:

@@ -70,7 +70,9 @@ clq_status check_k_b(int K, int b) {
 
 bool valid_dtype(int d) { return d == CLQ_F16 || d == CLQ_BF16; }
 
+// 4-bit layouts (W4A4 entry points) and every layout (rotate-quant, clq_linear).
 bool valid_codes(int f) { return f == CLQ_CODES_INT4_PACKED || f == CLQ_CODES_E4M3; }
+bool valid_any_codes(int f) { return valid_codes(f) || f == CLQ_CODES_E4M3_SPLIT; }
 
 // Launch of the fused kernel on a workspace laid out as `ws` (validated).
 clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
@@ -107,7 +109,7 @@ clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, in
 clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ld,
                                const int32_t* perm, int32_t b, const float* clip, int codes,
                                uint8_t* Q, float* S, float* rot, void* stream) {
-  if (!valid_dtype(dtype) || !valid_codes(codes) || M < 0) return CLQ_ERR_INVALID_ARG;
+  if (!valid_dtype(dtype) || !valid_any_codes(codes) || M < 0) return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
   if (ld < K) return CLQ_ERR_SHAPE;
@@ -132,7 +134,7 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   a.rot = rot;
   a.status = status;
   a.logb = log2i(b);
-  a.e4m3 = codes == CLQ_CODES_E4M3 ? 1 : 0;
+  a.e4m3 = codes == CLQ_CODES_E4M3 ? 1 : codes == CLQ_CODES_E4M3_SPLIT ? 2 : 0;
   return from_cuda(
       clq::launch_rotate_quant(a, dtype, log2i(b), static_cast<cudaStream_t>(stream)));
 }
@@ -215,6 +217,14 @@ clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N, int32_
                              w_rot_dbg, stream);
 }
 
+clq_status clq_prepare_weights_codes(const void* W, clq_dtype dtype, int32_t N, int32_t K,
+                                     int32_t ldw, const int32_t* perm, int32_t b,
+                                     const float* clip, clq_codes w_codes, uint8_t* Wq,
+                                     float* s_w, float* w_rot_dbg, void* stream) {
+  return rotate_quant_common(W, dtype, N, K, ldw, perm, b, clip, w_codes, Wq, s_w, w_rot_dbg,
+                             stream);
+}
+
 clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
                                 const int32_t* perm, int32_t b, clq_codes x_codes, uint8_t* Xq,
                                 float* s_x, float* x_rot_dbg, void* stream) {
@@ -239,9 +249,23 @@ clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_
                            const uint8_t* W, clq_codes w_codes, const float* s_w,
                            const void* bias, int32_t M, int32_t N, int32_t K, int32_t b,
                            clq_dtype out_dtype, void* Y, int32_t* acc_dbg, void* stream) {
-  if (!valid_dtype(out_dtype) || !valid_codes(x_codes) || !valid_codes(w_codes) || M < 0 ||
-      N < 0)
+  if (!valid_codes(x_codes) || !valid_codes(w_codes)) return CLQ_ERR_INVALID_ARG;
+  return clq_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b, out_dtype, Y, acc_dbg,
+                    stream);
+}
+
+clq_status clq_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x, const uint8_t* W,
+                      clq_codes w_codes, const float* s_w, const void* bias, int32_t M,
+                      int32_t N, int32_t K, int32_t b, clq_dtype out_dtype, void* Y,
+                      int32_t* acc_dbg, void* stream) {
+  if (!valid_dtype(out_dtype) || !valid_any_codes(x_codes) || !valid_any_codes(w_codes) ||
+      M < 0 || N < 0)
     return CLQ_ERR_INVALID_ARG;
+  // 8-bit operands: W4A8 (split activations, E4M3 weights) and W8A8 only.
+  if ((x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT) &&
+      !(x_codes == CLQ_CODES_E4M3_SPLIT &&
+        (w_codes == CLQ_CODES_E4M3 || w_codes == CLQ_CODES_E4M3_SPLIT)))
+    return CLQ_ERR_UNSUPPORTED;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
   if (M == 0 || N == 0) return CLQ_OK;

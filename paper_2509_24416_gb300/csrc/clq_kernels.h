@@ -15,13 +15,14 @@ struct RotateQuantArgs {
   int32_t M, K, ld;
   const int32_t* perm;   // [K]
   const float* clip;     // [M] or null (weights only)
-  uint8_t* Q;            // [M][K/2] packed, or [M][K] E4M3 when e4m3 != 0
+  uint8_t* Q;            // [M][K/2] packed, [M][K] E4M3, or [M][2][K] split planes
   float* S;              // [M]
   float* rot;            // [M][K] or null
   int32_t rows_per_tile; // filled in by the launcher
   int32_t* status;       // device status word
   int32_t logb;          // log2(b)
-  int32_t e4m3;          // codes layout: 0 packed nibbles, 1 one E4M3 byte each
+  int32_t e4m3;          // codes layout: 0 packed nibbles, 1 one E4M3 byte each,
+                         // 2 8-bit codes as two E4M3 planes (16 h, l)
 };
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
@@ -45,7 +46,9 @@ struct GemmArgs {
 };
 
 // A = activation codes, B = weight codes, each in layout CLQ_CODES_INT4_PACKED
-// ([rows][K/2]) or CLQ_CODES_E4M3 ([rows][K]); TMA maps are built here.
+// ([rows][K/2]), CLQ_CODES_E4M3 ([rows][K]) or, for 8-bit codes,
+// CLQ_CODES_E4M3_SPLIT ([rows][2][K]; A split with B E4M3 or split); TMA maps
+// are built here.
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st);
 
@@ -70,14 +73,19 @@ cudaError_t launch_wait_selftest(uint64_t timeout_ns, int32_t* status, cudaStrea
 bool encode_tma_2d(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize, const void* base,
                    uint64_t inner, uint64_t rows, uint32_t box_inner, uint32_t box_rows,
                    CUtensorMapSwizzle swz);
+bool encode_tma_2d_strided(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize,
+                           const void* base, uint64_t inner, uint64_t rows,
+                           uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows,
+                           CUtensorMapSwizzle swz);
 bool encode_tma_2d_u8(CUtensorMap* map, const void* base, uint64_t inner_bytes,
                       uint64_t rows, uint32_t box_inner, uint32_t box_rows);
 // 2-byte output tile map for the epilogue stores (box 32 columns x 128 rows).
 bool encode_tma_out_tile(CUtensorMap* map, void* Y, int M, int N);
 int sm_count();  // cached per device
-// TMA map of an INT4 code array (rows x K) in layout `codes`, box_rows rows.
+// TMA map of a code array (rows x K) in layout `codes`, box_rows rows; for
+// the split layout, of plane `plane` (0 or 1).
 bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows, int K,
-                      int box_rows);
+                      int box_rows, int plane);
 // Peak-rate microbenchmarks (peaks.cu); *macs / *ops receive the work done.
 cudaError_t launch_peak_tcgen05(int iters, int32_t* status, cudaStream_t st, long long* macs);
 cudaError_t launch_peak_mma_sync(int kind, int iters, int32_t* sink, cudaStream_t st,

@@ -131,8 +131,8 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   if (e != cudaSuccess) return e;
 
   CUtensorMap mapA, mapB, mapY;
-  if (!encode_codes_map(&mapA, rq.Q, CLQ_CODES_E4M3, g.M, g.K, BM) ||
-      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn))
+  if (!encode_codes_map(&mapA, rq.Q, CLQ_CODES_E4M3, g.M, g.K, BM, 0) ||
+      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn, 0))
     return cudaErrorInvalidValue;
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
   if (use_tma_store) {

@@ -8,6 +8,12 @@
 // tcgen05.mma kind::f8f6f4 with fp32 accumulation in tensor memory; the
 // integer accumulators come out exact as long as the fp32 sums are exact
 // (checked bit for bit against the int64 oracle, +-7 codes at K = 16384).
+// 8-bit codes (W4A8, W8A8) arrive as two E4M3 planes, 16 h and l with
+// q = 16 h + l, and every pair of planes is multiplied into the same
+// accumulator.  Every partial sum of W4A8 stays below 2^24 for K <= 16384
+// (at most (128 + 8) * 7 per code pair), so it is exact too; W8A8 is exact
+// while the partial sums stay below 2^24 (any codes at K <= 896: at most
+// (128 + 8)^2 per code pair) and takes fp32 rounding beyond.
 //
 // Persistent: one CTA per SM walks 128 (M) x 256 (N) tiles in a static
 // round-robin order, K step 128 codes.  Each operand arrives either as E4M3
@@ -47,7 +53,10 @@ constexpr int MIN_THREADS = (WARP_UNPACK0 + NUM_UNPACK / 32) * 32;  // 448
 constexpr int MAX_STAGES = 6;
 
 // Tile BM x BNT (BNT = 256, or 192 for E4M3 operands where N splits better).
-template <bool APACK, bool BPACK, int BNT = BN>
+// PA / PB: E4M3 planes per operand, 1 for 4-bit codes, 2 for 8-bit codes
+// split as q = 16 h + l (plane 0 holds 16 h, plane 1 holds l; both E4M3
+// values, so the MMAs of the two planes add up to q in one accumulator).
+template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1>
 struct Cfg {
   static constexpr bool UNPACK = APACK || BPACK;
   static constexpr int EPI_WARPS = UNPACK ? 4 : 8;
@@ -55,24 +64,27 @@ struct Cfg {
   static constexpr int EPI_THREADS = 32 * EPI_WARPS;
   static constexpr int EPI_NBUF = 8 / EPI_WARPS;  // staging buffers per warp
   static constexpr int EPI_NCOL = BNT * 4 / EPI_WARPS;  // columns per warp
-  static constexpr int BU = BNT * BK;    // E4M3 B stage
+  static constexpr int AU = PA * A_U;    // E4M3 A stage (all planes)
+  static constexpr int BU = PB * BNT * BK;  // E4M3 B stage (all planes)
   static constexpr int BP = BNT * BKP;   // packed B stage
-  static constexpr int STAGE = A_U + BU + (APACK ? A_P : 0) + (BPACK ? BP : 0);
+  static constexpr int STAGE = AU + BU + (APACK ? A_P : 0) + (BPACK ? BP : 0);
   static constexpr int FIXED = EPI_TOTAL + 4 * BNT * 4;
   static constexpr int S0 = (222 * 1024 - FIXED) / STAGE;
   static constexpr int S = S0 > MAX_STAGES ? MAX_STAGES : S0;  // pipeline stages
   static constexpr size_t OFF_UA = 0;                           // E4M3 operands
-  static constexpr size_t OFF_UB = OFF_UA + S * A_U;
+  static constexpr size_t OFF_UB = OFF_UA + S * AU;
   static constexpr size_t OFF_PA = OFF_UB + S * BU;             // packed staging
   static constexpr size_t OFF_PB = OFF_PA + (APACK ? S * A_P : 0);
   static constexpr size_t OFF_EPI = OFF_PB + (BPACK ? S * BP : 0);
   static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;        // [2][2][BNT] floats
   static constexpr size_t BYTES = OFF_COL + 4 * BNT * sizeof(float);
-  static constexpr uint32_t TX = (APACK ? A_P : A_U) + (BPACK ? BP : BU);
+  static constexpr uint32_t TX = (APACK ? A_P : AU) + (BPACK ? BP : BU);
   // two accumulators of BNT columns, 2 * BNT rounded up to the power of two
   // tcgen05.alloc takes
   static constexpr uint32_t TMEM = 2 * BNT <= 256 ? 256u : 512u;
   static_assert(S >= 2, "pipeline needs two stages");
+  static_assert((PA == 1 || PA == 2) && (PB == 1 || PB == 2), "one or two planes");
+  static_assert(!UNPACK || (PA == 1 && PB == 1), "8-bit planes come as E4M3 only");
 };
 
 struct __align__(8) Barriers {
@@ -89,7 +101,9 @@ struct __align__(8) Barriers {
 struct Maps {
   const CUtensorMap* A;
   const CUtensorMap* B;
-  const CUtensorMap* Y;  // null: direct stores
+  const CUtensorMap* Y;   // null: direct stores
+  const CUtensorMap* A2;  // second planes (PA / PB == 2), else unused
+  const CUtensorMap* B2;
 };
 
 __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
@@ -104,9 +118,9 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 
 // Barrier init (thread 0) and TMEM allocation (warp WARP_MMA); the caller
 // follows with tcgen05 fences around a CTA barrier.
-template <bool APACK, bool BPACK, int BNT = BN>
+template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1>
 __device__ __forceinline__ void setup(Barriers* bars) {
-  using C = Cfg<APACK, BPACK, BNT>;
+  using C = Cfg<APACK, BPACK, BNT, PA, PB>;
   constexpr int S = C::S;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -147,10 +161,11 @@ __device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, ui
 
 // EPI_PREFETCH: let the epilogue prefetch TMEM (taken only in the 320-thread
 // configuration, where registers allow it).
-template <typename OutT, bool APACK, bool BPACK, int BNT = BN, bool EPI_PREFETCH = true>
+template <typename OutT, bool APACK, bool BPACK, int BNT = BN, bool EPI_PREFETCH = true,
+          int PA = 1, int PB = 1>
 __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
                                          Barriers* bars, uint32_t tmem, const uint32_t* ready) {
-  using C = Cfg<APACK, BPACK, BNT>;
+  using C = Cfg<APACK, BPACK, BNT, PA, PB>;
   constexpr int S = C::S;
   volatile int32_t* abort = &bars->abort;
 
@@ -164,6 +179,8 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
     if (lane == 0) {
       prefetch_tensor_map(maps.A);
       prefetch_tensor_map(maps.B);
+      if (PA == 2) prefetch_tensor_map(maps.A2);
+      if (PB == 2) prefetch_tensor_map(maps.B2);
       if (maps.Y != nullptr) prefetch_tensor_map(maps.Y);
       int it = 0;  // K steps issued so far (all tiles)
       int ready_m = -1;
@@ -191,11 +208,17 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
           if (APACK)
             tma_load_2d(smem + C::OFF_PA + s * A_P, maps.A, kb * BKP, m0, &bars->tma_full[s]);
           else
-            tma_load_2d(smem + C::OFF_UA + s * A_U, maps.A, kb * BK, m0, &bars->tma_full[s]);
+            tma_load_2d(smem + C::OFF_UA + s * C::AU, maps.A, kb * BK, m0, &bars->tma_full[s]);
+          if (PA == 2)
+            tma_load_2d(smem + C::OFF_UA + s * C::AU + A_U, maps.A2, kb * BK, m0,
+                        &bars->tma_full[s]);
           if (BPACK)
             tma_load_2d(smem + C::OFF_PB + s * C::BP, maps.B, kb * BKP, n0, &bars->tma_full[s]);
           else
             tma_load_2d(smem + C::OFF_UB + s * C::BU, maps.B, kb * BK, n0, &bars->tma_full[s]);
+          if (PB == 2)
+            tma_load_2d(smem + C::OFF_UB + s * C::BU + BNT * BK, maps.B2, kb * BK, n0,
+                        &bars->tma_full[s]);
         }
       }
       // On an abort, the copies already in flight must land before exit.
@@ -226,12 +249,17 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_addr(smem + C::OFF_UA + s * A_U);
+          const uint32_t a0 = smem_addr(smem + C::OFF_UA + s * C::AU);
           const uint32_t b0 = smem_addr(smem + C::OFF_UB + s * C::BU);
 #pragma unroll
-          for (int k = 0; k < BK / 32; ++k)
-            mma_e4m3(d, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc,
-                     (kb | k) != 0 ? 1u : 0u);
+          for (int pa = 0; pa < PA; ++pa)
+#pragma unroll
+            for (int pb = 0; pb < PB; ++pb)
+#pragma unroll
+              for (int k = 0; k < BK / 32; ++k)
+                mma_e4m3(d, sw128_desc(a0 + pa * A_U + k * 32),
+                         sw128_desc(b0 + pb * BNT * BK + k * 32), idesc,
+                         (kb | pa | pb | k) != 0 ? 1u : 0u);
           mma_commit(&bars->mma_done[s]);
         }
         if (ok) mma_commit(&bars->acc_full[buf]);
@@ -295,7 +323,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
           break;
         }
         if (APACK)
-          unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * A_U,
+          unpack_rows<BM, NUM_UNPACK>(smem + C::OFF_PA + s * A_P, smem + C::OFF_UA + s * C::AU,
                                       ut);
         if (BPACK)
           unpack_rows<BNT, NUM_UNPACK>(smem + C::OFF_PB + s * C::BP,

@@ -2,7 +2,8 @@
 // linear kernel.  It applies the OBS transform of arxiv 2509.24416 Sec. 3.3
 // to rows of X (column gather by the swap vector `perm`, then the block
 // Sylvester Hadamard H_b) and quantizes each row to symmetric INT4 with a
-// dynamic fp32 scale (Sec. 3.1, Eq. 1 with l = -r).
+// dynamic fp32 scale (Sec. 3.1, Eq. 1 with l = -r), or to symmetric INT8
+// (qmax 127) for the split-plane layout of the W4A8 / W8A8 settings.
 //
 // Every thread of the CTA takes part.  The CTA walks tiles of R rows.  Raw
 // rows stream into a ring of STAGES shared-memory buffers (STRIDE bytes
@@ -19,9 +20,10 @@
 //  2. the remaining butterfly stages up to stride 16 in registers (paired
 //     fp32x2 arithmetic), strides 32 .. b / 2 across lanes with shuffles,
 //     then the row's |x| maximum: warp reduction and a shared atomicMax;
-//  3. one CTA barrier; then s = absmax / 7, codes rint(x / s) (x times an
+//  3. one CTA barrier; then s = absmax / qmax, codes rint(x / s) (x times an
 //     approximate reciprocal of s, rounded with the 1.5 * 2^23 constant,
-//     ties to even), stored as packed nibbles or one E4M3 byte per code.
+//     ties to even), stored as packed nibbles, one E4M3 byte per code, or
+//     (8 bits) two E4M3 planes 16 h and l with q = 16 h + l, l in [-8, 7].
 // The row maxima are triple-buffered over tiles, so the barrier of tile i
 // also separates the readers of tile i - 1 from the reset for tile i + 2.
 #pragma once
@@ -128,8 +130,10 @@ __device__ __forceinline__ void issue_tile(const RotateQuantArgs& a, uint8_t* ds
 // == null) or are claimed one at a time from a global counter (so that CTAs
 // which never become resident own no rows).  After each tile, every thread
 // calls publish(row0, rows) once its own stores of that tile are issued.
-// LOGB = log2(b) when known at compile time, or -1 to read a.logb.
-template <typename T, int LOGB, bool CLIP, int STRIDE, int STAGES, typename Publish>
+// LOGB = log2(b) when known at compile time, or -1 to read a.logb.  SPLIT:
+// 8-bit codes in the split-plane layout (a.e4m3 == 2), else 4-bit codes.
+template <typename T, int LOGB, bool CLIP, int STRIDE, int STAGES, bool SPLIT = false,
+          typename Publish = NoPublish>
 __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
                                     uint32_t* tile_counter, Publish publish) {
   const int K = a.K;
@@ -306,10 +310,12 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
         const int row = row0 + r_local;
         float am = __uint_as_float(amax[par * R + r_local]);
         if (CLIP) am = fminf(am, __ldg(a.clip + row));
-        // s = am / 7: quotient by the reciprocal constant, one residual
+        // s = am / qmax: quotient by the reciprocal constant, one residual
         // correction.
-        const float q1 = am * (1.0f / 7.0f);
-        const float s_row = fmaf(fmaf(-7.0f, q1, am), 1.0f / 7.0f, q1);
+        constexpr float qmax = SPLIT ? 127.0f : 7.0f;
+        constexpr float rqmax = SPLIT ? 1.0f / 127.0f : 1.0f / 7.0f;
+        const float q1 = am * rqmax;
+        const float s_row = fmaf(fmaf(-qmax, q1, am), rqmax, q1);
         if (seg == 0) a.S[row] = s_row;
         if (a.rot != nullptr) {
           float4* dst = reinterpret_cast<float4*>(a.rot + static_cast<size_t>(row) * K + seg * 32);
@@ -333,14 +339,46 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
 #pragma unroll
           for (int k = 0; k < 16; ++k) v[k] = __ffma2_rn(v[k], rc2, magic);
         }
-        if (CLIP) {  // clipped weight rows: |v / s| may exceed 7
+        if (CLIP) {  // clipped weight rows: |v / s| may exceed qmax
+          const float lo = 12582912.0f - qmax, hi = 12582912.0f + qmax;
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
-            v[k].x = fminf(fmaxf(v[k].x, 12582905.0f), 12582919.0f);
-            v[k].y = fminf(fmaxf(v[k].y, 12582905.0f), 12582919.0f);
+            v[k].x = fminf(fmaxf(v[k].x, lo), hi);
+            v[k].y = fminf(fmaxf(v[k].y, lo), hi);
           }
         }
-        if (a.e4m3) {
+        if constexpr (SPLIT) {
+          // q = 16 h + l with h = floor((q + 8) / 16): plane 0 gets the E4M3
+          // encoding of 16 h (a multiple of 16 in [-128, 128]), plane 1 that
+          // of l in [-8, 7]; every step is exact in fp32.
+          uint32_t wh[8], wl[8];
+#pragma unroll
+          for (int k = 0; k < 16; k += 2) {
+            uint32_t hh[2], ll[2];
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              const float2 q = __fadd2_rn(v[k + j], make_float2(-12582912.0f, -12582912.0f));
+              const float2 t = __fmul2_rn(__fadd2_rn(q, make_float2(8.f, 8.f)),
+                                          make_float2(0.0625f, 0.0625f));
+              const float2 h16 = make_float2(16.f * floorf(t.x), 16.f * floorf(t.y));
+              const float2 l = __fadd2_rn(q, make_float2(-h16.x, -h16.y));
+              uint16_t eh, el;
+              asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(eh) : "f"(h16.y), "f"(h16.x));
+              asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(el) : "f"(l.y), "f"(l.x));
+              hh[j] = eh;
+              ll[j] = el;
+            }
+            wh[k >> 1] = hh[0] | (hh[1] << 16);
+            wl[k >> 1] = ll[0] | (ll[1] << 16);
+          }
+          uint4* qh = reinterpret_cast<uint4*>(a.Q + static_cast<size_t>(row) * 2 * K + seg * 32);
+          uint4* ql = reinterpret_cast<uint4*>(a.Q + (static_cast<size_t>(row) * 2 + 1) * K +
+                                               seg * 32);
+          qh[0] = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+          qh[1] = make_uint4(wh[4], wh[5], wh[6], wh[7]);
+          ql[0] = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+          ql[1] = make_uint4(wl[4], wl[5], wl[6], wl[7]);
+        } else if (a.e4m3) {
           // one byte per code: the E4M3 encoding of the integer code
           uint32_t w[8];
 #pragma unroll

@@ -16,21 +16,25 @@ namespace {
 
 using namespace gemm;
 
-template <bool APACK, bool BPACK, int BNT>
+template <bool APACK, bool BPACK, int BNT, int PA, int PB>
 constexpr size_t smem_bytes() {
-  return Cfg<APACK, BPACK, BNT>::BYTES + 1024;  // + alignment slack
+  return Cfg<APACK, BPACK, BNT, PA, PB>::BYTES + 1024;  // + alignment slack
 }
 
-template <typename OutT, bool APACK, bool BPACK, int BNT>
-__global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT>::THREADS), 1)
+// PA / PB = 2: the activation / weight codes are 8-bit, as two E4M3 planes
+// (mapA2 / mapB2 the second plane).
+template <typename OutT, bool APACK, bool BPACK, int BNT, int PA, int PB>
+__global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                      const __grid_constant__ CUtensorMap mapB,
-                     const __grid_constant__ CUtensorMap mapY, GemmArgs g, int use_tma_store) {
+                     const __grid_constant__ CUtensorMap mapY,
+                     const __grid_constant__ CUtensorMap mapA2,
+                     const __grid_constant__ CUtensorMap mapB2, GemmArgs g, int use_tma_store) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  setup<APACK, BPACK, BNT>(&bars);
+  setup<APACK, BPACK, BNT, PA, PB>(&bars);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -38,11 +42,11 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT>::THREADS), 1)
   // Barriers and TMEM are set up; global inputs are read only from here on.
   pdl_wait();
   pdl_launch_dependents();
-  const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
-  pipeline<OutT, APACK, BPACK, BNT>(maps, g, smem, &bars, tmem, nullptr);
+  const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr, &mapA2, &mapB2};
+  pipeline<OutT, APACK, BPACK, BNT, true, PA, PB>(maps, g, smem, &bars, tmem, nullptr);
   tc_fence_before();
   __syncthreads();
-  teardown(tmem, Cfg<APACK, BPACK, BNT>::TMEM);
+  teardown(tmem, Cfg<APACK, BPACK, BNT, PA, PB>::TMEM);
 }
 
 // Packed INT4 weights -> E4M3 execution layout (one code per byte, the byte
@@ -61,9 +65,10 @@ __global__ void expand_weights_kernel(const uint4* __restrict__ src, uint4* __re
 
 }  // namespace
 
-bool encode_tma_2d(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize, const void* base,
-                   uint64_t inner, uint64_t rows, uint32_t box_inner, uint32_t box_rows,
-                   CUtensorMapSwizzle swz) {
+bool encode_tma_2d_strided(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize,
+                           const void* base, uint64_t inner, uint64_t rows,
+                           uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows,
+                           CUtensorMapSwizzle swz) {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (fn == nullptr) {
     void* p = nullptr;
@@ -75,13 +80,20 @@ bool encode_tma_2d(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize, con
     fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
   }
   const cuuint64_t dims[2] = {inner, rows};
-  const cuuint64_t strides[1] = {inner * esize};
+  const cuuint64_t strides[1] = {row_stride_bytes};
   const cuuint32_t box[2] = {box_inner, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   const CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool encode_tma_2d(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize, const void* base,
+                   uint64_t inner, uint64_t rows, uint32_t box_inner, uint32_t box_rows,
+                   CUtensorMapSwizzle swz) {
+  return encode_tma_2d_strided(map, dt, esize, base, inner, rows, inner * esize, box_inner,
+                               box_rows, swz);
 }
 
 
@@ -143,46 +155,56 @@ cudaError_t kernel_setup(const void* func, size_t smem, int threads, int* per_sm
 
 namespace {
 
-template <typename OutT, bool APACK, bool BPACK, int BNT>
-cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB,
-                          const CUtensorMap& mapY, const GemmArgs& g, int use_tma_store,
-                          int grid, cudaStream_t st) {
-  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT>;
-  constexpr size_t smem = smem_bytes<APACK, BPACK, BNT>();
-  constexpr int threads = Cfg<APACK, BPACK, BNT>::THREADS;
+struct MapSet {
+  CUtensorMap A, B, Y, A2, B2;
+};
+
+template <typename OutT, bool APACK, bool BPACK, int BNT, int PA = 1, int PB = 1>
+cudaError_t launch_gemm_t(const MapSet& m, const GemmArgs& g, int use_tma_store, int grid,
+                          cudaStream_t st) {
+  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT, PA, PB>;
+  constexpr size_t smem = smem_bytes<APACK, BPACK, BNT, PA, PB>();
+  constexpr int threads = Cfg<APACK, BPACK, BNT, PA, PB>::THREADS;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, threads, nullptr);
   if (e != cudaSuccess) return e;
-  return launch_pdl(k, grid, threads, smem, st, mapA, mapB, mapY, g, use_tma_store);
+  return launch_pdl(k, grid, threads, smem, st, m.A, m.B, m.Y, m.A2, m.B2, g, use_tma_store);
 }
 
 template <typename OutT>
-cudaError_t launch_gemm_dt(const CUtensorMap& mapA, const CUtensorMap& mapB,
-                           const CUtensorMap& mapY, const GemmArgs& g, bool apack, bool bpack,
-                           int bn, int use_tma_store, int grid, cudaStream_t st) {
+cudaError_t launch_gemm_dt(const MapSet& m, const GemmArgs& g, int x_codes, int w_codes, int bn,
+                           int use_tma_store, int grid, cudaStream_t st) {
+  const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
+  const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
+  if (x_codes == CLQ_CODES_E4M3_SPLIT)
+    return w_codes == CLQ_CODES_E4M3_SPLIT
+               ? launch_gemm_t<OutT, false, false, BN, 2, 2>(m, g, use_tma_store, grid, st)
+               : launch_gemm_t<OutT, false, false, BN, 2, 1>(m, g, use_tma_store, grid, st);
   if (apack)
-    return bpack ? launch_gemm_t<OutT, true, true, BN>(mapA, mapB, mapY, g, use_tma_store, grid,
-                                                       st)
-                 : launch_gemm_t<OutT, true, false, BN>(mapA, mapB, mapY, g, use_tma_store, grid,
-                                                        st);
-  if (bpack)
-    return launch_gemm_t<OutT, false, true, BN>(mapA, mapB, mapY, g, use_tma_store, grid, st);
-  if (bn == 192)
-    return launch_gemm_t<OutT, false, false, 192>(mapA, mapB, mapY, g, use_tma_store, grid, st);
-  return launch_gemm_t<OutT, false, false, BN>(mapA, mapB, mapY, g, use_tma_store, grid, st);
+    return bpack ? launch_gemm_t<OutT, true, true, BN>(m, g, use_tma_store, grid, st)
+                 : launch_gemm_t<OutT, true, false, BN>(m, g, use_tma_store, grid, st);
+  if (bpack) return launch_gemm_t<OutT, false, true, BN>(m, g, use_tma_store, grid, st);
+  if (bn == 192) return launch_gemm_t<OutT, false, false, 192>(m, g, use_tma_store, grid, st);
+  return launch_gemm_t<OutT, false, false, BN>(m, g, use_tma_store, grid, st);
 }
 
 }  // namespace
 
-// TMA map of an INT4 code array (rows x K codes) in either layout: packed
-// boxes of 64 bytes x box_rows (no swizzle, staged for unpacking) or E4M3
-// boxes of 128 bytes x box_rows with the 128-byte swizzle (MMA operand).
+// TMA map of a code array (rows x K codes) in any layout: packed boxes of 64
+// bytes x box_rows (no swizzle, staged for unpacking) or E4M3 boxes of 128
+// bytes x box_rows with the 128-byte swizzle (MMA operand).  For the split
+// layout ([rows][2][K]) the map covers plane `plane` of every row (row stride
+// 2K bytes); for the others `plane` must be 0.
 bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows, int K,
-                      int box_rows) {
+                      int box_rows, int plane) {
   if (codes == CLQ_CODES_INT4_PACKED)
     return encode_tma_2d_u8(map, base, static_cast<uint64_t>(K) / 2, static_cast<uint64_t>(rows),
                             BKP, box_rows);
-  return encode_tma_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, base, static_cast<uint64_t>(K),
-                       static_cast<uint64_t>(rows), BK, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
+  const bool split = codes == CLQ_CODES_E4M3_SPLIT;
+  return encode_tma_2d_strided(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1,
+                               base + (split ? static_cast<size_t>(plane) * K : 0),
+                               static_cast<uint64_t>(K), static_cast<uint64_t>(rows),
+                               static_cast<uint64_t>(K) * (split ? 2 : 1), BK, box_rows,
+                               CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
@@ -196,8 +218,9 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   // walk ceil(tiles / SMs) rounds.  256 wins unless 192 splits N into whole
   // tiles with no more rounds (N = 1152: 6 x 192 instead of 4.5 x 256).  128
   // measured slower everywhere.
+  const bool split = x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT;
   int bn = BN;
-  if (!apack && !bpack) {
+  if (!apack && !bpack && !split) {
     const long mt = (g.M + BM - 1) / BM;
     auto cost = [&](int w) {
       const long rounds = (mt * ((g.N + w - 1) / w) + sms - 1) / sms;
@@ -205,23 +228,27 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
     };
     if (cost(192) < cost(256)) bn = 192;
   }
-  CUtensorMap mapA, mapB, mapY;
-  if (!encode_codes_map(&mapA, Xq, x_codes, g.M, g.K, BM) ||
-      !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn))
+  MapSet m;
+  if (!encode_codes_map(&m.A, Xq, x_codes, g.M, g.K, BM, 0) ||
+      !encode_codes_map(&m.B, W, w_codes, g.N, g.K, bn, 0))
+    return cudaErrorInvalidValue;
+  m.A2 = m.A;  // unused unless split
+  m.B2 = m.B;
+  if (x_codes == CLQ_CODES_E4M3_SPLIT && !encode_codes_map(&m.A2, Xq, x_codes, g.M, g.K, BM, 1))
+    return cudaErrorInvalidValue;
+  if (w_codes == CLQ_CODES_E4M3_SPLIT && !encode_codes_map(&m.B2, W, w_codes, g.N, g.K, bn, 1))
     return cudaErrorInvalidValue;
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
   if (use_tma_store) {
-    if (!encode_tma_out_tile(&mapY, g.Y, g.M, g.N)) return cudaErrorInvalidValue;
+    if (!encode_tma_out_tile(&m.Y, g.Y, g.M, g.N)) return cudaErrorInvalidValue;
   } else {
-    mapY = mapA;  // unused
+    m.Y = m.A;  // unused
   }
   const int tiles = ((g.M + BM - 1) / BM) * ((g.N + bn - 1) / bn);
   const int grid = std::min(tiles, sms);
   if (out_dtype == CLQ_F16)
-    return launch_gemm_dt<__half>(mapA, mapB, mapY, g, apack, bpack, bn, use_tma_store, grid,
-                                  st);
-  return launch_gemm_dt<__nv_bfloat16>(mapA, mapB, mapY, g, apack, bpack, bn, use_tma_store,
-                                       grid, st);
+    return launch_gemm_dt<__half>(m, g, x_codes, w_codes, bn, use_tma_store, grid, st);
+  return launch_gemm_dt<__nv_bfloat16>(m, g, x_codes, w_codes, bn, use_tma_store, grid, st);
 }
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st) {

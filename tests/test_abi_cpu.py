@@ -84,6 +84,32 @@ def test_w4a4_host_validation(lib, args, code):
     assert clq.clq_w4a4_linear(*args, None) == code
 
 
+@pytest.mark.parametrize("args,code", [
+    # (Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b, out_dtype, Y, acc)
+    ((P, 2, P, P, 0, P, None, 4, 4, 64, 32, 0, P, None), 4),     # W4A8, packed W
+    ((P, 0, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 4),     # W8A4
+    ((P, 1, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 4),     # W8A4
+    ((P, 3, P, P, 1, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad x layout
+    ((P, 2, P, P, 2, P, None, 4, 4, 48, 16, 0, P, None), 2),     # K % 32
+    ((P, 2, P, P, 1, P, None, 4, 4, 64, 32, 0, P + 2, None), 3), # misaligned Y
+    ((None, 2, None, None, 2, None, None, 0, 4, 64, 32, 0, None, None), 0),
+])
+def test_linear_host_validation(lib, args, code):
+    assert clq.clq_linear(*args, None) == code
+
+
+def test_prepare_weights_codes_host_validation(lib):
+    # (W, dtype, N, K, ldw, perm, b, clip, w_codes, Wq, s_w, rot, stream)
+    assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 32, None, 3, P, P,
+                                         None, None) == 1
+    assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 32, P + 2, 2, P,
+                                         P, None, None) == 3
+    assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 5, None, 2, P, P,
+                                         None, None) == 2
+    assert clq.clq_prepare_weights_codes(None, 0, 0, 64, 64, None, 32, None, 2,
+                                         None, None, None, None) == 0
+
+
 def test_fused_and_prepare_host_validation(lib):
     ws = clq.clq_fused_linear_workspace_size(256, 1152)
     # 256 x 1152 E4M3 codes, 256 scales, 2 block counters + 1 tile counter
