@@ -46,6 +46,9 @@ def parse():
     p.add_argument("--fused", action="store_true")
     p.add_argument("--sweep", action="store_true",
                    help="time the 100-cell M x (K, N) x b grid, one JSON line per cell")
+    p.add_argument("--bits", action="store_true",
+                   help="time the workload at W4A4, W4A8 and W8A8 (separate "
+                        "kernels), one JSON line per bit setting")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--layer", default=None,
@@ -389,6 +392,114 @@ def run_sweep(args):
         raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
 
 
+BIT_SETTINGS = (("w4a4", 4, 4), ("w4a8", 8, 4), ("w8a8", 8, 8))
+
+
+def run_bits(args):
+    """The workload's layers at the paper's three bit settings (Sec. 4.1),
+    rotate-quant + GEMM as separate kernels on synthetic inputs rotated over
+    sets larger than L2: per layer the rotate-quant and GEMM durations (CUDA
+    events around each kernel, after warm-up), and per setting the whole
+    step (events around the step only).  One JSON line per bit setting."""
+    import torch
+    from paper_2509_24416_gb300 import clq, synth
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    clq.load()
+    cfg = dict(synth.WORKLOADS[args.workload])
+    if args.tokens is not None:
+        cfg["M"] = int(args.tokens)
+    M, b = cfg["M"], cfg["b"]
+    td = {"f16": torch.float16, "bf16": torch.bfloat16}[cfg["dtype"]]
+    stream = torch.cuda.current_stream()
+    data = []
+    for li in range(len(cfg["layers"])):
+        d = synth.layer_inputs(cfg, li)
+        calib = torch.from_numpy(d["calib"]).to(td).to(dev)
+        perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
+        data.append((d, perm))
+    set_bytes = sum(d["X"].numel() * 2 for d, _ in data)
+    nsets = max(2, math.ceil(2 * L2_BYTES / set_bytes) + 1)
+    xsets = [[d["X"].to(dev) for d, _ in data] for _ in range(nsets)]
+    base_tops = None
+    for name, a_bits, w_bits in BIT_SETTINGS:
+        lays = [clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b, bias=d["bias"].to(dev),
+                                               a_bits=a_bits, w_bits=w_bits)
+                for d, perm in data]
+        width = 2 if a_bits == 8 else 1
+        xq = [torch.empty((M, width * d["K"]), dtype=torch.uint8, device=dev) for d, _ in data]
+        sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in data]
+        ys = [torch.empty((M, d["N"]), dtype=td, device=dev) for d, _ in data]
+
+        x_codes = clq.CLQ_CODES_E4M3_SPLIT if a_bits == 8 else clq.CLQ_CODES_E4M3
+        w_codes = clq.CLQ_CODES_E4M3_SPLIT if w_bits == 8 else clq.CLQ_CODES_E4M3
+        sp = stream.cuda_stream
+        dt = clq._dt(xsets[0][0])
+
+        def step(k, ev=None):
+            xs = xsets[k % nsets]
+            for i, lay in enumerate(lays):
+                K, N = data[i][0]["K"], data[i][0]["N"]
+                if ev is not None:
+                    ev[3 * i].record(stream)
+                st = clq.clq_rotate_quant_act(xs[i].data_ptr(), dt, M, K, K,
+                                              lay.perm.data_ptr(), b, x_codes,
+                                              xq[i].data_ptr(), sx[i].data_ptr(), None, sp)
+                if st:
+                    raise clq.ClqError(st, "clq_rotate_quant_act")
+                if ev is not None:
+                    ev[3 * i + 1].record(stream)
+                st = clq.clq_linear(xq[i].data_ptr(), x_codes, sx[i].data_ptr(),
+                                    lay.We.data_ptr(), w_codes, lay.s_w.data_ptr(),
+                                    lay.bias.data_ptr(), M, N, K, b, dt, ys[i].data_ptr(),
+                                    None, sp)
+                if st:
+                    raise clq.ClqError(st, "clq_linear")
+                if ev is not None:
+                    ev[3 * i + 2].record(stream)
+
+        for k in range(max(3, args.warmup)):
+            step(k)
+        torch.cuda.synchronize()
+        a0, z0 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for k in range(args.steps):
+            step(k)
+        z0.record(stream)
+        torch.cuda.synchronize()
+        step_ms = a0.elapsed_time(z0) / args.steps
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3 * len(lays))]
+               for _ in range(args.steps)]
+        for k in range(args.steps):
+            step(k, evs[k])
+        torch.cuda.synchronize()
+        ops = sum(2.0 * M * d["N"] * d["K"] for d, _ in data)
+        per_layer = []
+        for i, (d, _) in enumerate(data):
+            rq = sum(e[3 * i].elapsed_time(e[3 * i + 1]) for e in evs) / args.steps
+            gm = sum(e[3 * i + 1].elapsed_time(e[3 * i + 2]) for e in evs) / args.steps
+            K, N = d["K"], d["N"]
+            rq_bytes = M * (2.0 * K + width * K + 4)
+            per_layer.append({
+                "layer": d["name"], "K": K, "N": N,
+                "rotate_quant_us": round(rq * 1e3, 2),
+                "rotate_quant_GBps": round(rq_bytes / (rq * 1e-3) / 1e9, 1),
+                "gemm_us": round(gm * 1e3, 2),
+                "gemm_TOPS": round(2.0 * M * N * K / (gm * 1e-3) / 1e12, 1)})
+        tops = ops / (step_ms * 1e-3) / 1e12
+        base_tops = tops if base_tops is None else base_tops
+        print(json.dumps({
+            "bits": name, "workload": args.workload, "tokens_per_layer": M, "b": b,
+            "value": round(tops, 1), "unit": "TOPS", "ms_per_step": round(step_ms, 4),
+            "vs_w4a4": round(tops / base_tops, 3), "steps": args.steps,
+            "layers": per_layer}), flush=True)
+        del lays, xq, sx, ys
+        torch.cuda.empty_cache()
+    status = clq.device_status()
+    if status != 0:
+        raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
+
+
 # --------------------------------------------------------------- GPU arm ---
 def main():
     args = parse()
@@ -397,6 +508,9 @@ def main():
         return
     if args.sweep:
         run_sweep(args)
+        return
+    if args.bits:
+        run_bits(args)
         return
     import torch
     import torch.distributed as dist
