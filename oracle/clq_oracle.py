@@ -58,6 +58,14 @@ Readings of the paper that this file fixes (the paper leaves them open):
    reading 5 generalizes to n bits as qmax = 2^(n-1) - 1 (7 or 127): codes in
    [-qmax, qmax], s = r / qmax, code -2^(n-1) unused.  The product of n-bit
    codes is the same exact integer sum, dequantized by the same epilogue.
+10. Asymmetric activations.  Eq. 1 as printed returns
+   Round((Clip(x, l, r) - l) / (r - l) (2^n - 1)) (r - l) / (2^n - 1), which
+   drops the offset l; read as x^ = q D + l with D = (r - l) / (2^n - 1) and
+   q in [0, 2^n - 1] (the usual asymmetric fake quantization, and the only
+   reading under which x^ approximates x).  Dynamic bounds l = min, r = max
+   of the rotated row (Sec. 3.1).  The ratio is taken in the printed order,
+   ((x - l) / (r - l)) (2^n - 1), in fp32, rounded half to even.  A constant
+   row (r = l) has D = 0 and all codes 0, so x^ = l exactly.
 """
 
 import numpy as np
@@ -238,6 +246,62 @@ def quantize_symmetric(V, clip=None, bits=4):
         codes[nz] = np.clip(np.rint(ratio), -qmax, qmax).astype(np.int8)
     scale = np.where(nz, scale, np.float32(0)).astype(np.float32)
     return codes, scale
+
+
+def quantize_asymmetric(V, bits=4):
+    """Per-row asymmetric n-bit quantization of fp32 rows with dynamic bounds
+    (Eq. 1 with l = min, r = max of the row; Sec. 3.1; reading 10).
+
+    Returns (codes int16 [R, K] in [0, 2^n - 1], delta fp32 [R], lo fp32 [R]);
+    the dequantized row is delta * codes + lo.
+    """
+    if bits not in BIT_WIDTHS:
+        raise ValueError("bit width must be 4 or 8")
+    levels = np.float32(2 ** bits - 1)
+    V = np.asarray(V, dtype=np.float32)
+    lo = np.min(V, axis=1).astype(np.float32)
+    hi = np.max(V, axis=1).astype(np.float32)
+    span = (hi - lo).astype(np.float32)
+    codes = np.zeros(V.shape, dtype=np.int16)
+    nz = span > 0
+    if np.any(nz):
+        shifted = (V[nz] - lo[nz][:, None]).astype(np.float32)
+        frac = (shifted / span[nz][:, None]).astype(np.float32)
+        ratio = (frac * levels).astype(np.float32)
+        codes[nz] = np.clip(np.rint(ratio), 0, levels).astype(np.int16)
+    delta = np.where(nz, span / levels, np.float32(0)).astype(np.float32)
+    return codes, delta, lo
+
+
+def dequantize_asymmetric(codes, delta, lo):
+    """x^ = delta * q + lo per row, in fp64 (reading 10)."""
+    return (np.asarray(codes, np.float64) * np.asarray(delta, np.float64)[:, None]
+            + np.asarray(lo, np.float64)[:, None])
+
+
+def rotate_quant_act_asym(X, perm, b, bits=4):
+    """Online activation path with asymmetric dynamic quantization: gather by
+    s, block Hadamard, then Eq. 1 per token (reading 10).
+
+    Returns (codes int16 [M, K] in [0, 2^n - 1], delta fp32 [M], lo fp32 [M],
+    x_rot fp32 [M, K]).
+    """
+    x_rot = rotate(X, perm, b)
+    codes, delta, lo = quantize_asymmetric(x_rot, bits)
+    return codes, delta, lo, x_rot
+
+
+def asym_linear(qx, delta, lo, qw, s_w, b, bias=None):
+    """The product of dequantized asymmetric activations and symmetric
+    weights, by definition: y = X^ W^T / b + bias with X^ = delta q_x + lo
+    and W^ = s_w q_w, all in fp64 (Sec. 3.3's G G^T = b I with the
+    unnormalized H, reading 4)."""
+    xh = dequantize_asymmetric(qx, delta, lo)
+    wh = np.asarray(qw, np.float64) * np.asarray(s_w, np.float64)[:, None]
+    y = xh @ wh.T / float(b)
+    if bias is not None:
+        y = y + np.asarray(bias).astype(np.float64)[None, :]
+    return y
 
 
 def pack_int4(codes):

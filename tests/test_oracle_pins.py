@@ -555,3 +555,103 @@ def test_8bit_planted_grid_mistake_is_caught(monkeypatch, wrong):
     monkeypatch.setattr(orc, "qmax_for_bits", wrong)
     with pytest.raises(AssertionError):
         test_8bit_hand_example()
+
+
+# ------------------------------------- asymmetric activations (Eq. 1) ----
+def test_asym_hand_example():
+    """Eq. 1 with l = min, r = max by hand: the row (-1, 0, 0.5, 2) has
+    r - l = 3, so the codes are 5 (x + 1) rounded half to even at 4 bits and
+    85 (x + 1) at 8 bits; a constant row reconstructs exactly."""
+    V = np.array([[-1, 0, 0.5, 2], [3, 3, 3, 3]], dtype=np.float32)
+    q4, d4, l4 = orc.quantize_asymmetric(V, 4)
+    assert q4.tolist() == [[0, 5, 8, 15], [0, 0, 0, 0]]
+    assert d4.tolist() == [np.float32(0.2), 0.0] and l4.tolist() == [-1.0, 3.0]
+    q8, d8, l8 = orc.quantize_asymmetric(V, 8)
+    assert q8.tolist() == [[0, 85, 128, 255], [0, 0, 0, 0]]
+    assert d8[0] == np.float32(np.float32(3) / np.float32(255))
+    xh = orc.dequantize_asymmetric(q4, d4, l4)
+    assert np.allclose(xh[0], [-1, 0, 0.6, 2], rtol=0, atol=1e-7)
+    assert xh[1].tolist() == [3, 3, 3, 3]
+
+
+def test_asym_range_extremes_and_error_bound():
+    rng = np.random.default_rng(41)
+    X = (rng.standard_normal((24, 192)) * rng.uniform(0.1, 20, (24, 1))
+         + rng.uniform(-5, 5, (24, 1))).astype(np.float16)
+    perm = _perm(192, 2)
+    for bits in (4, 8):
+        q, d, lo, xr = orc.rotate_quant_act_asym(X, perm, 64, bits)
+        top = 2 ** bits - 1
+        assert q.min() >= 0 and q.max() <= top
+        rows = np.arange(24)
+        assert np.all(q[rows, np.argmin(xr, axis=1)] == 0)
+        assert np.all(q[rows, np.argmax(xr, axis=1)] == top)
+        err = np.abs(xr - orc.dequantize_asymmetric(q, d, lo))
+        assert np.all(err <= d[:, None] * (0.5 + 1e-5) + 1e-6 * np.abs(lo)[:, None])
+
+
+def test_asym_linear_bruteforce_and_zero_point_identity():
+    rng = np.random.default_rng(43)
+    M, N, K, b = 3, 4, 32, 16
+    qx = rng.integers(0, 16, (M, K))
+    qw = rng.integers(-7, 8, (N, K))
+    d = rng.uniform(0.01, 0.2, M).astype(np.float32)
+    lo = rng.uniform(-3, 1, M).astype(np.float32)
+    s_w = rng.uniform(0.01, 0.1, N).astype(np.float32)
+    bias = rng.standard_normal(N).astype(np.float32)
+    y = orc.asym_linear(qx, d, lo, qw, s_w, b, bias)
+    for i in range(M):
+        for n in range(N):
+            t = sum((float(d[i]) * int(qx[i, k]) + float(lo[i]))
+                    * (float(s_w[n]) * int(qw[n, k])) for k in range(K))
+            assert abs(y[i, n] - (t / b + float(bias[n]))) <= 1e-12 * max(1.0, abs(t))
+    # the zero-point form a kernel evaluates: s_w / b (D acc + l sum_k q_w) + bias
+    acc = orc.int_gemm(qx, qw)
+    wsum = qw.sum(axis=1)
+    zp = (s_w.astype(np.float64)[None, :] / b
+          * (d.astype(np.float64)[:, None] * acc + lo.astype(np.float64)[:, None] * wsum[None, :])
+          + bias.astype(np.float64)[None, :])
+    assert np.allclose(y, zp, rtol=1e-12, atol=1e-12)
+
+
+def test_asym_beats_symmetric_on_shifted_rows():
+    """Rows with a common offset (post-GELU-like) lose half of the symmetric
+    grid; the asymmetric grid spends all 2^n levels on [min, max]."""
+    rng = np.random.default_rng(47)
+    V = (np.abs(rng.standard_normal((64, 256))) + 0.5).astype(np.float32)
+    qs, ss = orc.quantize_symmetric(V)
+    qa, da, la = orc.quantize_asymmetric(V)
+    e_sym = np.linalg.norm(V - qs * ss[:, None])
+    e_asym = np.linalg.norm(V - orc.dequantize_asymmetric(qa, da, la))
+    assert e_asym < 0.6 * e_sym
+
+
+def _dequant_no_offset(codes, delta, lo):
+    return np.asarray(codes, np.float64) * np.asarray(delta, np.float64)[:, None]
+
+
+def _asym_levels_pow2(V, bits=4):
+    V = np.asarray(V, np.float32)
+    lo, hi = V.min(axis=1), V.max(axis=1)
+    span = hi - lo
+    safe = np.where(span > 0, span, 1)[:, None]
+    q = np.clip(np.rint((V - lo[:, None]) / safe * 2 ** bits), 0, 2 ** bits)
+    return q.astype(np.int16), (span / 2 ** bits).astype(np.float32), lo
+
+
+def _asym_floor(V, bits=4):
+    V = np.asarray(V, np.float32)
+    lo, hi = V.min(axis=1), V.max(axis=1)
+    span = hi - lo
+    top = 2 ** bits - 1
+    q = np.floor((V - lo[:, None]) / np.where(span > 0, span, 1)[:, None] * top)
+    return q.astype(np.int16), (span / top).astype(np.float32), lo
+
+
+@pytest.mark.parametrize("name,fn", [("dequantize_asymmetric", _dequant_no_offset),
+                                     ("quantize_asymmetric", _asym_levels_pow2),
+                                     ("quantize_asymmetric", _asym_floor)])
+def test_asym_planted_mistakes_are_caught(monkeypatch, name, fn):
+    monkeypatch.setattr(orc, name, fn)
+    with pytest.raises(AssertionError):
+        test_asym_hand_example()
