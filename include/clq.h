@@ -243,6 +243,57 @@ clq_status clq_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x,
                       int32_t* acc_dbg, void* stream);
 
 /*
+ * Asymmetric activation quantization (Eq. 1 with dynamic bounds, Sec. 3.1):
+ * after the same rotation as clq_rotate_quant_act, each token row X~[i] is
+ * quantized with l = min_k X~[i][k], r = max_k X~[i][k]:
+ *   delta[i] = (r - l) / (2^n - 1),
+ *   q = rint((X~ - l) / (r - l) * (2^n - 1)) in [0, 2^n - 1], ties to even,
+ * and x^ = delta q + l (Eq. 1 as printed omits the + l; this is the reading
+ * under which x^ approximates x).  A constant row gets delta = 0, q = 0.
+ * The codes are stored CENTERED, c = q - 2^(n-1), so they share the signed
+ * containers of the symmetric path: n = 4 for CLQ_CODES_INT4_PACKED and
+ * CLQ_CODES_E4M3 (c in [-8, 7]), n = 8 for CLQ_CODES_E4M3_SPLIT
+ * (c in [-128, 127]).  delta, lo: device fp32 [M] (lo receives l).  Other
+ * arguments as for clq_rotate_quant_act.
+ */
+clq_status clq_rotate_quant_act_asym(const void* X, clq_dtype dtype, int32_t M,
+                                     int32_t K, int32_t ldx,
+                                     const int32_t* perm, int32_t b,
+                                     clq_codes x_codes, uint8_t* Xq,
+                                     float* delta, float* lo, float* x_rot_dbg,
+                                     void* stream);
+
+/*
+ * wsum[n] = sum_k qw[n][k], the integer code sums of each weight row, for
+ * the zero-point epilogue of clq_linear_asym (exact in fp32: |wsum| <=
+ * 127 * 16384).  W: device codes [N][...] in layout `w_codes`; wsum: device
+ * fp32 [N].  Offline, once per layer.
+ */
+clq_status clq_weight_code_sums(const uint8_t* W, clq_codes w_codes, int32_t N,
+                                int32_t K, float* wsum, void* stream);
+
+/*
+ * The product of asymmetric activations (centered codes from
+ * clq_rotate_quant_act_asym, delta, lo) and symmetric weights, with the
+ * zero-point epilogue that equals X^ W^^T / b + bias:
+ *   Y[i][n] = out_dtype(s_w[n] / b * (delta[i] acc[i][n] + m[i] wsum[n])
+ *                       + bias[n]),
+ *   acc[i][n] = sum_k c[i][k] qw[n][k],  m[i] = lo[i] + 2^(n-1) delta[i]
+ * (m is the value of centered code 0).  Layouts: x_codes CLQ_CODES_E4M3 with
+ * w_codes CLQ_CODES_E4M3 (A4), or x_codes CLQ_CODES_E4M3_SPLIT (A8) with
+ * w_codes CLQ_CODES_E4M3 or CLQ_CODES_E4M3_SPLIT; packed operands return
+ * CLQ_ERR_UNSUPPORTED.  wsum from clq_weight_code_sums.  acc_dbg receives
+ * acc (centered codes).  Other arguments as for clq_linear.
+ */
+clq_status clq_linear_asym(const uint8_t* Xq, clq_codes x_codes,
+                           const float* delta, const float* lo,
+                           const uint8_t* W, clq_codes w_codes,
+                           const float* s_w, const float* wsum,
+                           const void* bias, int32_t M, int32_t N, int32_t K,
+                           int32_t b, clq_dtype out_dtype, void* Y,
+                           int32_t* acc_dbg, void* stream);
+
+/*
  * Bytes of device workspace clq_fused_linear needs for M tokens of K
  * channels (E4M3 activation codes, scales and per-tile readiness counters).
  */

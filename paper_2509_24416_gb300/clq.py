@@ -33,7 +33,9 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_selftest_bounded_wait", "clq_outlier_scores_metric",
            "clq_peak_tcgen05_e4m3",
            "clq_peak_mma_sync", "clq_peak_hbm_read",
-           "clq_prepare_weights_codes", "clq_linear")
+           "clq_prepare_weights_codes", "clq_linear",
+           "clq_rotate_quant_act_asym", "clq_weight_code_sums",
+           "clq_linear_asym")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -66,6 +68,11 @@ _SIGS = {
                                        _P, _P, _P, _P]),
     "clq_linear": (_I, [_P, _I, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P,
                         _P, _P]),
+    "clq_rotate_quant_act_asym": (_I, [_P, _I, _I, _I, _I, _P, _I, _I, _P,
+                                       _P, _P, _P, _P]),
+    "clq_weight_code_sums": (_I, [_P, _I, _I, _I, _P, _P]),
+    "clq_linear_asym": (_I, [_P, _I, _P, _P, _P, _I, _P, _P, _P, _I, _I, _I,
+                             _I, _I, _P, _P, _P]),
 }
 
 
@@ -125,6 +132,24 @@ def clq_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b,
                out_dtype, Y, acc_dbg, stream):
     return load().clq_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N,
                              K, b, out_dtype, Y, acc_dbg, stream)
+
+
+def clq_rotate_quant_act_asym(X, dtype, M, K, ldx, perm, b, x_codes, Xq, delta,
+                              lo, x_rot_dbg, stream):
+    return load().clq_rotate_quant_act_asym(X, dtype, M, K, ldx, perm, b,
+                                            x_codes, Xq, delta, lo, x_rot_dbg,
+                                            stream)
+
+
+def clq_weight_code_sums(W, w_codes, N, K, wsum, stream):
+    return load().clq_weight_code_sums(W, w_codes, N, K, wsum, stream)
+
+
+def clq_linear_asym(Xq, x_codes, delta, lo, W, w_codes, s_w, wsum, bias, M, N,
+                    K, b, out_dtype, Y, acc_dbg, stream):
+    return load().clq_linear_asym(Xq, x_codes, delta, lo, W, w_codes, s_w, wsum,
+                                  bias, M, N, K, b, out_dtype, Y, acc_dbg,
+                                  stream)
 
 
 def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, x_codes, Xq, s_x,
@@ -298,6 +323,42 @@ def rotate_quant_act(X, perm, b, codes=CLQ_CODES_INT4_PACKED, Xq=None, s_x=None,
     return (Xq, s_x, rot) if with_rot else (Xq, s_x)
 
 
+def rotate_quant_act_asym(X, perm, b, codes=CLQ_CODES_E4M3, Xq=None,
+                          delta=None, lo=None, with_rot=False, stream=None):
+    """X [M, K] -> (Xq uint8, delta fp32 [M], lo fp32 [M][, x_rot fp32
+    [M, K]]): asymmetric codes (Eq. 1, dynamic min / max) stored centered,
+    4-bit in CLQ_CODES_E4M3 / CLQ_CODES_INT4_PACKED, 8-bit in
+    CLQ_CODES_E4M3_SPLIT."""
+    _row_major(X, "X")
+    M, K = X.shape
+    dev = X.device
+    if Xq is None:
+        Xq = torch.empty((M, codes_width(codes, K)), dtype=torch.uint8,
+                         device=dev)
+    if delta is None:
+        delta = torch.empty(M, dtype=torch.float32, device=dev)
+    if lo is None:
+        lo = torch.empty(M, dtype=torch.float32, device=dev)
+    rot = (torch.empty((M, K), dtype=torch.float32, device=dev)
+           if with_rot else None)
+    _check(clq_rotate_quant_act_asym(_ptr(X), _dt(X), M, K, X.stride(0),
+                                     _ptr(perm), b, codes, _ptr(Xq),
+                                     _ptr(delta), _ptr(lo), _ptr(rot),
+                                     _stream(stream)),
+           "clq_rotate_quant_act_asym")
+    return (Xq, delta, lo, rot) if with_rot else (Xq, delta, lo)
+
+
+def weight_code_sums(W, K, stream=None):
+    """Integer code sums of each row of a weight code array (any layout) ->
+    fp32 [N]."""
+    N = W.shape[0]
+    wsum = torch.empty(N, dtype=torch.float32, device=W.device)
+    _check(clq_weight_code_sums(_ptr(W), codes_layout(W, K), N, K, _ptr(wsum),
+                                _stream(stream)), "clq_weight_code_sums")
+    return wsum
+
+
 def expand_weights(Wq, stream=None):
     """Packed codes [N, K/2] -> E4M3 execution layout [N, K] (uint8)."""
     N, Kh = Wq.shape
@@ -354,6 +415,25 @@ def linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
                       codes_layout(W, K), _ptr(s_w), _ptr(bias), M, N, K, b,
                       _dt(Y), _ptr(Y), _ptr(acc), _stream(stream)),
            "clq_linear")
+    return (Y, acc) if with_acc else Y
+
+
+def linear_asym(Xq, delta, lo, W, s_w, wsum, b, K, bias=None,
+                out_dtype=torch.float16, Y=None, with_acc=False, stream=None):
+    """Asymmetric activation codes (rotate_quant_act_asym) x weight codes
+    with the zero-point epilogue -> Y [M, N][, acc int32 [M, N]]."""
+    M = Xq.shape[0]
+    N = W.shape[0]
+    if Y is None:
+        Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
+    acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
+           if with_acc else None)
+    if bias is not None and bias.dtype != Y.dtype:
+        raise TypeError("bias must have the output dtype")
+    _check(clq_linear_asym(_ptr(Xq), codes_layout(Xq, K), _ptr(delta), _ptr(lo),
+                           _ptr(W), codes_layout(W, K), _ptr(s_w), _ptr(wsum),
+                           _ptr(bias), M, N, K, b, _dt(Y), _ptr(Y), _ptr(acc),
+                           _stream(stream)), "clq_linear_asym")
     return (Y, acc) if with_acc else Y
 
 

@@ -108,7 +108,8 @@ clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, in
 
 clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ld,
                                const int32_t* perm, int32_t b, const float* clip, int codes,
-                               uint8_t* Q, float* S, float* rot, void* stream) {
+                               uint8_t* Q, float* S, float* rot, void* stream,
+                               float* lo = nullptr) {
   if (!valid_dtype(dtype) || !valid_any_codes(codes) || M < 0) return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
@@ -117,7 +118,8 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   if (M == 0) return CLQ_OK;
   if (X == nullptr || perm == nullptr || Q == nullptr || S == nullptr) return CLQ_ERR_INVALID_ARG;
   if (!aligned(X, 16) || !aligned(Q, 16) || !aligned(perm, 4) || !aligned(S, 4) ||
-      (rot != nullptr && !aligned(rot, 16)) || (clip != nullptr && !aligned(clip, 4)))
+      (rot != nullptr && !aligned(rot, 16)) || (clip != nullptr && !aligned(clip, 4)) ||
+      (lo != nullptr && !aligned(lo, 4)))
     return CLQ_ERR_ALIGN;
   int32_t* status = nullptr;
   st = device_setup(&status);
@@ -132,11 +134,58 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   a.Q = Q;
   a.S = S;
   a.rot = rot;
+  a.lo = lo;
   a.status = status;
   a.logb = log2i(b);
   a.e4m3 = codes == CLQ_CODES_E4M3 ? 1 : codes == CLQ_CODES_E4M3_SPLIT ? 2 : 0;
   return from_cuda(
       clq::launch_rotate_quant(a, dtype, log2i(b), static_cast<cudaStream_t>(stream)));
+}
+
+// The product with its epilogue; lo / wsum non-null select the asymmetric
+// (zero-point) epilogue.
+clq_status linear_common(const uint8_t* Xq, int x_codes, const float* s_x, const float* lo,
+                         const uint8_t* W, int w_codes, const float* s_w, const float* wsum,
+                         const void* bias, int32_t M, int32_t N, int32_t K, int32_t b,
+                         int out_dtype, void* Y, int32_t* acc_dbg, void* stream) {
+  if (!valid_dtype(out_dtype) || !valid_any_codes(x_codes) || !valid_any_codes(w_codes) ||
+      M < 0 || N < 0)
+    return CLQ_ERR_INVALID_ARG;
+  // 8-bit operands: W4A8 (split activations, E4M3 weights) and W8A8 only.
+  if ((x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT) &&
+      !(x_codes == CLQ_CODES_E4M3_SPLIT &&
+        (w_codes == CLQ_CODES_E4M3 || w_codes == CLQ_CODES_E4M3_SPLIT)))
+    return CLQ_ERR_UNSUPPORTED;
+  clq_status st = check_k_b(K, b);
+  if (st != CLQ_OK) return st;
+  if (M == 0 || N == 0) return CLQ_OK;
+  if (Xq == nullptr || s_x == nullptr || W == nullptr || s_w == nullptr || Y == nullptr)
+    return CLQ_ERR_INVALID_ARG;
+  if (!aligned(Xq, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(s_x, 4) ||
+      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)) ||
+      (acc_dbg != nullptr && !aligned(acc_dbg, 4)) || (lo != nullptr && !aligned(lo, 4)) ||
+      (wsum != nullptr && !aligned(wsum, 4)))
+    return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  clq::GemmArgs g{};
+  g.s_x = s_x;
+  g.s_w = s_w;
+  g.bias = bias;
+  g.Y = Y;
+  g.acc_dbg = acc_dbg;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.inv_b = 1.0f / static_cast<float>(b);
+  g.status = status;
+  g.lo = lo;
+  g.wsum = wsum;
+  g.zp_shift = x_codes == CLQ_CODES_E4M3_SPLIT ? 128.0f : 8.0f;
+  return from_cuda(
+      clq::launch_w4a4_gemm(Xq, x_codes, W, w_codes, g, out_dtype,
+                            static_cast<cudaStream_t>(stream)));
 }
 
 }  // namespace
@@ -232,6 +281,15 @@ clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M, int32
                              stream);
 }
 
+clq_status clq_rotate_quant_act_asym(const void* X, clq_dtype dtype, int32_t M, int32_t K,
+                                     int32_t ldx, const int32_t* perm, int32_t b,
+                                     clq_codes x_codes, uint8_t* Xq, float* delta, float* lo,
+                                     float* x_rot_dbg, void* stream) {
+  if (M > 0 && lo == nullptr) return CLQ_ERR_INVALID_ARG;
+  return rotate_quant_common(X, dtype, M, K, ldx, perm, b, nullptr, x_codes, Xq, delta,
+                             x_rot_dbg, stream, lo);
+}
+
 clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K, uint8_t* We,
                               void* stream) {
   if (N < 0 || K < 0) return CLQ_ERR_INVALID_ARG;
@@ -258,40 +316,35 @@ clq_status clq_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x, co
                       clq_codes w_codes, const float* s_w, const void* bias, int32_t M,
                       int32_t N, int32_t K, int32_t b, clq_dtype out_dtype, void* Y,
                       int32_t* acc_dbg, void* stream) {
-  if (!valid_dtype(out_dtype) || !valid_any_codes(x_codes) || !valid_any_codes(w_codes) ||
-      M < 0 || N < 0)
-    return CLQ_ERR_INVALID_ARG;
-  // 8-bit operands: W4A8 (split activations, E4M3 weights) and W8A8 only.
-  if ((x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT) &&
-      !(x_codes == CLQ_CODES_E4M3_SPLIT &&
-        (w_codes == CLQ_CODES_E4M3 || w_codes == CLQ_CODES_E4M3_SPLIT)))
-    return CLQ_ERR_UNSUPPORTED;
-  clq_status st = check_k_b(K, b);
-  if (st != CLQ_OK) return st;
-  if (M == 0 || N == 0) return CLQ_OK;
-  if (Xq == nullptr || s_x == nullptr || W == nullptr || s_w == nullptr || Y == nullptr)
-    return CLQ_ERR_INVALID_ARG;
-  if (!aligned(Xq, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(s_x, 4) ||
-      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)) ||
-      (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
-    return CLQ_ERR_ALIGN;
+  return linear_common(Xq, x_codes, s_x, nullptr, W, w_codes, s_w, nullptr, bias, M, N, K, b,
+                       out_dtype, Y, acc_dbg, stream);
+}
+
+clq_status clq_linear_asym(const uint8_t* Xq, clq_codes x_codes, const float* delta,
+                           const float* lo, const uint8_t* W, clq_codes w_codes,
+                           const float* s_w, const float* wsum, const void* bias, int32_t M,
+                           int32_t N, int32_t K, int32_t b, clq_dtype out_dtype, void* Y,
+                           int32_t* acc_dbg, void* stream) {
+  if (x_codes == CLQ_CODES_INT4_PACKED || w_codes == CLQ_CODES_INT4_PACKED)
+    return valid_any_codes(x_codes) && valid_any_codes(w_codes) ? CLQ_ERR_UNSUPPORTED
+                                                                : CLQ_ERR_INVALID_ARG;
+  if (M > 0 && N > 0 && (lo == nullptr || wsum == nullptr)) return CLQ_ERR_INVALID_ARG;
+  return linear_common(Xq, x_codes, delta, lo, W, w_codes, s_w, wsum, bias, M, N, K, b,
+                       out_dtype, Y, acc_dbg, stream);
+}
+
+clq_status clq_weight_code_sums(const uint8_t* W, clq_codes w_codes, int32_t N, int32_t K,
+                                float* wsum, void* stream) {
+  if (!valid_any_codes(w_codes) || N < 0) return CLQ_ERR_INVALID_ARG;
+  if (K < 32 || K > 16384 || K % 32 != 0) return CLQ_ERR_SHAPE;
+  if (N == 0) return CLQ_OK;
+  if (W == nullptr || wsum == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(W, 16) || !aligned(wsum, 4)) return CLQ_ERR_ALIGN;
   int32_t* status = nullptr;
-  st = device_setup(&status);
+  clq_status st = device_setup(&status);
   if (st != CLQ_OK) return st;
-  clq::GemmArgs g{};
-  g.s_x = s_x;
-  g.s_w = s_w;
-  g.bias = bias;
-  g.Y = Y;
-  g.acc_dbg = acc_dbg;
-  g.M = M;
-  g.N = N;
-  g.K = K;
-  g.inv_b = 1.0f / static_cast<float>(b);
-  g.status = status;
   return from_cuda(
-      clq::launch_w4a4_gemm(Xq, x_codes, W, w_codes, g, out_dtype,
-                            static_cast<cudaStream_t>(stream)));
+      clq::launch_code_sums(W, w_codes, N, K, wsum, static_cast<cudaStream_t>(stream)));
 }
 
 size_t clq_fused_linear_workspace_size(int32_t M, int32_t K) {

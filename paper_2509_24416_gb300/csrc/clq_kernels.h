@@ -16,7 +16,8 @@ struct RotateQuantArgs {
   const int32_t* perm;   // [K]
   const float* clip;     // [M] or null (weights only)
   uint8_t* Q;            // [M][K/2] packed, [M][K] E4M3, or [M][2][K] split planes
-  float* S;              // [M]
+  float* S;              // [M] scales (asymmetric: delta)
+  float* lo;             // [M] row minima (asymmetric codes), or null (symmetric)
   float* rot;            // [M][K] or null
   int32_t rows_per_tile; // filled in by the launcher
   int32_t* status;       // device status word
@@ -43,6 +44,12 @@ struct GemmArgs {
   int32_t M, N, K;
   float inv_b;
   int32_t* status;
+  // Asymmetric activation codes (centered, q - 2^(n-1)): s_x holds each row's
+  // step delta, lo its minimum, wsum[N] the weight-code row sums, zp_shift
+  // 2^(n-1).  lo == null: symmetric codes.
+  const float* lo;
+  const float* wsum;
+  float zp_shift;
 };
 
 // A = activation codes, B = weight codes, each in layout CLQ_CODES_INT4_PACKED
@@ -51,6 +58,10 @@ struct GemmArgs {
 // are built here.
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st);
+
+// wsum[n] = sum_k of the integer codes of row n, any layout (exact in fp32).
+cudaError_t launch_code_sums(const uint8_t* W, int codes, int N, int K, float* wsum,
+                             cudaStream_t st);
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st);
 

@@ -131,11 +131,15 @@ __device__ __forceinline__ void tmem_ld_wait_tie(uint32_t (&r)[32]) {
 // TMA map for Y the block goes through one of the warp's NBUF 64-byte-swizzled
 // staging buffers and one bulk tensor store issued by lane 0; otherwise (N not
 // a multiple of 8) each lane stores its row directly.
-template <typename OutT, int NBUF>
+// ASYM (asymmetric activation codes, centered): s_x[row] is the row's step
+// delta, zm the value of code 0, col_zw holds sum_k q_w[col][k] * s_w / b,
+// and y = acc * delta * s_w / b + zm * col_zw + bias.
+template <typename OutT, int NBUF, bool ASYM = false>
 __device__ __forceinline__ void epilogue_block(const uint32_t (&r)[32], int c, int quarter,
                                                int lane, int m0, int n0, int M, int N,
                                                float sx, const float* col_scale,
-                                               const float* col_bias, uint8_t* staging,
+                                               const float* col_bias, float zm,
+                                               const float* col_zw, uint8_t* staging,
                                                const CUtensorMap* mapY, void* Y,
                                                int32_t* acc_dbg, int& store_count) {
   const int row = m0 + quarter * 32 + lane;
@@ -144,7 +148,14 @@ __device__ __forceinline__ void epilogue_block(const uint32_t (&r)[32], int c, i
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const float4 cs = *reinterpret_cast<const float4*>(col_scale + c + 4 * j);
-    const float4 cb = *reinterpret_cast<const float4*>(col_bias + c + 4 * j);
+    float4 cb = *reinterpret_cast<const float4*>(col_bias + c + 4 * j);
+    if constexpr (ASYM) {
+      const float4 cz = *reinterpret_cast<const float4*>(col_zw + c + 4 * j);
+      const float2 zm2 = make_float2(zm, zm);
+      const float2 b0 = __ffma2_rn(zm2, make_float2(cz.x, cz.y), make_float2(cb.x, cb.y));
+      const float2 b1 = __ffma2_rn(zm2, make_float2(cz.z, cz.w), make_float2(cb.z, cb.w));
+      cb = make_float4(b0.x, b0.y, b1.x, b1.y);
+    }
     const float2 a0 = make_float2(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]));
     const float2 a1 = make_float2(__uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
     const float2 y0 =
@@ -194,10 +205,11 @@ __device__ __forceinline__ void epilogue_block(const uint32_t (&r)[32], int c, i
 // processed, so its latency hides behind the arithmetic and the store (32
 // more registers a thread).  `store_count` counts this warp's stores (it
 // selects the staging buffer).
-template <typename OutT, int NCOL, int NBUF, bool PREFETCH>
+template <typename OutT, int NCOL, int NBUF, bool PREFETCH, bool ASYM = false>
 __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, int col0,
                                               int lane, int m0, int n0, int M, int N, float sx,
                                               const float* col_scale, const float* col_bias,
+                                              float zm, const float* col_zw,
                                               uint8_t* staging, const CUtensorMap* mapY,
                                               void* Y, int32_t* acc_dbg, int& store_count) {
   static_assert(NCOL % EPI_COLS == 0, "column share must be whole 32-column blocks");
@@ -209,8 +221,9 @@ __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, in
       uint32_t r[32];
       tmem_ld32(lane_base + c, r);
       tmem_ld_wait_tie(r);
-      epilogue_block<OutT, NBUF>(r, c, quarter, lane, m0, n0, M, N, sx, col_scale, col_bias,
-                                 staging, mapY, Y, acc_dbg, store_count);
+      epilogue_block<OutT, NBUF, ASYM>(r, c, quarter, lane, m0, n0, M, N, sx, col_scale,
+                                       col_bias, zm, col_zw, staging, mapY, Y, acc_dbg,
+                                       store_count);
     }
     return;
   }
@@ -222,14 +235,16 @@ __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, in
     tmem_ld_wait_tie(ra);
     const bool more1 = c + EPI_COLS < col0 + NCOL && n0 + c + EPI_COLS < N;
     if (more1) tmem_ld32(lane_base + c + EPI_COLS, rb);
-    epilogue_block<OutT, NBUF>(ra, c, quarter, lane, m0, n0, M, N, sx, col_scale, col_bias,
-                               staging, mapY, Y, acc_dbg, store_count);
+    epilogue_block<OutT, NBUF, ASYM>(ra, c, quarter, lane, m0, n0, M, N, sx, col_scale,
+                                     col_bias, zm, col_zw, staging, mapY, Y, acc_dbg,
+                                     store_count);
     if (!more1) break;
     tmem_ld_wait_tie(rb);
     const bool more2 = c + 2 * EPI_COLS < col0 + NCOL && n0 + c + 2 * EPI_COLS < N;
     if (more2) tmem_ld32(lane_base + c + 2 * EPI_COLS, ra);
-    epilogue_block<OutT, NBUF>(rb, c + EPI_COLS, quarter, lane, m0, n0, M, N, sx, col_scale,
-                               col_bias, staging, mapY, Y, acc_dbg, store_count);
+    epilogue_block<OutT, NBUF, ASYM>(rb, c + EPI_COLS, quarter, lane, m0, n0, M, N, sx,
+                                     col_scale, col_bias, zm, col_zw, staging, mapY, Y,
+                                     acc_dbg, store_count);
     if (!more2) break;
   }
 }

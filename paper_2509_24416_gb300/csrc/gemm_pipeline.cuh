@@ -68,7 +68,7 @@ struct Cfg {
   static constexpr int BU = PB * BNT * BK;  // E4M3 B stage (all planes)
   static constexpr int BP = BNT * BKP;   // packed B stage
   static constexpr int STAGE = AU + BU + (APACK ? A_P : 0) + (BPACK ? BP : 0);
-  static constexpr int FIXED = EPI_TOTAL + 4 * BNT * 4;
+  static constexpr int FIXED = EPI_TOTAL + 6 * BNT * 4;
   static constexpr int S0 = (222 * 1024 - FIXED) / STAGE;
   static constexpr int S = S0 > MAX_STAGES ? MAX_STAGES : S0;  // pipeline stages
   static constexpr size_t OFF_UA = 0;                           // E4M3 operands
@@ -76,8 +76,8 @@ struct Cfg {
   static constexpr size_t OFF_PA = OFF_UB + S * BU;             // packed staging
   static constexpr size_t OFF_PB = OFF_PA + (APACK ? S * A_P : 0);
   static constexpr size_t OFF_EPI = OFF_PB + (BPACK ? S * BP : 0);
-  static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;        // [2][2][BNT] floats
-  static constexpr size_t BYTES = OFF_COL + 4 * BNT * sizeof(float);
+  static constexpr size_t OFF_COL = OFF_EPI + EPI_TOTAL;        // [2][3][BNT] floats
+  static constexpr size_t BYTES = OFF_COL + 6 * BNT * sizeof(float);
   static constexpr uint32_t TX = (APACK ? A_P : AU) + (BPACK ? BP : BU);
   // two accumulators of BNT columns, 2 * BNT rounded up to the power of two
   // tcgen05.alloc takes
@@ -161,8 +161,9 @@ __device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, ui
 
 // EPI_PREFETCH: let the epilogue prefetch TMEM (taken only in the 320-thread
 // configuration, where registers allow it).
+// ASYM: asymmetric activation codes (zero-point epilogue, g.lo / g.wsum).
 template <typename OutT, bool APACK, bool BPACK, int BNT = BN, bool EPI_PREFETCH = true,
-          int PA = 1, int PB = 1>
+          int PA = 1, int PB = 1, bool ASYM = false>
 __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
                                          Barriers* bars, uint32_t tmem, const uint32_t* ready) {
   using C = Cfg<APACK, BPACK, BNT, PA, PB>;
@@ -281,8 +282,9 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       const int buf = tc & 1;
       // Column data of this tile into the buffer of its parity; the buffer of
       // the other parity may still be read by slower warps (previous tile).
-      float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL) + buf * 2 * BNT;
+      float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL) + buf * 3 * BNT;
       float* col_bias = col_scale + BNT;
+      float* col_zw = col_scale + 2 * BNT;
       for (int j = et; j < BNT; j += C::EPI_THREADS) {
         const int col = n0 + j;
         float sc = 0.f, bi = 0.f;
@@ -292,6 +294,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
         }
         col_scale[j] = sc;
         col_bias[j] = bi;
+        if (ASYM) col_zw[j] = col < g.N ? g.wsum[col] * sc : 0.f;
       }
       bool ok = mbar_wait_bounded(&bars->acc_full[buf], (tc >> 1) & 1, abort, g.status,
                                   kWaitLimitNs);
@@ -303,9 +306,11 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       // read it from L2, after the tile's MMAs have completed.
       const int row = m0 + quarter * 32 + lane;
       const float sx = row < g.M ? __ldcg(g.s_x + row) : 0.f;
-      epilogue_part<OutT, C::EPI_NCOL, C::EPI_NBUF, EPI_PREFETCH && !C::UNPACK>(
+      // asymmetric codes: the value of code 0 is min + 2^(n-1) delta
+      const float zm = ASYM && row < g.M ? fmaf(g.zp_shift, sx, __ldcg(g.lo + row)) : 0.f;
+      epilogue_part<OutT, C::EPI_NCOL, C::EPI_NBUF, EPI_PREFETCH && !C::UNPACK, ASYM>(
           tmem + buf * BNT, quarter, part * C::EPI_NCOL, lane, m0, n0, g.M, g.N, sx, col_scale,
-          col_bias, staging, maps.Y, g.Y, g.acc_dbg, stores);
+          col_bias, zm, col_zw, staging, maps.Y, g.Y, g.acc_dbg, stores);
       tc_fence_before();
       mbar_arrive(&bars->acc_empty[buf]);
     }

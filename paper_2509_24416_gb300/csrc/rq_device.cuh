@@ -3,7 +3,9 @@
 // to rows of X (column gather by the swap vector `perm`, then the block
 // Sylvester Hadamard H_b) and quantizes each row to symmetric INT4 with a
 // dynamic fp32 scale (Sec. 3.1, Eq. 1 with l = -r), or to symmetric INT8
-// (qmax 127) for the split-plane layout of the W4A8 / W8A8 settings.
+// (qmax 127) for the split-plane layout of the W4A8 / W8A8 settings, or
+// (ASYM) asymmetrically with the row's min and max as bounds (Eq. 1 with
+// dynamic l and r), stored as centered codes q - 2^(n-1).
 //
 // Every thread of the CTA takes part.  The CTA walks tiles of R rows.  Raw
 // rows stream into a ring of STAGES shared-memory buffers (STRIDE bytes
@@ -42,10 +44,21 @@ constexpr int kStride = 32 * 1024;
 constexpr int kStages = 2;
 constexpr int kMaxRegs = 128;            // register cap of the tile-loop kernels
 
-// Shared memory of the tile loop: STAGES raw tiles, 3R row maxima, STAGES
-// barriers and tile indices, abort flag.
+// Shared memory of the tile loop: STAGES raw tiles, 3R row maxima and 3R row
+// minima (asymmetric mode), STAGES barriers and tile indices, abort flag.
 __host__ __device__ inline size_t smem_bytes(int R, int stride, int stages) {
-  return static_cast<size_t>(stages) * stride + 12u * R + 8u + 12u * stages + 16u;
+  return static_cast<size_t>(stages) * stride + 24u * R + 8u + 12u * stages + 16u;
+}
+
+// Order-preserving map of a float to an unsigned key (and back), so that
+// signed maxima can be taken with integer max reductions; key 0 is below
+// every float.
+__device__ __forceinline__ uint32_t order_key(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float order_key_inv(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
 struct NoPublish {
@@ -132,8 +145,9 @@ __device__ __forceinline__ void issue_tile(const RotateQuantArgs& a, uint8_t* ds
 // calls publish(row0, rows) once its own stores of that tile are issued.
 // LOGB = log2(b) when known at compile time, or -1 to read a.logb.  SPLIT:
 // 8-bit codes in the split-plane layout (a.e4m3 == 2), else 4-bit codes.
+// ASYM: asymmetric codes with per-row a.S = delta and a.lo = min.
 template <typename T, int LOGB, bool CLIP, int STRIDE, int STAGES, bool SPLIT = false,
-          typename Publish = NoPublish>
+          bool ASYM = false, typename Publish = NoPublish>
 __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
                                     uint32_t* tile_counter, Publish publish) {
   const int K = a.K;
@@ -147,8 +161,9 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
 
   uint8_t* raw = smem;
   uint32_t* amax = reinterpret_cast<uint32_t*>(smem + STAGES * STRIDE);  // [3][R]
+  uint32_t* amin = amax + 3 * R;  // [3][R] keys of -min (asymmetric mode)
   uint64_t* full = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(amax + 3 * R) + 7) & ~static_cast<uintptr_t>(7));
+      (reinterpret_cast<uintptr_t>(amin + 3 * R) + 7) & ~static_cast<uintptr_t>(7));
   int32_t* tile_of = reinterpret_cast<int32_t*>(full + STAGES);  // tile in each stage
   int32_t* abort = tile_of + STAGES;
 
@@ -177,7 +192,7 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
     *abort = 0;
     fence_mbarrier_init();
   }
-  for (int i = tid; i < 3 * R; i += nthr) amax[i] = 0u;
+  for (int i = tid; i < 6 * R; i += nthr) amax[i] = 0u;
   __syncthreads();
   // Global inputs are read only from here on (the previous kernel on the
   // stream may still be finishing when this grid starts).
@@ -289,17 +304,37 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
           }
         }
       }
-      // |x| maximum of the segment as a tree (short dependency chain)
-      float mk[16];
+      if constexpr (ASYM) {
+        // max and min of the segment as trees, reduced as order keys
+        float mk[16];
 #pragma unroll
-      for (int k = 0; k < 16; ++k) mk[k] = fmaxf(fabsf(v[k].x), fabsf(v[k].y));
+        for (int k = 0; k < 16; ++k) mk[k] = fmaxf(v[k].x, v[k].y);
 #pragma unroll
-      for (int w = 8; w >= 1; w >>= 1)
+        for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll
-        for (int k = 0; k < w; ++k) mk[k] = fmaxf(mk[k], mk[k + w]);
-      const float m = mk[0];
-      {
-        const unsigned mx = __reduce_max_sync(grp, __float_as_uint(m));
+          for (int k = 0; k < w; ++k) mk[k] = fmaxf(mk[k], mk[k + w]);
+        const unsigned kx = __reduce_max_sync(grp, order_key(mk[0]));
+#pragma unroll
+        for (int k = 0; k < 16; ++k) mk[k] = fminf(v[k].x, v[k].y);
+#pragma unroll
+        for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+          for (int k = 0; k < w; ++k) mk[k] = fminf(mk[k], mk[k + w]);
+        const unsigned kn = __reduce_max_sync(grp, order_key(-mk[0]));
+        if (active && lane == leader && r_local < rows) {
+          atomicMax(&amax[par * R + r_local], kx);
+          atomicMax(&amin[par * R + r_local], kn);
+        }
+      } else {
+        // |x| maximum of the segment as a tree (short dependency chain)
+        float mk[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) mk[k] = fmaxf(fabsf(v[k].x), fabsf(v[k].y));
+#pragma unroll
+        for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+          for (int k = 0; k < w; ++k) mk[k] = fmaxf(mk[k], mk[k + w]);
+        const unsigned mx = __reduce_max_sync(grp, __float_as_uint(mk[0]));
         if (active && lane == leader && r_local < rows) atomicMax(&amax[par * R + r_local], mx);
       }
       __syncthreads();  // row maxima complete; raw stage s fully read
@@ -308,15 +343,26 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
       // ---- 3. scale, codes, pack, store --------------------------------------
       if (active && r_local < rows) {
         const int row = row0 + r_local;
-        float am = __uint_as_float(amax[par * R + r_local]);
-        if (CLIP) am = fminf(am, __ldg(a.clip + row));
-        // s = am / qmax: quotient by the reciprocal constant, one residual
-        // correction.
         constexpr float qmax = SPLIT ? 127.0f : 7.0f;
-        constexpr float rqmax = SPLIT ? 1.0f / 127.0f : 1.0f / 7.0f;
-        const float q1 = am * rqmax;
-        const float s_row = fmaf(fmaf(-qmax, q1, am), rqmax, q1);
-        if (seg == 0) a.S[row] = s_row;
+        float am, row_lo = 0.f;
+        if constexpr (ASYM) {
+          // span = max - min; delta = span / (2^n - 1)
+          row_lo = -order_key_inv(amin[par * R + r_local]);
+          am = __fsub_rn(order_key_inv(amax[par * R + r_local]), row_lo);
+        } else {
+          am = __uint_as_float(amax[par * R + r_local]);
+          if (CLIP) am = fminf(am, __ldg(a.clip + row));
+        }
+        // s = am / qmax (symmetric) or am / (2 qmax + 1) (asymmetric):
+        // quotient by the reciprocal constant, one residual correction.
+        constexpr float div = ASYM ? 2.0f * qmax + 1.0f : qmax;
+        constexpr float rdiv = 1.0f / div;
+        const float q1 = am * rdiv;
+        const float s_row = fmaf(fmaf(-div, q1, am), rdiv, q1);
+        if (seg == 0) {
+          a.S[row] = s_row;
+          if (ASYM) a.lo[row] = row_lo;
+        }
         if (a.rot != nullptr) {
           float4* dst = reinterpret_cast<float4*>(a.rot + static_cast<size_t>(row) * K + seg * 32);
 #pragma unroll
@@ -328,7 +374,28 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
         // codes; a subnormal s (a row maximum below about 1e-37) takes exact
         // divisions instead of the reciprocal.
         const float2 magic = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
-        if (s_row > 0.f && s_row < 1.17549435e-38f) {
+        if constexpr (ASYM) {
+          // q = rint((x - min) / span * (2^n - 1)), stored as q - 2^(n-1): the
+          // magic constant is lowered by 2^(n-1) (it stays even, so ties
+          // still go to even q).  A constant row (span 0) gets q = 0.
+          constexpr float half = SPLIT ? 128.0f : 8.0f;
+          const float2 mg = make_float2(12582912.0f - half, 12582912.0f - half);
+          const float2 nlo = make_float2(-row_lo, -row_lo);
+          if (am > 0.f && am < 1.17549435e-38f) {
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              const float2 d = __fadd2_rn(v[k], nlo);
+              v[k] = __fadd2_rn(make_float2(__fmul_rn(__fdiv_rn(d.x, am), div),
+                                            __fmul_rn(__fdiv_rn(d.y, am), div)),
+                                mg);
+            }
+          } else {
+            const float inv = am > 0.f ? div * rcp_approx(am) : 0.f;
+            const float2 inv2 = make_float2(inv, inv);
+#pragma unroll
+            for (int k = 0; k < 16; ++k) v[k] = __ffma2_rn(__fadd2_rn(v[k], nlo), inv2, mg);
+          }
+        } else if (s_row > 0.f && s_row < 1.17549435e-38f) {
 #pragma unroll
           for (int k = 0; k < 16; ++k)
             v[k] = __fadd2_rn(make_float2(__fdiv_rn(v[k].x, s_row), __fdiv_rn(v[k].y, s_row)),
@@ -414,7 +481,10 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
           *reinterpret_cast<uint4*>(qrow + seg * 16) = make_uint4(w[0], w[1], w[2], w[3]);
         }
       }
-      if (tid < R) amax[((i + 2) % 3) * R + tid] = 0u;
+      if (tid < R) {
+        amax[((i + 2) % 3) * R + tid] = 0u;
+        if (ASYM) amin[((i + 2) % 3) * R + tid] = 0u;
+      }
       publish(row0, rows);
     }
   }

@@ -23,7 +23,7 @@ constexpr size_t smem_bytes() {
 
 // PA / PB = 2: the activation / weight codes are 8-bit, as two E4M3 planes
 // (mapA2 / mapB2 the second plane).
-template <typename OutT, bool APACK, bool BPACK, int BNT, int PA, int PB>
+template <typename OutT, bool APACK, bool BPACK, int BNT, int PA, int PB, bool ASYM>
 __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                      const __grid_constant__ CUtensorMap mapB,
@@ -43,7 +43,7 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
   pdl_wait();
   pdl_launch_dependents();
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr, &mapA2, &mapB2};
-  pipeline<OutT, APACK, BPACK, BNT, true, PA, PB>(maps, g, smem, &bars, tmem, nullptr);
+  pipeline<OutT, APACK, BPACK, BNT, true, PA, PB, ASYM>(maps, g, smem, &bars, tmem, nullptr);
   tc_fence_before();
   __syncthreads();
   teardown(tmem, Cfg<APACK, BPACK, BNT, PA, PB>::TMEM);
@@ -63,7 +63,55 @@ __global__ void expand_weights_kernel(const uint4* __restrict__ src, uint4* __re
   }
 }
 
+// Value of an E4M3 byte that holds an integer code (exact): sign, exponent
+// with bias 7, three mantissa bits.
+__device__ __forceinline__ int e4m3_int(uint32_t byte) {
+  const int e = (byte >> 3) & 0xF;
+  const int m = byte & 0x7;
+  const float v = e == 0 ? 0.f : ldexpf(static_cast<float>(8 + m), e - 10);
+  const int i = static_cast<int>(v);
+  return (byte & 0x80u) ? -i : i;
+}
+
+// sum_k q[n][k] of each row of a code array (any layout), one warp a row.
+__global__ void code_sums_kernel(const uint8_t* __restrict__ W, int codes, int N, int K,
+                                 float* __restrict__ wsum) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= N) return;
+  const int width = codes == CLQ_CODES_INT4_PACKED ? K / 2
+                    : codes == CLQ_CODES_E4M3_SPLIT ? 2 * K : K;
+  const uint4* row = reinterpret_cast<const uint4*>(W + static_cast<size_t>(warp) * width);
+  int acc = 0;
+  for (int i = lane; i < width / 16; i += 32) {
+    const uint4 p = __ldg(row + i);
+    const uint32_t w[4] = {p.x, p.y, p.z, p.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t byte = (w[j] >> (8 * k)) & 0xFFu;
+        if (codes == CLQ_CODES_INT4_PACKED) {
+          const int lo = static_cast<int>(byte & 0xFu), hi = static_cast<int>(byte >> 4);
+          acc += (lo >= 8 ? lo - 16 : lo) + (hi >= 8 ? hi - 16 : hi);
+        } else {
+          acc += e4m3_int(byte);
+        }
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) wsum[warp] = static_cast<float>(acc);
+}
+
 }  // namespace
+
+cudaError_t launch_code_sums(const uint8_t* W, int codes, int N, int K, float* wsum,
+                             cudaStream_t st) {
+  const int blocks = (N + 7) / 8;
+  code_sums_kernel<<<blocks, 256, 0, st>>>(W, codes, N, K, wsum);
+  return cudaGetLastError();
+}
 
 bool encode_tma_2d_strided(CUtensorMap* map, CUtensorMapDataType dt, uint32_t esize,
                            const void* base, uint64_t inner, uint64_t rows,
@@ -159,10 +207,11 @@ struct MapSet {
   CUtensorMap A, B, Y, A2, B2;
 };
 
-template <typename OutT, bool APACK, bool BPACK, int BNT, int PA = 1, int PB = 1>
+template <typename OutT, bool APACK, bool BPACK, int BNT, int PA = 1, int PB = 1,
+          bool ASYM = false>
 cudaError_t launch_gemm_t(const MapSet& m, const GemmArgs& g, int use_tma_store, int grid,
                           cudaStream_t st) {
-  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT, PA, PB>;
+  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT, PA, PB, ASYM>;
   constexpr size_t smem = smem_bytes<APACK, BPACK, BNT, PA, PB>();
   constexpr int threads = Cfg<APACK, BPACK, BNT, PA, PB>::THREADS;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, threads, nullptr);
@@ -175,6 +224,14 @@ cudaError_t launch_gemm_dt(const MapSet& m, const GemmArgs& g, int x_codes, int 
                            int use_tma_store, int grid, cudaStream_t st) {
   const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
   const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
+  if (g.lo != nullptr) {  // asymmetric activations: E4M3 / split operands only
+    if (x_codes == CLQ_CODES_E4M3_SPLIT)
+      return w_codes == CLQ_CODES_E4M3_SPLIT
+                 ? launch_gemm_t<OutT, false, false, BN, 2, 2, true>(m, g, use_tma_store, grid, st)
+                 : launch_gemm_t<OutT, false, false, BN, 2, 1, true>(m, g, use_tma_store, grid,
+                                                                     st);
+    return launch_gemm_t<OutT, false, false, BN, 1, 1, true>(m, g, use_tma_store, grid, st);
+  }
   if (x_codes == CLQ_CODES_E4M3_SPLIT)
     return w_codes == CLQ_CODES_E4M3_SPLIT
                ? launch_gemm_t<OutT, false, false, BN, 2, 2>(m, g, use_tma_store, grid, st)
@@ -220,7 +277,7 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   // measured slower everywhere.
   const bool split = x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT;
   int bn = BN;
-  if (!apack && !bpack && !split) {
+  if (!apack && !bpack && !split && g.lo == nullptr) {
     const long mt = (g.M + BM - 1) / BM;
     auto cost = [&](int w) {
       const long rounds = (mt * ((g.N + w - 1) / w) + sms - 1) / sms;

@@ -110,6 +110,34 @@ def test_prepare_weights_codes_host_validation(lib):
                                          None, None, None, None) == 0
 
 
+def test_asym_host_validation(lib):
+    # rotate-quant asym: (X, dtype, M, K, ldx, perm, b, codes, Xq, delta, lo, rot, stream)
+    assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 1, P, P, None, None,
+                                         None) == 1                    # lo missing
+    assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 3, P, P, P, None,
+                                         None) == 1                    # bad layout
+    assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 1, P, P, P + 2, None,
+                                         None) == 3                    # misaligned lo
+    assert clq.clq_rotate_quant_act_asym(None, 0, 0, 64, 64, None, 32, 1, None, None,
+                                         None, None, None) == 0        # empty
+    # code sums: (W, codes, N, K, wsum, stream)
+    assert clq.clq_weight_code_sums(P, 3, 4, 64, P, None) == 1
+    assert clq.clq_weight_code_sums(P, 1, 4, 48, P, None) == 2
+    assert clq.clq_weight_code_sums(P, 1, 4, 64, P + 1, None) == 3
+    assert clq.clq_weight_code_sums(None, 1, 0, 64, None, None) == 0
+    # linear asym: (Xq, xc, delta, lo, W, wc, s_w, wsum, bias, M, N, K, b, dt, Y, acc, st)
+    assert clq.clq_linear_asym(P, 0, P, P, P, 1, P, P, None, 4, 4, 64, 32, 0, P, None,
+                               None) == 4                              # packed A
+    assert clq.clq_linear_asym(P, 1, P, P, P, 2, P, P, None, 4, 4, 64, 32, 0, P, None,
+                               None) == 4                              # W8A4
+    assert clq.clq_linear_asym(P, 1, P, None, P, 1, P, P, None, 4, 4, 64, 32, 0, P, None,
+                               None) == 1                              # lo missing
+    assert clq.clq_linear_asym(P, 1, P, P, P, 1, P, P + 2, None, 4, 4, 64, 32, 0, P, None,
+                               None) == 3                              # misaligned wsum
+    assert clq.clq_linear_asym(P, 5, P, P, P, 1, P, P, None, 4, 4, 64, 32, 0, P, None,
+                               None) == 1                              # bad layout
+
+
 def test_fused_and_prepare_host_validation(lib):
     ws = clq.clq_fused_linear_workspace_size(256, 1152)
     # 256 x 1152 E4M3 codes, 256 scales, 2 block counters + 1 tile counter
