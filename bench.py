@@ -392,15 +392,21 @@ def run_sweep(args):
         raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
 
 
-BIT_SETTINGS = (("w4a4", 4, 4), ("w4a8", 8, 4), ("w8a8", 8, 8))
+BIT_SETTINGS = (("w4a4", 4, 4, False), ("w4a8", 8, 4, False), ("w8a8", 8, 8, False),
+                ("w4a4_asym", 4, 4, True), ("w4a8_asym", 8, 4, True),
+                ("w8a8_asym", 8, 8, True))
+ERR_ROWS = 512  # token rows per layer for the output-error figure
 
 
 def run_bits(args):
     """The workload's layers at the paper's three bit settings (Sec. 4.1),
-    rotate-quant + GEMM as separate kernels on synthetic inputs rotated over
-    sets larger than L2: per layer the rotate-quant and GEMM durations (CUDA
-    events around each kernel, after warm-up), and per setting the whole
-    step (events around the step only).  One JSON line per bit setting."""
+    with symmetric and with asymmetric (Eq. 1, zero-point epilogue)
+    activation codes, rotate-quant + GEMM as separate kernels on synthetic
+    inputs rotated over sets larger than L2: per layer the rotate-quant and
+    GEMM durations (CUDA events around each kernel, after warm-up), per
+    setting the whole step (events around the step only), and the output's
+    relative Frobenius error against the fp64 product X W^T + bias on the
+    first ERR_ROWS tokens of each layer.  One JSON line per setting."""
     import torch
     from paper_2509_24416_gb300 import clq, synth
     dev = torch.device("cuda", 0)
@@ -422,13 +428,19 @@ def run_bits(args):
     nsets = max(2, math.ceil(2 * L2_BYTES / set_bytes) + 1)
     xsets = [[d["X"].to(dev) for d, _ in data] for _ in range(nsets)]
     base_tops = None
-    for name, a_bits, w_bits in BIT_SETTINGS:
+    refs = []
+    for d, _ in data:
+        x64 = d["X32"][:ERR_ROWS].astype("float64")
+        refs.append(x64 @ d["W32"].astype("float64").T + d["bias32"].astype("float64")[None, :])
+    for name, a_bits, w_bits, asym in BIT_SETTINGS:
         lays = [clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b, bias=d["bias"].to(dev),
                                                a_bits=a_bits, w_bits=w_bits)
                 for d, perm in data]
+        wsums = [clq.weight_code_sums(lay.We, d["K"]) for lay, (d, _) in zip(lays, data)]
         width = 2 if a_bits == 8 else 1
         xq = [torch.empty((M, width * d["K"]), dtype=torch.uint8, device=dev) for d, _ in data]
         sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in data]
+        los = [torch.empty(M, dtype=torch.float32, device=dev) for _ in data]
         ys = [torch.empty((M, d["N"]), dtype=td, device=dev) for d, _ in data]
 
         x_codes = clq.CLQ_CODES_E4M3_SPLIT if a_bits == 8 else clq.CLQ_CODES_E4M3
@@ -442,19 +454,32 @@ def run_bits(args):
                 K, N = data[i][0]["K"], data[i][0]["N"]
                 if ev is not None:
                     ev[3 * i].record(stream)
-                st = clq.clq_rotate_quant_act(xs[i].data_ptr(), dt, M, K, K,
-                                              lay.perm.data_ptr(), b, x_codes,
-                                              xq[i].data_ptr(), sx[i].data_ptr(), None, sp)
+                if asym:
+                    st = clq.clq_rotate_quant_act_asym(xs[i].data_ptr(), dt, M, K, K,
+                                                       lay.perm.data_ptr(), b, x_codes,
+                                                       xq[i].data_ptr(), sx[i].data_ptr(),
+                                                       los[i].data_ptr(), None, sp)
+                else:
+                    st = clq.clq_rotate_quant_act(xs[i].data_ptr(), dt, M, K, K,
+                                                  lay.perm.data_ptr(), b, x_codes,
+                                                  xq[i].data_ptr(), sx[i].data_ptr(), None, sp)
                 if st:
-                    raise clq.ClqError(st, "clq_rotate_quant_act")
+                    raise clq.ClqError(st, "rotate-quant")
                 if ev is not None:
                     ev[3 * i + 1].record(stream)
-                st = clq.clq_linear(xq[i].data_ptr(), x_codes, sx[i].data_ptr(),
-                                    lay.We.data_ptr(), w_codes, lay.s_w.data_ptr(),
-                                    lay.bias.data_ptr(), M, N, K, b, dt, ys[i].data_ptr(),
-                                    None, sp)
+                if asym:
+                    st = clq.clq_linear_asym(xq[i].data_ptr(), x_codes, sx[i].data_ptr(),
+                                             los[i].data_ptr(), lay.We.data_ptr(), w_codes,
+                                             lay.s_w.data_ptr(), wsums[i].data_ptr(),
+                                             lay.bias.data_ptr(), M, N, K, b, dt,
+                                             ys[i].data_ptr(), None, sp)
+                else:
+                    st = clq.clq_linear(xq[i].data_ptr(), x_codes, sx[i].data_ptr(),
+                                        lay.We.data_ptr(), w_codes, lay.s_w.data_ptr(),
+                                        lay.bias.data_ptr(), M, N, K, b, dt, ys[i].data_ptr(),
+                                        None, sp)
                 if st:
-                    raise clq.ClqError(st, "clq_linear")
+                    raise clq.ClqError(st, "product")
                 if ev is not None:
                     ev[3 * i + 2].record(stream)
 
@@ -479,9 +504,11 @@ def run_bits(args):
             rq = sum(e[3 * i].elapsed_time(e[3 * i + 1]) for e in evs) / args.steps
             gm = sum(e[3 * i + 1].elapsed_time(e[3 * i + 2]) for e in evs) / args.steps
             K, N = d["K"], d["N"]
-            rq_bytes = M * (2.0 * K + width * K + 4)
+            rq_bytes = M * (2.0 * K + width * K + (8 if asym else 4))
+            y = ys[i][:ERR_ROWS].double().cpu().numpy()
+            err = float(((y - refs[i]) ** 2).sum() ** 0.5 / (refs[i] ** 2).sum() ** 0.5)
             per_layer.append({
-                "layer": d["name"], "K": K, "N": N,
+                "layer": d["name"], "K": K, "N": N, "rel_err": round(err, 5),
                 "rotate_quant_us": round(rq * 1e3, 2),
                 "rotate_quant_GBps": round(rq_bytes / (rq * 1e-3) / 1e9, 1),
                 "gemm_us": round(gm * 1e3, 2),
@@ -492,8 +519,9 @@ def run_bits(args):
             "bits": name, "workload": args.workload, "tokens_per_layer": M, "b": b,
             "value": round(tops, 1), "unit": "TOPS", "ms_per_step": round(step_ms, 4),
             "vs_w4a4": round(tops / base_tops, 3), "steps": args.steps,
+            "activations": "asymmetric" if asym else "symmetric",
             "layers": per_layer}), flush=True)
-        del lays, xq, sx, ys
+        del lays, xq, sx, ys, los, wsums
         torch.cuda.empty_cache()
     status = clq.device_status()
     if status != 0:
