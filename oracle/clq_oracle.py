@@ -66,6 +66,16 @@ Readings of the paper that this file fixes (the paper leaves them open):
    of the rotated row (Sec. 3.1).  The ratio is taken in the printed order,
    ((x - l) / (r - l)) (2^n - 1), in fp32, rounded half to even.  A constant
    row (r = l) has D = 0 and all codes 0, so x^ = l exactly.
+11. Per-layer clip search (Sec. 3.4, Eq. 3, with the target layer taken to
+   be the layer itself, since Eq. 2's cross-layer target needs a model).
+   Under the symmetric weight grid (reading 5) the bounds satisfy l = -r, so
+   the grid over (l, r) collapses to one percentile p in [beta, gamma]
+   (beta = 0, gamma = 0.01, Sec. 4.1), the same p for every output channel
+   of a matrix (Sec. 4.1), with r_n(p) the floor(p K)-th largest |W~[n, :]|
+   (0-based, so p = 0 is the row's absolute maximum: no clipping).  The
+   objective is ||Y - Y^||_F^2 on calibration tokens, Y = X W^T + bias in
+   fp64 and Y^ the quantized layer (rotate-quant of X, weights prepared with
+   clip r(p)) in fp64.  The smallest error wins; ties go to the smaller p.
 """
 
 import numpy as np
@@ -409,3 +419,55 @@ def linear_fp64(X, W, bias=None):
     if bias is not None:
         y = y + np.asarray(bias).astype(np.float64)[None, :]
     return y
+
+
+# --------------------------------------------- Sec. 3.4 Eq. 3 clip search --
+CLIP_BETA, CLIP_GAMMA = 0.0, 0.01  # Sec. 4.1: beta = 0, gamma = 0.01
+
+
+def clip_grid(G, beta=CLIP_BETA, gamma=CLIP_GAMMA):
+    """G evenly spaced percentiles from beta to gamma (fp64)."""
+    if G < 1:
+        raise ValueError("grid needs at least one point")
+    if G == 1:
+        return np.array([beta], dtype=np.float64)
+    return beta + (gamma - beta) * np.arange(G, dtype=np.float64) / (G - 1)
+
+
+def clip_rank(p, K):
+    """0-based rank, from the top, of the clip bound at percentile p
+    (reading 11): floor(p K)."""
+    return int(np.floor(float(p) * K))
+
+
+def clip_table(w_rot, J):
+    """The J largest |w_rot[n, k]| of every row, largest first (fp32)."""
+    A = np.abs(np.asarray(w_rot, dtype=np.float32))
+    return -np.sort(-A, axis=1)[:, :J]
+
+
+def clip_search(X, W, perm, b, bias=None, grid=None):
+    """Eq. 3 per layer (reading 11): for every percentile p of the grid, clip
+    each output channel of W~ at r_n(p), quantize, run the W4A4 layer on the
+    calibration tokens X and measure ||Y - Y^||_F^2 against the fp64 layer.
+
+    Returns (errors fp64 [G], best grid index, clip fp32 [N] of the best p,
+    grid fp64 [G]).
+    """
+    grid = clip_grid(11) if grid is None else np.asarray(grid, np.float64)
+    W = np.asarray(W)
+    K = W.shape[1]
+    w_rot = rotate(W, perm, b)
+    J = max(clip_rank(p, K) for p in grid) + 1
+    table = clip_table(w_rot, J)
+    Y = linear_fp64(X, W, bias)
+    errors = np.empty(len(grid), dtype=np.float64)
+    clips = []
+    for g, p in enumerate(grid):
+        clip = table[:, clip_rank(p, K)].astype(np.float32)
+        Wq, s_w, _, _ = prepare_weights(W, perm, b, clip)
+        Yh = fused_linear(X, perm, b, Wq, s_w, bias)
+        errors[g] = float(np.sum((Y - Yh) ** 2))
+        clips.append(clip)
+    best = int(np.argmin(errors))  # first minimum: ties to the smaller p
+    return errors, best, clips[best], grid

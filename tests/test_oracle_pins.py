@@ -655,3 +655,88 @@ def test_asym_planted_mistakes_are_caught(monkeypatch, name, fn):
     monkeypatch.setattr(orc, name, fn)
     with pytest.raises(AssertionError):
         test_asym_hand_example()
+
+
+# ------------------------------------------- per-layer clip search (Eq. 3) --
+def _outlier_case(sign=1.0):
+    """Every weight row carries one large weight on a column whose input is
+    always 0: it adds nothing to Y, but unclipped it sets the row's scale
+    and zeroes the other codes, so any clip below it must win."""
+    rng = np.random.default_rng(61)
+    K, N, M = 64, 8, 32
+    W = rng.standard_normal((N, K)).astype(np.float32)
+    X = rng.standard_normal((M, K)).astype(np.float32)
+    W[:, 5] = 40.0 * sign
+    X[:, 5] = 0.0
+    return X, W, np.arange(K, dtype=np.int32)
+
+
+def test_clip_grid_and_rank():
+    g = orc.clip_grid(11)
+    assert g[0] == 0.0 and g[-1] == 0.01 and len(g) == 11
+    assert [orc.clip_rank(p, 1152) for p in g] == [0, 1, 2, 3, 4, 5, 6, 8, 9, 10, 11]
+    assert orc.clip_grid(1).tolist() == [0.0]
+
+
+def test_clip_table_bruteforce():
+    rng = np.random.default_rng(62)
+    w = rng.standard_normal((5, 40)).astype(np.float32)
+    t = orc.clip_table(w, 7)
+    for n in range(5):
+        assert t[n].tolist() == sorted((abs(float(v)) for v in w[n]), reverse=True)[:7]
+
+
+def test_clip_search_finds_the_harmless_outlier():
+    for sign in (1.0, -1.0):
+        X, W, perm = _outlier_case(sign)
+        e, best, clip, grid = orc.clip_search(X, W, perm, 1, grid=orc.clip_grid(5, 0, 0.05))
+        assert orc.clip_rank(grid[best], 64) >= 1
+        assert e[0] > 10 * e[best]
+        assert np.all(clip < 39.0)
+
+
+def test_clip_p0_is_unclipped():
+    rng = np.random.default_rng(63)
+    W = rng.standard_normal((6, 128)).astype(np.float16)
+    perm = _perm(128, 4)
+    w_rot = orc.rotate(W, perm, 32)
+    clip = orc.clip_table(w_rot, 1)[:, 0]
+    a = orc.prepare_weights(W, perm, 32)
+    c = orc.prepare_weights(W, perm, 32, clip)
+    assert np.array_equal(a[0], c[0]) and np.array_equal(a[1], c[1])
+
+
+def test_clip_search_scale_invariance_and_direct_error():
+    rng = np.random.default_rng(64)
+    K, N, M, b = 128, 12, 24, 32
+    X = rng.standard_normal((M, K)).astype(np.float32)
+    W = (rng.standard_normal((N, K)) * rng.uniform(0.5, 3, (N, 1))).astype(np.float32)
+    bias = rng.standard_normal(N).astype(np.float32)
+    perm = _perm(K, 5)
+    grid = orc.clip_grid(4, 0, 0.03)
+    e1, b1, c1, _ = orc.clip_search(X, W, perm, b, bias, grid)
+    e2, b2, c2, _ = orc.clip_search(X, 2 * W, perm, b, 2 * bias, grid)
+    assert b1 == b2 and np.array_equal(2 * c1, c2)
+    assert np.allclose(e2, 4 * e1, rtol=1e-12, atol=0)
+    # the best point's error through dequantized operands
+    _, s_w, _, qw = orc.prepare_weights(W, perm, b, c1)
+    _, s_x, _, qx = orc.rotate_quant_act(X, perm, b)
+    yh = ((qx * s_x[:, None].astype(np.float64)) @ (qw * s_w[:, None].astype(np.float64)).T
+          / b + bias[None, :])
+    y = X.astype(np.float64) @ W.astype(np.float64).T + bias[None, :]
+    assert np.isclose(np.sum((y - yh) ** 2), e1[b1], rtol=1e-10)
+
+
+def _table_ascending(w_rot, J):
+    return np.sort(np.abs(np.asarray(w_rot, np.float32)), axis=1)[:, :J]
+
+
+def _table_signed(w_rot, J):
+    return -np.sort(-np.asarray(w_rot, np.float32), axis=1)[:, :J]
+
+
+@pytest.mark.parametrize("fn", [_table_ascending, _table_signed])
+def test_clip_planted_mistakes_are_caught(monkeypatch, fn):
+    monkeypatch.setattr(orc, "clip_table", fn)
+    with pytest.raises(AssertionError):
+        test_clip_search_finds_the_harmless_outlier()
