@@ -49,6 +49,9 @@ def parse():
     p.add_argument("--bits", action="store_true",
                    help="time the workload at W4A4, W4A8 and W8A8 (separate "
                         "kernels), one JSON line per bit setting")
+    p.add_argument("--clip", action="store_true",
+                   help="run the per-layer clip search on each layer of the "
+                        "workload (offline cost and chosen percentile)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--layer", default=None,
@@ -528,6 +531,51 @@ def run_bits(args):
         raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
 
 
+def run_clip(args):
+    """The per-layer clip search (Sec. 3.4, Eq. 3 with the layer as its own
+    target) on every layer of the workload: calibration tokens = the first
+    --tokens rows (default 1024) of the layer's synthetic input, Yref the
+    fp32 product X W^T + bias (torch), the default 11-point grid over
+    [0, 0.01].  Reports the wall time of the call (it synchronizes), the
+    chosen percentile and the error against the unclipped point.  One JSON
+    line per layer."""
+    import torch
+    from paper_2509_24416_gb300 import clq, synth
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    clq.load()
+    cfg = dict(synth.WORKLOADS[args.workload])
+    M = int(args.tokens) if args.tokens is not None else 1024
+    cfg["M"] = M
+    for li in range(len(cfg["layers"])):
+        d = synth.layer_inputs(cfg, li)
+        calib = torch.from_numpy(d["calib"]).to(d["X"].dtype).to(dev)
+        perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
+        X, W, bias = d["X"].to(dev), d["W"].to(dev), d["bias"].to(dev)
+        yref = torch.addmm(bias.float(), X.float(), W.float().t())
+        clq.clip_search(W, perm, d["b"], X, yref, bias)  # warm-up
+        times = []
+        for _ in range(max(1, args.steps)):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            clip, errors, best = clq.clip_search(W, perm, d["b"], X, yref, bias)
+            times.append(time.perf_counter() - t0)
+        ms = 1e3 * sorted(times)[len(times) // 2]
+        G = len(clq.CLIP_GRID)
+        ops = G * 2.0 * M * d["N"] * d["K"]
+        print(json.dumps({
+            "layer": d["name"], "K": d["K"], "N": d["N"], "calib_tokens": M,
+            "grid_points": G, "ms": round(ms, 3),
+            "inner_products_TOPS": round(ops / (ms * 1e-3) / 1e12, 2),
+            "best_p": clq.CLIP_GRID[best],
+            "err_unclipped": float(errors[0]), "err_best": float(errors[best]),
+            "err_ratio": round(float(errors[best] / errors[0]), 4),
+            "errors": [float(e) for e in errors]}), flush=True)
+    status = clq.device_status()
+    if status != 0:
+        raise RuntimeError("device status %s" % clq.STATUS.get(status, status))
+
+
 # --------------------------------------------------------------- GPU arm ---
 def main():
     args = parse()
@@ -539,6 +587,9 @@ def main():
         return
     if args.bits:
         run_bits(args)
+        return
+    if args.clip:
+        run_clip(args)
         return
     import torch
     import torch.distributed as dist

@@ -21,7 +21,8 @@
  *    launched; on an error nothing is launched and no output is touched.
  *  - Tensor pointers are DEVICE pointers owned by the caller unless the name
  *    starts with host_.  The library allocates, frees and synchronizes
- *    nothing in these calls (clq_get_device_status synchronizes by design).
+ *    nothing in these calls (clq_get_device_status and the offline
+ *    clq_clip_search synchronize by design).
  *  - Launches are asynchronous on `stream` (a cudaStream_t passed as void*;
  *    NULL is the legacy default stream).
  *  - Row-major layouts; `ld*` arguments are row strides in ELEMENTS.
@@ -292,6 +293,39 @@ clq_status clq_linear_asym(const uint8_t* Xq, clq_codes x_codes,
                            const void* bias, int32_t M, int32_t N, int32_t K,
                            int32_t b, clq_dtype out_dtype, void* Y,
                            int32_t* acc_dbg, void* stream);
+
+/*
+ * Per-layer clip search (Sec. 3.4, Eq. 3, with the layer as its own target
+ * layer; Eq. 2's cross-layer target needs a model).  With the symmetric
+ * weight grid, l = -r, so the search runs over one percentile p per matrix
+ * (the same for every output channel, Sec. 4.1), from host_grid[0 .. G)
+ * (values in [0, 1); the paper's range is [beta, gamma] = [0, 0.01]): the
+ * clip bound of output channel n is r_n(p) = the floor(p K)-th largest
+ * |W~[n][k]| (0-based; p = 0 is the row's absolute maximum, no clipping),
+ * W~ = W_p H as in clq_prepare_weights.  For every p the layer runs on the
+ * calibration tokens Xcal with the library's own kernels (rotate-quant of
+ * Xcal, weights prepared with clip r(p), W4A4 GEMM with bias, output in
+ * `dtype`), and host_errors[g] receives sum (Y^ - Yref)^2 over the M x N
+ * outputs (fp64, summed in a fixed order).  *host_best receives the index of
+ * the smallest error (ties to the smaller index) and clip_out (device fp32
+ * [N]) its clip bounds, ready for clq_prepare_weights.
+ * W: device [N][ldw], Xcal: device [M][ldx], both of `dtype`; perm: device
+ * int32 [K]; Yref: device fp32 [M][N], the layer's full-precision output
+ * (X W^T + bias) computed by the caller; bias: device [N] of `dtype` or
+ * NULL.  workspace: device, 256-byte aligned, at least
+ * clq_clip_search_workspace_size(M, N, K, host_grid, G) bytes.  Offline: the
+ * call SYNCHRONIZES `stream` to read the errors back.
+ */
+size_t clq_clip_search_workspace_size(int32_t M, int32_t N, int32_t K,
+                                      const float* host_grid, int32_t G);
+clq_status clq_clip_search(const void* W, clq_dtype dtype, int32_t N, int32_t K,
+                           int32_t ldw, const int32_t* perm, int32_t b,
+                           const void* Xcal, int32_t M, int32_t ldx,
+                           const float* Yref, const void* bias,
+                           const float* host_grid, int32_t G, float* clip_out,
+                           double* host_errors, int32_t* host_best,
+                           void* workspace, size_t workspace_bytes,
+                           void* stream);
 
 /*
  * Bytes of device workspace clq_fused_linear needs for M tokens of K

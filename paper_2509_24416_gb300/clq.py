@@ -35,7 +35,8 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_peak_mma_sync", "clq_peak_hbm_read",
            "clq_prepare_weights_codes", "clq_linear",
            "clq_rotate_quant_act_asym", "clq_weight_code_sums",
-           "clq_linear_asym")
+           "clq_linear_asym", "clq_clip_search_workspace_size",
+           "clq_clip_search")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -73,6 +74,9 @@ _SIGS = {
     "clq_weight_code_sums": (_I, [_P, _I, _I, _I, _P, _P]),
     "clq_linear_asym": (_I, [_P, _I, _P, _P, _P, _I, _P, _P, _P, _I, _I, _I,
                              _I, _I, _P, _P, _P]),
+    "clq_clip_search_workspace_size": (_Z, [_I, _I, _I, _P, _I]),
+    "clq_clip_search": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I, _I, _P, _P,
+                             _P, _I, _P, _P, _P, _P, _Z, _P]),
 }
 
 
@@ -150,6 +154,19 @@ def clq_linear_asym(Xq, x_codes, delta, lo, W, w_codes, s_w, wsum, bias, M, N,
     return load().clq_linear_asym(Xq, x_codes, delta, lo, W, w_codes, s_w, wsum,
                                   bias, M, N, K, b, out_dtype, Y, acc_dbg,
                                   stream)
+
+
+def clq_clip_search_workspace_size(M, N, K, host_grid, G):
+    return load().clq_clip_search_workspace_size(M, N, K, host_grid, G)
+
+
+def clq_clip_search(W, dtype, N, K, ldw, perm, b, Xcal, M, ldx, Yref, bias,
+                    host_grid, G, clip_out, host_errors, host_best, workspace,
+                    workspace_bytes, stream):
+    return load().clq_clip_search(W, dtype, N, K, ldw, perm, b, Xcal, M, ldx,
+                                  Yref, bias, host_grid, G, clip_out,
+                                  host_errors, host_best, workspace,
+                                  workspace_bytes, stream)
 
 
 def clq_rotate_quant_act(X, dtype, M, K, ldx, perm, b, x_codes, Xq, s_x,
@@ -435,6 +452,36 @@ def linear_asym(Xq, delta, lo, W, s_w, wsum, b, K, bias=None,
                            _ptr(bias), M, N, K, b, _dt(Y), _ptr(Y), _ptr(acc),
                            _stream(stream)), "clq_linear_asym")
     return (Y, acc) if with_acc else Y
+
+
+CLIP_GRID = tuple(0.001 * i for i in range(11))  # [beta, gamma] = [0, 0.01]
+
+
+def clip_search(W, perm, b, Xcal, Yref, bias=None, grid=CLIP_GRID, stream=None):
+    """Per-layer clip search (Sec. 3.4, Eq. 3): W [N, K], Xcal [M, K] (same
+    dtype, on the GPU), Yref fp32 [M, N] the full-precision layer output.
+    Returns (clip fp32 [N] of the best percentile, errors fp64 [G] (host),
+    best index).  Synchronizes the stream."""
+    _row_major(W, "W")
+    _row_major(Xcal, "Xcal")
+    N, K = W.shape
+    M = Xcal.shape[0]
+    g32 = torch.tensor(grid, dtype=torch.float32)
+    G = g32.numel()
+    nbytes = clq_clip_search_workspace_size(M, N, K, _ptr(g32), G)
+    if nbytes == 0:
+        raise ValueError("invalid clip search shape or grid")
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=W.device)
+    clip = torch.empty(N, dtype=torch.float32, device=W.device)
+    errors = torch.empty(G, dtype=torch.float64)
+    best = torch.zeros(1, dtype=torch.int32)
+    Yref = Yref.to(torch.float32).contiguous()
+    _check(clq_clip_search(_ptr(W), _dt(W), N, K, W.stride(0),
+                           _ptr(perm), b, _ptr(Xcal), M, Xcal.stride(0),
+                           _ptr(Yref), _ptr(bias), _ptr(g32), G, _ptr(clip),
+                           _ptr(errors), _ptr(best), _ptr(ws), nbytes,
+                           _stream(stream)), "clq_clip_search")
+    return clip, errors, int(best.item())
 
 
 def fused_workspace(M, K, device):

@@ -188,6 +188,43 @@ clq_status linear_common(const uint8_t* Xq, int x_codes, const float* s_x, const
                             static_cast<cudaStream_t>(stream)));
 }
 
+// Workspace of clq_clip_search, 256-byte aligned pieces.
+struct ClipWorkspace {
+  size_t w_rot, wq, s_w, table, clip, xq, s_x, yh, partial, errors, bytes;
+};
+constexpr int kClipPartials = 256;
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+int clip_table_width(int K, const float* grid, int G) {
+  int J = 1;
+  for (int g = 0; g < G; ++g)
+    J = std::max(J, static_cast<int>(std::floor(static_cast<double>(grid[g]) * K)) + 1);
+  return J;
+}
+
+ClipWorkspace clip_workspace_layout(int M, int N, int K, int J, int G) {
+  ClipWorkspace w{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align256(off + bytes);
+    return at;
+  };
+  w.w_rot = take(static_cast<size_t>(N) * K * 4);
+  w.wq = take(static_cast<size_t>(N) * K);
+  w.s_w = take(static_cast<size_t>(N) * 4);
+  w.table = take(static_cast<size_t>(N) * J * 4);
+  w.clip = take(static_cast<size_t>(N) * 4);
+  w.xq = take(static_cast<size_t>(M) * K);
+  w.s_x = take(static_cast<size_t>(M) * 4);
+  w.yh = take(static_cast<size_t>(M) * N * 2);
+  w.partial = take(static_cast<size_t>(G) * kClipPartials * 8);
+  w.errors = take(static_cast<size_t>(G) * 8);
+  w.bytes = off;
+  return w;
+}
+
 }  // namespace
 
 extern "C" {
@@ -437,6 +474,116 @@ clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void
   st = from_cuda(clq::launch_peak_hbm_read(buf, bytes, status, static_cast<cudaStream_t>(stream)));
   *ops = static_cast<int64_t>(bytes);
   return st;
+}
+
+}  // extern "C"
+
+extern "C" {
+
+size_t clq_clip_search_workspace_size(int32_t M, int32_t N, int32_t K, const float* host_grid,
+                                      int32_t G) {
+  if (M < 1 || N < 1 || K < 32 || K > 16384 || K % 32 != 0 || G < 1 || host_grid == nullptr)
+    return 0;
+  for (int g = 0; g < G; ++g)
+    if (!(host_grid[g] >= 0.f && host_grid[g] < 1.f)) return 0;
+  return clip_workspace_layout(M, N, K, clip_table_width(K, host_grid, G), G).bytes;
+}
+
+clq_status clq_clip_search(const void* W, clq_dtype dtype, int32_t N, int32_t K, int32_t ldw,
+                           const int32_t* perm, int32_t b, const void* Xcal, int32_t M,
+                           int32_t ldx, const float* Yref, const void* bias,
+                           const float* host_grid, int32_t G, float* clip_out,
+                           double* host_errors, int32_t* host_best, void* workspace,
+                           size_t workspace_bytes, void* stream) {
+  if (!valid_dtype(dtype) || N < 1 || M < 1 || G < 1) return CLQ_ERR_INVALID_ARG;
+  clq_status st = check_k_b(K, b);
+  if (st != CLQ_OK) return st;
+  if (ldw < K || ldx < K) return CLQ_ERR_SHAPE;
+  if (ldw % 8 != 0 || ldx % 8 != 0) return CLQ_ERR_ALIGN;
+  if (W == nullptr || perm == nullptr || Xcal == nullptr || Yref == nullptr ||
+      host_grid == nullptr || clip_out == nullptr || host_errors == nullptr ||
+      host_best == nullptr || workspace == nullptr)
+    return CLQ_ERR_INVALID_ARG;
+  for (int g = 0; g < G; ++g)
+    if (!(host_grid[g] >= 0.f && host_grid[g] < 1.f)) return CLQ_ERR_INVALID_ARG;
+  const int J = clip_table_width(K, host_grid, G);
+  const ClipWorkspace ws = clip_workspace_layout(M, N, K, J, G);
+  if (workspace_bytes < ws.bytes) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(W, 16) || !aligned(Xcal, 16) || !aligned(perm, 4) || !aligned(Yref, 4) ||
+      !aligned(clip_out, 4) || (bias != nullptr && !aligned(bias, 2)) ||
+      !aligned(workspace, 256))
+    return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* base = static_cast<uint8_t*>(workspace);
+  float* w_rot = reinterpret_cast<float*>(base + ws.w_rot);
+  uint8_t* wq = base + ws.wq;
+  float* s_w = reinterpret_cast<float*>(base + ws.s_w);
+  float* table = reinterpret_cast<float*>(base + ws.table);
+  float* clip = reinterpret_cast<float*>(base + ws.clip);
+  uint8_t* xq = base + ws.xq;
+  float* s_x = reinterpret_cast<float*>(base + ws.s_x);
+  void* yh = base + ws.yh;
+  double* partial = reinterpret_cast<double*>(base + ws.partial);
+  double* errors = reinterpret_cast<double*>(base + ws.errors);
+
+  auto rq = [&](const void* X, int rows, int ld, const float* c, uint8_t* Q, float* S,
+                float* rot) {
+    clq::RotateQuantArgs a{};
+    a.X = X;
+    a.M = rows;
+    a.K = K;
+    a.ld = ld;
+    a.perm = perm;
+    a.clip = c;
+    a.Q = Q;
+    a.S = S;
+    a.rot = rot;
+    a.status = status;
+    a.logb = log2i(b);
+    a.e4m3 = 1;
+    return clq::launch_rotate_quant(a, dtype, log2i(b), s);
+  };
+  // W~ (unclipped) and its table of largest magnitudes; the calibration
+  // activations' codes, which every grid point reuses.
+  cudaError_t e = rq(W, N, ldw, nullptr, wq, s_w, w_rot);
+  if (e == cudaSuccess) e = clq::launch_clip_table(w_rot, N, K, J, table, s);
+  if (e == cudaSuccess) e = rq(Xcal, M, ldx, nullptr, xq, s_x, nullptr);
+  clq::GemmArgs g{};
+  g.s_x = s_x;
+  g.s_w = s_w;
+  g.bias = bias;
+  g.Y = yh;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.inv_b = 1.0f / static_cast<float>(b);
+  g.status = status;
+  for (int gi = 0; gi < G && e == cudaSuccess; ++gi) {
+    const int j = static_cast<int>(std::floor(static_cast<double>(host_grid[gi]) * K));
+    e = clq::launch_clip_gather(table, N, J, j, clip, s);
+    if (e == cudaSuccess) e = rq(W, N, ldw, clip, wq, s_w, nullptr);
+    if (e == cudaSuccess)
+      e = clq::launch_w4a4_gemm(xq, CLQ_CODES_E4M3, wq, CLQ_CODES_E4M3, g, dtype, s);
+    if (e == cudaSuccess)
+      e = clq::launch_sq_err_partial(yh, dtype, Yref, static_cast<size_t>(M) * N,
+                                     partial + static_cast<size_t>(gi) * kClipPartials,
+                                     kClipPartials, s);
+  }
+  if (e == cudaSuccess) e = clq::launch_sum_partials(partial, G, kClipPartials, errors, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(host_errors, errors, static_cast<size_t>(G) * sizeof(double),
+                        cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return CLQ_ERR_CUDA;
+  int best = 0;
+  for (int gi = 1; gi < G; ++gi)
+    if (host_errors[gi] < host_errors[best]) best = gi;  // ties: the smaller p
+  *host_best = best;
+  const int jb = static_cast<int>(std::floor(static_cast<double>(host_grid[best]) * K));
+  return from_cuda(clq::launch_clip_gather(table, N, J, jb, clip_out, s));
 }
 
 }  // extern "C"

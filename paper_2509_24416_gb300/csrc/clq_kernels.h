@@ -59,6 +59,19 @@ struct GemmArgs {
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st);
 
+// Clip search (clip_search.cu): table[n][j] = j-th largest |w_rot[n][:]|
+// (j < J); clip[n] = table[n][j]; partial[b] = block b's share of
+// sum (yh - yref)^2 in fp64 over n elements (P blocks); out[g] = the fixed-order
+// sum of partial[g][0 .. P).
+cudaError_t launch_clip_table(const float* w_rot, int N, int K, int J, float* table,
+                              cudaStream_t st);
+cudaError_t launch_clip_gather(const float* table, int N, int J, int j, float* clip,
+                               cudaStream_t st);
+cudaError_t launch_sq_err_partial(const void* yh, int dtype, const float* yref, size_t n,
+                                  double* partial, int P, cudaStream_t st);
+cudaError_t launch_sum_partials(const double* partial, int G, int P, double* out,
+                                cudaStream_t st);
+
 // wsum[n] = sum_k of the integer codes of row n, any layout (exact in fp32).
 cudaError_t launch_code_sums(const uint8_t* W, int codes, int N, int K, float* wsum,
                              cudaStream_t st);

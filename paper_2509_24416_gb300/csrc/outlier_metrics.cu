@@ -15,31 +15,13 @@
 // it with a bitonic network where an order statistic is needed.
 #include "clq_device.cuh"
 #include "clq_kernels.h"
+#include "sort_util.cuh"
 
 namespace clq {
 
 namespace {
 
 constexpr int kThreads = 256;
-
-__device__ __forceinline__ void bitonic_sort_ascending(float* v, int n) {
-  for (int k = 2; k <= n; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const int ixj = i ^ j;
-        if (ixj > i) {
-          const bool up = (i & k) == 0;
-          const float a = v[i], b = v[ixj];
-          if ((a > b) == up) {
-            v[i] = b;
-            v[ixj] = a;
-          }
-        }
-      }
-      __syncthreads();
-    }
-  }
-}
 
 // Block-wide max of x (every thread contributes); the result in every thread.
 __device__ __forceinline__ float block_max(float x, float* red) {

@@ -138,6 +138,32 @@ def test_asym_host_validation(lib):
                                None) == 1                              # bad layout
 
 
+def test_clip_search_host_validation(lib):
+    import ctypes
+    grid = (ctypes.c_float * 3)(0.0, 0.005, 0.01)
+    bad = (ctypes.c_float * 2)(0.0, 1.5)
+    g = ctypes.addressof(grid)
+    assert clq.clq_clip_search_workspace_size(256, 128, 1152, g, 3) > 0
+    assert clq.clq_clip_search_workspace_size(256, 128, 1152, ctypes.addressof(bad), 2) == 0
+    assert clq.clq_clip_search_workspace_size(256, 128, 48, g, 3) == 0
+    assert clq.clq_clip_search_workspace_size(0, 128, 1152, g, 3) == 0
+    errs = (ctypes.c_double * 3)()
+    best = ctypes.c_int32(0)
+    e, bp = ctypes.addressof(errs), ctypes.addressof(best)
+    # (W, dtype, N, K, ldw, perm, b, X, M, ldx, Yref, bias, grid, G, clip,
+    #  errors, best, ws, ws_bytes, stream)
+    assert clq.clq_clip_search(P, 0, 8, 64, 64, P, 32, P, 8, 64, P, None, g, 3, P, e, bp,
+                               P, 16, None) == 1                       # workspace small
+    assert clq.clq_clip_search(P, 0, 8, 64, 64, P, 3, P, 8, 64, P, None, g, 3, P, e, bp,
+                               P, 1 << 30, None) == 2                  # b
+    assert clq.clq_clip_search(P, 0, 8, 64, 64, P, 32, P, 8, 64, P, None,
+                               ctypes.addressof(bad), 2, P, e, bp, P, 1 << 30, None) == 1
+    assert clq.clq_clip_search(P, 0, 8, 64, 64, P, 32, P, 8, 64, P, None, g, 3, P, e, bp,
+                               P + 16, 1 << 30, None) == 3              # ws alignment
+    assert clq.clq_clip_search(P, 0, 0, 64, 64, P, 32, P, 8, 64, P, None, g, 3, P, e, bp,
+                               P, 1 << 30, None) == 1                  # N = 0
+
+
 def test_fused_and_prepare_host_validation(lib):
     ws = clq.clq_fused_linear_workspace_size(256, 1152)
     # 256 x 1152 E4M3 codes, 256 scales, 2 block counters + 1 tile counter
