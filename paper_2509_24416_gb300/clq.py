@@ -249,6 +249,17 @@ def _check(st, where):
         raise ClqError(st, where)
 
 
+def _buffer(t, shape, dtype, device, name):
+    """A caller-provided output buffer, checked against what the call will
+    write (the C ABI takes plain pointers and cannot check sizes)."""
+    if tuple(t.shape) != tuple(shape) or t.dtype != dtype or not t.is_contiguous():
+        raise ValueError("%s must be a contiguous %s tensor of shape %s, got %s %s"
+                         % (name, dtype, tuple(shape), t.dtype, tuple(t.shape)))
+    if t.device != torch.device(device):
+        raise ValueError("%s must be on %s" % (name, device))
+    return t
+
+
 def _row_major(t, name):
     if t.dim() != 2 or t.stride(1) != 1:
         raise ValueError("%s must be a 2-D tensor with unit column stride"
@@ -329,8 +340,12 @@ def rotate_quant_act(X, perm, b, codes=CLQ_CODES_INT4_PACKED, Xq=None, s_x=None,
     if Xq is None:
         Xq = torch.empty((M, codes_width(codes, K)), dtype=torch.uint8,
                          device=dev)
+    else:
+        _buffer(Xq, (M, codes_width(codes, K)), torch.uint8, dev, "Xq")
     if s_x is None:
         s_x = torch.empty(M, dtype=torch.float32, device=dev)
+    else:
+        _buffer(s_x, (M,), torch.float32, dev, "s_x")
     rot = (torch.empty((M, K), dtype=torch.float32, device=dev)
            if with_rot else None)
     _check(clq_rotate_quant_act(_ptr(X), _dt(X), M, K, X.stride(0),
@@ -352,10 +367,16 @@ def rotate_quant_act_asym(X, perm, b, codes=CLQ_CODES_E4M3, Xq=None,
     if Xq is None:
         Xq = torch.empty((M, codes_width(codes, K)), dtype=torch.uint8,
                          device=dev)
+    else:
+        _buffer(Xq, (M, codes_width(codes, K)), torch.uint8, dev, "Xq")
     if delta is None:
         delta = torch.empty(M, dtype=torch.float32, device=dev)
+    else:
+        _buffer(delta, (M,), torch.float32, dev, "delta")
     if lo is None:
         lo = torch.empty(M, dtype=torch.float32, device=dev)
+    else:
+        _buffer(lo, (M,), torch.float32, dev, "lo")
     rot = (torch.empty((M, K), dtype=torch.float32, device=dev)
            if with_rot else None)
     _check(clq_rotate_quant_act_asym(_ptr(X), _dt(X), M, K, X.stride(0),
@@ -405,6 +426,8 @@ def w4a4_linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
     N = W.shape[0]
     if Y is None:
         Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
+    else:
+        _buffer(Y, (M, N), Y.dtype, Xq.device, "Y")
     acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
            if with_acc else None)
     if bias is not None and bias.dtype != Y.dtype:
@@ -424,6 +447,8 @@ def linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
     N = W.shape[0]
     if Y is None:
         Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
+    else:
+        _buffer(Y, (M, N), Y.dtype, Xq.device, "Y")
     acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
            if with_acc else None)
     if bias is not None and bias.dtype != Y.dtype:
@@ -443,6 +468,8 @@ def linear_asym(Xq, delta, lo, W, s_w, wsum, b, K, bias=None,
     N = W.shape[0]
     if Y is None:
         Y = torch.empty((M, N), dtype=out_dtype, device=Xq.device)
+    else:
+        _buffer(Y, (M, N), Y.dtype, Xq.device, "Y")
     acc = (torch.empty((M, N), dtype=torch.int32, device=Xq.device)
            if with_acc else None)
     if bias is not None and bias.dtype != Y.dtype:
@@ -499,6 +526,8 @@ def fused_linear(X, perm, b, W, s_w, bias=None, Y=None, workspace=None,
     N = W.shape[0]
     if Y is None:
         Y = torch.empty((M, N), dtype=X.dtype, device=X.device)
+    else:
+        _buffer(Y, (M, N), X.dtype, X.device, "Y")
     if workspace is None:
         workspace = fused_workspace(M, K, X.device)
     _check(clq_fused_linear(_ptr(X), _dt(X), M, K, X.stride(0), _ptr(perm), b,
@@ -608,8 +637,9 @@ class HostPipeline:
         dev = torch.device(device)
         self.xd = [torch.empty((M, K), dtype=dtype, device=dev) for (_, M, K, _) in layers]
         self.yd = [torch.empty((M, N), dtype=dtype, device=dev) for (_, M, _, N) in layers]
-        self.xq = [torch.empty((M, K), dtype=torch.uint8, device=dev)
-                   for (_, M, K, _) in layers]
+        self.xq = [torch.empty((M, K * (2 if lay.a_bits == 8 else 1)), dtype=torch.uint8,
+                               device=dev)
+                   for (lay, M, K, _) in layers]
         self.sx = [torch.empty(M, dtype=torch.float32, device=dev) for (_, M, _, _) in layers]
         self.ws = [fused_workspace(M, K, dev) if fused else None for (_, M, K, _) in layers]
         self.s_in = torch.cuda.Stream(device=dev)

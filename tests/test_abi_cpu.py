@@ -233,3 +233,25 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(clq, "LIB_PATH", str(tmp_path / "nope.so"))
     with pytest.raises(RuntimeError, match="not built"):
         clq.load()
+
+
+def test_binding_rejects_mis_sized_output_buffers():
+    """The C ABI cannot check buffer sizes; the binding checks what it is
+    handed against what the call will write, before any launch."""
+    import torch
+    X = torch.zeros((4, 64), dtype=torch.float16)
+    perm = torch.arange(64, dtype=torch.int32)
+    small = torch.empty((4, 64), dtype=torch.uint8)      # split layout needs [4, 128]
+    with pytest.raises(ValueError):
+        clq.rotate_quant_act(X, perm, 32, clq.CLQ_CODES_E4M3_SPLIT, Xq=small)
+    with pytest.raises(ValueError):
+        clq.rotate_quant_act(X, perm, 32, clq.CLQ_CODES_E4M3,
+                             s_x=torch.empty(3, dtype=torch.float32))
+    with pytest.raises(ValueError):
+        clq.rotate_quant_act_asym(X, perm, 32, clq.CLQ_CODES_E4M3,
+                                  lo=torch.empty(4, dtype=torch.float64))
+    Xq = torch.empty((4, 64), dtype=torch.uint8)
+    W = torch.empty((8, 64), dtype=torch.uint8)
+    s = torch.empty(8, dtype=torch.float32)
+    with pytest.raises(ValueError):
+        clq.linear(Xq, s[:4], W, s, 32, 64, Y=torch.empty((4, 7), dtype=torch.float16))

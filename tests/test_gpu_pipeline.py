@@ -12,14 +12,15 @@ pytestmark = pytest.mark.gpu
 DEV = torch.device("cuda:0")
 
 
-def _layers(seed, shapes, b=64):
+def _layers(seed, shapes, b=64, bits=(4, 4)):
     g = torch.Generator().manual_seed(seed)
     out = []
     for (M, K, N) in shapes:
         W = (torch.randn(N, K, generator=g) * 0.02).half().to(DEV)
         bias = (torch.randn(N, generator=g) * 0.01).half().to(DEV)
         perm = torch.randperm(K, generator=g).to(torch.int32).to(DEV)
-        out.append((clq.PreparedLinear.from_weight(W, perm, b, bias=bias), M, K, N))
+        out.append((clq.PreparedLinear.from_weight(W, perm, b, bias=bias, a_bits=bits[0],
+                                                   w_bits=bits[1]), M, K, N))
     return out
 
 
@@ -43,3 +44,23 @@ def test_host_pipeline_matches_direct_calls(fused):
         for (lay, M, K, N), x, y in zip(layers, xh, yh):
             ref = lay(x.to(DEV), fused=fused).cpu()
             assert torch.equal(y.view(torch.int16), ref.view(torch.int16))
+
+
+@pytest.mark.parametrize("bits", [(8, 4), (8, 8)])
+def test_host_pipeline_8bit_layers(bits):
+    """8-bit activation codes need twice the code buffer; the pipeline sizes
+    it from each layer's bit setting."""
+    shapes = [(200, 1152, 384), (96, 4608, 512)]
+    layers = _layers(5, shapes, bits=bits)
+    g = torch.Generator().manual_seed(6)
+    xh = [(torch.randn(M, K, generator=g) * 3).half().pin_memory() for (_, M, K, _) in layers]
+    yh = [torch.empty((M, N), dtype=torch.float16).pin_memory() for (_, M, _, N) in layers]
+    pipe = clq.HostPipeline(layers, torch.float16, DEV)
+    pipe.run(xh, yh)
+    pipe.run(xh, yh)
+    pipe.join()
+    torch.cuda.synchronize()
+    assert clq.device_status() == 0
+    for (lay, M, K, N), x, y in zip(layers, xh, yh):
+        ref = lay(x.to(DEV)).cpu()
+        assert torch.equal(y.view(torch.int16), ref.view(torch.int16))
