@@ -1,16 +1,22 @@
 /*
  * clq.h - C ABI of libclq, the GB300 (sm_103a) inference path of CLQ's
- * W4A4 orthogonal-based-smoothing (OBS) linear layer, arxiv 2509.24416.
+ * W4A4 orthogonal-based-smoothing (OBS) linear layer, arxiv 2509.24416, with
+ * the paper's other bit settings (W4A8, W8A8), asymmetric activation codes
+ * (Eq. 1), the alternative outlier metrics (Sec. 4.4) and the per-layer clip
+ * search (Eq. 3).
  *
  * The layer computes Y = X W^T + bias with both operands quantized to 4 bits
- * after the OBS transform G = S H (Sec. 3.3): S is a column swap stored as
- * an index vector `perm` (position k holds the original column perm[k]) and
+ * (or 8, see clq_linear) after the OBS transform G = S H (Sec. 3.3): S is a
+ * column swap stored as an index vector `perm` (position k holds the
+ * original column perm[k]) and
  * H = diag(H_b, ..., H_b) with H_b the Sylvester Hadamard matrix of order b,
  * H_b[i][j] = (-1)^popcount(i & j).  G is absorbed into W offline; the
  * activations are rotated online with a fast Walsh-Hadamard transform and
  * quantized per token with dynamic bounds (Sec. 3.1).  Quantization is the
  * symmetric reading of Eq. 1: r = max|row| (optionally clipped), s = r / 7
- * in fp32, q = clamp(rint(v / s), -7, 7), ties to even, code -8 unused.
+ * in fp32, q = clamp(rint(v / s), -7, 7), ties to even, code -8 unused
+ * (qmax 127 for 8-bit codes; Eq. 1 itself, with dynamic min and max, for
+ * clq_rotate_quant_act_asym).
  * H is unnormalized (H_b H_b^T = b I), so the epilogue divides by b once:
  *     Y[i][n] = acc[i][n] * s_x[i] * s_w[n] / b + bias[n],
  *     acc[i][n] = sum_k qx[i][k] * qw[n][k]  (exact integer).

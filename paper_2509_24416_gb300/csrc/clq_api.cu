@@ -577,7 +577,12 @@ clq_status clq_clip_search(const void* W, clq_dtype dtype, int32_t N, int32_t K,
     e = cudaMemcpyAsync(host_errors, errors, static_cast<size_t>(G) * sizeof(double),
                         cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-  if (e != cudaSuccess) return CLQ_ERR_CUDA;
+  if (e != cudaSuccess) {
+    // Nothing launched before the failure may still use the workspace when
+    // the caller regains control.
+    cudaStreamSynchronize(s);
+    return CLQ_ERR_CUDA;
+  }
   int best = 0;
   for (int gi = 1; gi < G; ++gi)
     if (host_errors[gi] < host_errors[best]) best = gi;  // ties: the smaller p
