@@ -584,6 +584,32 @@ class PreparedLinear:
         Wq, s_w = prepare_weights(W.contiguous(), perm, b, clip, codes=codes)
         return cls(Wq, s_w, perm, b, bias, a_bits=a_bits)
 
+    @classmethod
+    def calibrate(cls, W, calib, b, bias=None, metric="absmax", clip_grid=None,
+                  a_bits=4, w_bits=4, stream=None):
+        """The offline steps in the paper's order (Sec. 3.3, Sec. 3.4), all on
+        the GPU: outlier scores of the calibration batch calib [B, T, K]
+        under `metric` (Sec. 4.4 names the alternatives), the swap vector,
+        then, when `clip_grid` is given (e.g. CLIP_GRID) and the weights are
+        4-bit, the per-layer clip search (Eq. 3) on the B * T calibration
+        tokens against their fp32 product, and finally the prepared layer.
+        Returns (layer, info) with info = dict(scores, perm, clip, errors,
+        best)."""
+        K = W.shape[1]
+        scores = outlier_scores(calib, metric=metric, stream=stream)
+        perm = build_permutation(scores).to(W.device)
+        clip = errors = best = None
+        if clip_grid is not None and w_bits == 4:
+            Xcal = calib.reshape(-1, K).contiguous()
+            Yref = Xcal.float() @ W.float().t()
+            if bias is not None:
+                Yref = Yref + bias.float()[None, :]
+            clip, errors, best = clip_search(W.contiguous(), perm, b, Xcal, Yref, bias,
+                                             grid=clip_grid, stream=stream)
+        layer = cls.from_weight(W, perm, b, bias=bias, clip=clip, a_bits=a_bits,
+                                w_bits=w_bits)
+        return layer, dict(scores=scores, perm=perm, clip=clip, errors=errors, best=best)
+
     def state_dict(self):
         d = dict(Wq=self.Wq, s_w=self.s_w, perm=self.perm,
                  b=torch.tensor(self.b), a_bits=torch.tensor(self.a_bits))

@@ -90,3 +90,32 @@ def test_clip_search_grid_of_one_is_unclipped():
     perm = rng.permutation(K).astype(np.int32)
     e, best, _, _ = _run(W, X, None, perm, 64, "f16", [0.0])
     assert best == 0 and e.shape == (1,)
+
+
+@pytest.mark.parametrize("metric", ["absmax", "topk_mean"])
+def test_prepared_linear_calibrate_runs_the_offline_steps(metric):
+    """PreparedLinear.calibrate = outlier scores under the metric, swap
+    vector, clip search on the calibration tokens, prepared weights, each
+    step equal to its own call."""
+    cfg = dict(synth.WORKLOADS["pixart_1024"], M=256)
+    d = synth.layer_inputs(cfg, 0)
+    b = d["b"]
+    calib = torch.from_numpy(d["calib"]).to(TD[d["dtype"]]).to(DEV)
+    W, bias = d["W"].to(DEV), d["bias"].to(DEV)
+    layer, info = clq.PreparedLinear.calibrate(W, calib, b, bias, metric=metric,
+                                               clip_grid=clq.CLIP_GRID)
+    scores = clq.outlier_scores(calib, metric=metric)
+    perm = clq.build_permutation(scores)
+    assert torch.equal(info["perm"].cpu(), perm)
+    K = W.shape[1]
+    Xcal = calib.reshape(-1, K).contiguous()
+    Yref = Xcal.float() @ W.float().t() + bias.float()[None, :]
+    clip, errors, best = clq.clip_search(W, perm.to(DEV), b, Xcal, Yref, bias)
+    assert best == info["best"] and torch.equal(clip, info["clip"])
+    ref = clq.PreparedLinear.from_weight(W, perm.to(DEV), b, bias=bias, clip=clip)
+    X = d["X"].to(DEV)
+    torch.cuda.synchronize()
+    assert torch.equal(layer(X), ref(X))
+    # the oracle's permutation from the same calibration batch
+    o = oracle.build_permutation(oracle.outlier_scores(d["calib"], metric))
+    assert np.array_equal(perm.numpy(), o)
