@@ -476,10 +476,6 @@ clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void
   return st;
 }
 
-}  // extern "C"
-
-extern "C" {
-
 size_t clq_clip_search_workspace_size(int32_t M, int32_t N, int32_t K, const float* host_grid,
                                       int32_t G) {
   if (M < 1 || N < 1 || K < 32 || K > 16384 || K % 32 != 0 || G < 1 || host_grid == nullptr)
