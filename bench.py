@@ -88,6 +88,29 @@ KERNEL_SOURCES = {
 }
 
 
+SM_INTAKE_BYTES_PER_CLK = 64.0  # measured per-SM L2 -> SM ceiling (profiles/peaks_gb300.md)
+
+
+def gemm_intake_bound(M, shapes, sms, sm_mhz):
+    """The GEMM's structural ceiling on this part: every SM takes at most
+    SM_INTAKE_BYTES_PER_CLK from L2 per clock, and each 128 x w output tile
+    brings (128 + w) K operand bytes in and sends 2 x 128 w output bytes out
+    through the same port.  Tiles are those the launcher picks (w = 192 when
+    it covers N in whole tiles with no more rounds, else 256), dealt round-
+    robin, so a layer takes ceil(tiles / SMs) tile-times.  Returns TFLOP/s
+    over the layer set."""
+    rate = SM_INTAKE_BYTES_PER_CLK * sm_mhz * 1e6
+    mt = (M + 127) // 128
+    t_total, ops = 0.0, 0.0
+    for (K, N) in shapes:
+        def rounds(w):
+            return (mt * ((N + w - 1) // w) + sms - 1) // sms
+        w = 192 if rounds(192) * (16 + 192 / 8) < rounds(256) * (16 + 256 / 8) else 256
+        t_total += rounds(w) * ((128 + w) * K + 2 * 128 * w) / rate
+        ops += 2.0 * M * N * K
+    return ops / t_total / 1e12
+
+
 def job_throughput(local_ms, ops_per_step, steps, world, device=None):
     """Whole-job rate of a weak-scaling run: every rank processes its own
     batch, so the job takes the slowest rank's time; returns (that time in
@@ -788,6 +811,14 @@ def main():
                 "frac_of_int8_mma_sync": round(achieved / measured["mma_sync_s8_tops"], 4),
                 "traffic": recorded_traffic(gemm_kernel, args.workload),
                 "peak_note": "E4M3 kind::f8f6f4 dense = 2 x bf16 %s (%s)" % (bf16_peak, peak_src)}
+    if not args.fused:
+        sm_mhz = (clocks or {}).get("sm_mhz") or 2070.0
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        bound = gemm_intake_bound(M, list(zip(K_list, N_list)), sms, sm_mhz)
+        roofline["intake_bound"] = {
+            "tflops": round(bound, 1), "frac": round(achieved / bound, 4),
+            "model": "per-SM L2 intake %.0f B/clk (measured) at the median SM clock, output "
+                     "writes on the same port, the launcher's tiles" % SM_INTAKE_BYTES_PER_CLK}
     rq_roof = None
     if not args.fused:
         rq_ach = rq_bytes_all / rq_total_s / 1e9
