@@ -45,6 +45,10 @@
  *    offending access instead of faulting.
  *  - The library keeps no per-call state and is safe to call from several
  *    host threads.
+ *  - The hot-path calls (rotate-quant, the products, the fused kernel) launch
+ *    kernels only, so they can be captured in a CUDA graph; the first call of
+ *    each kernel configuration on a device sets the kernel's shared-memory
+ *    limit, so make one call of the same shape before capturing.
  */
 #ifndef CLQ_H
 #define CLQ_H
