@@ -20,6 +20,12 @@ paper's order, in plain numpy, slowly and without blocking or fusion:
   quantization to n = 4 bits, read here in its symmetric form l = -r.
 * The INT4 x INT4 product, accumulated exactly in int64, then dequantized in
   fp64 with the bias added.
+* Sec. 4.1's other bit settings (W4A8, W8A8): the same symmetric grid at
+  8 bits and the same exact product (quant_linear, obs_linear).
+* Eq. 1 itself for activations, asymmetric with the row's min and max as
+  dynamic bounds, and the product of the dequantized operands (asym_linear).
+* Sec. 3.4 / Eq. 3: the per-layer clip search over one percentile p of the
+  rotated weights' magnitudes (clip_search).
 
 Readings of the paper that this file fixes (the paper leaves them open):
 
