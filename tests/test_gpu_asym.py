@@ -209,3 +209,29 @@ def test_layer_asym_end_to_end(a_bits, w_bits):
     y64 = oracle.asym_linear(oq, od, olo, owc, os_w, b, d["bias32"])
     y = Y.float().cpu().numpy()
     check_output_frobenius(y, y64)
+
+
+@pytest.mark.parametrize("li", [0, 3])
+def test_pixart_layer_full_size_sampled_rows_asym(li):
+    """Asymmetric W4A4 on a PixArt-1024 layer at its full 8192 tokens, 42
+    sampled rows against the oracle."""
+    cfg = synth.WORKLOADS["pixart_1024"]
+    d = synth.layer_inputs(cfg, li)
+    b, K = d["b"], d["K"]
+    M = cfg["M"]
+    rows = np.sort(np.concatenate([np.random.default_rng(li).choice(M, 40, replace=False),
+                                   [0, M - 1]]))
+    perm = oracle.build_permutation(oracle.outlier_scores(d["calib"]))
+    permd = torch.from_numpy(perm).to(DEV)
+    Wq, s_w = clq.prepare_weights(d["W"].to(DEV), permd, b, codes=E4M3)
+    wsum = clq.weight_code_sums(Wq, K)
+    Xq, delta, lo = clq.rotate_quant_act_asym(d["X"].to(DEV), permd, b, codes=E4M3)
+    Y = clq.linear_asym(Xq, delta, lo, Wq, s_w, wsum, b, K, d["bias"].to(DEV),
+                        out_dtype=TD[d["dtype"]])
+    torch.cuda.synchronize()
+    oq, od, olo, orot = oracle.rotate_quant_act_asym(d["X32"][rows], perm, b, 4)
+    gq = _from_layout(Xq.cpu().numpy()[rows], E4M3, K) + 8
+    _check_asym(gq, delta.cpu().numpy()[rows], lo.cpu().numpy()[rows], oq, od, olo, orot, 4)
+    _, os_w, _, owc = oracle.prepare_weights(d["W32"], perm, b)
+    y64 = oracle.asym_linear(oq, od, olo, owc, os_w, b, d["bias32"])
+    check_output_frobenius(Y.float().cpu().numpy()[rows], y64)

@@ -265,3 +265,34 @@ def test_prepared_linear_bit_settings(a_bits, w_bits):
     else:
         with pytest.raises(ValueError):
             layer(X, fused=True)
+
+
+@pytest.mark.parametrize("li", [0, 3])
+@pytest.mark.parametrize("a_bits,w_bits", [(8, 4), (8, 8)])
+def test_pixart_layer_full_size_sampled_rows_8bit(li, a_bits, w_bits):
+    """The PixArt-1024 layer at its full 8192 tokens, every row through the
+    GPU as the bench launches it, 42 sampled rows against the oracle."""
+    from paper_2509_24416_gb300 import synth
+    cfg = synth.WORKLOADS["pixart_1024"]
+    d = synth.layer_inputs(cfg, li)
+    b, K = d["b"], d["K"]
+    M = cfg["M"]
+    rows = np.sort(np.concatenate([np.random.default_rng(li).choice(M, 40, replace=False),
+                                   [0, M - 1]]))
+    perm = oracle.build_permutation(oracle.outlier_scores(d["calib"]))
+    permd = torch.from_numpy(perm).to(DEV)
+    layout_w = SPLIT if w_bits == 8 else clq.CLQ_CODES_E4M3
+    Wq, s_w = clq.prepare_weights(d["W"].to(DEV), permd, b, codes=layout_w)
+    Xq, s_x, rot = clq.rotate_quant_act(d["X"].to(DEV), permd, b, codes=SPLIT, with_rot=True)
+    Y = clq.linear(Xq, s_x, Wq, s_w, b, K, d["bias"].to(DEV), out_dtype=TD[d["dtype"]])
+    torch.cuda.synchronize()
+    _, os_w, orot_w, owc = oracle.prepare_weights(d["W32"], perm, b, bits=w_bits)
+    _, os_x, orot, oxc = oracle.rotate_quant_act(d["X32"][rows], perm, b, bits=8)
+    check_rot(rot.cpu().numpy()[rows], orot)
+    check_scales(s_x.cpu().numpy()[rows], os_x)
+    check_codes(_split_codes(Xq.cpu().numpy()[rows], K), oxc, orot, os_x)
+    gw = (_split_codes(Wq.cpu().numpy(), K) if w_bits == 8
+          else _decode_e4m3(Wq.cpu().numpy()).astype(np.int16))
+    check_codes(gw, owc, orot_w, os_w)
+    y64, _ = oracle.quant_linear(oxc, os_x, owc, os_w, b, d["bias32"])
+    check_output_frobenius(Y.float().cpu().numpy()[rows], y64)
