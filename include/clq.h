@@ -86,7 +86,8 @@ typedef int32_t clq_dtype;
  *                         code's exact E4M3 encoding (every integer in
  *                         [-7, 7] is an E4M3 value); the execution layout the
  *                         tensor-core GEMM loads with TMA directly, without
- *                         expanding nibbles in every CTA.
+ *                         expanding nibbles in every CTA.  A zero code may
+ *                         be written as either E4M3 zero (0x00 or 0x80).
  * The codes are the same INT4 values in both layouts and every call gives
  * identical results for either.  The 8-bit layout (the W4A8 and W8A8 bit
  * settings of Sec. 4.1; codes q in [-127, 127], s = r / 127):

@@ -18,7 +18,12 @@
 //     column perm[position] (one 16-bit shared load; the 32 byte offsets are
 //     computed once per CTA), and the first butterfly stage (stride 1) is
 //     done on the way in with mixed-precision add / sub (one 16-bit operand,
-//     one fp32 operand, fp32 result);
+//     one fp32 operand, fp32 result).  For the symmetric E4M3 output each
+//     lane group reads its segment in the order position ^ m (m a multiple
+//     of 4 that differs between neighbouring lane groups), which spreads the
+//     lanes' 16-bit loads over the shared-memory banks (a swap vector is
+//     mostly ascending, so in natural order the lanes of a warp hit the same
+//     banks); see xor_order below for why the result only changes sign;
 //  2. the remaining butterfly stages up to stride 16 in registers (paired
 //     fp32x2 arithmetic), strides 32 .. b / 2 across lanes with shuffles,
 //     then the row's |x| maximum: warp reduction and a shared atomicMax;
@@ -210,6 +215,23 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
   // replaced by column 0, so a bad swap vector gives wrong values, never a
   // stray access.
   uint32_t src[32];
+  // xor_order: register k holds segment position k ^ m.  The butterflies
+  // then compute H_b P_m x, and since H[i][j ^ m] = (-1)^popc(i & m) H[i][j]
+  // for Sylvester H, that is D_m H_b x with D_m = diag((-1)^popc(i & m)):
+  // the transform up to a sign per output.  Lanes combined by the
+  // cross-lane stages share m, so the signs factor out of those stages too.
+  // The row maximum ignores signs; the codes get them back when stored (for
+  // m a multiple of 4 the sign is the same for the 4 codes of one 32-bit
+  // word: bit q of flip_words).  Only the symmetric E4M3 path uses it.
+  const bool xor_order = a.e4m3 == 1 && !CLIP && !SPLIT && !ASYM && lb >= 3 &&
+                         (reinterpret_cast<uintptr_t>(a.perm) & 15u) == 0;
+  const int xm = xor_order ? ((4 * (lane >> (lb > 5 ? lb - 5 : 0))) &
+                              ((1 << (lb < 5 ? lb : 5)) - 4))
+                           : 0;
+  uint32_t flip_words = 0;
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    if (__popc(q & (xm >> 2)) & 1) flip_words |= 1u << q;
   {
     const uint32_t base = smem_addr(raw) + static_cast<uint32_t>(r_local) * row_bytes;
     int pc[32];
@@ -217,7 +239,8 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
     if ((reinterpret_cast<uintptr_t>(a.perm) & 15u) == 0) {  // 16-byte loads
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
-        const int4 t = active ? __ldg(reinterpret_cast<const int4*>(pp) + q) : make_int4(0, 0, 0, 0);
+        const int4 t = active ? __ldg(reinterpret_cast<const int4*>(pp) + (q ^ (xm >> 2)))
+                              : make_int4(0, 0, 0, 0);
         pc[4 * q] = t.x;
         pc[4 * q + 1] = t.y;
         pc[4 * q + 2] = t.z;
@@ -366,8 +389,11 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
         if (a.rot != nullptr) {
           float4* dst = reinterpret_cast<float4*>(a.rot + static_cast<size_t>(row) * K + seg * 32);
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            dst[q] = make_float4(v[2 * q].x, v[2 * q].y, v[2 * q + 1].x, v[2 * q + 1].y);
+          for (int q = 0; q < 8; ++q) {
+            const float sg = ((flip_words >> q) & 1u) ? -1.f : 1.f;
+            dst[q] = make_float4(sg * v[2 * q].x, sg * v[2 * q].y, sg * v[2 * q + 1].x,
+                                 sg * v[2 * q + 1].y);
+          }
         }
         // v <- rint(v / s) + 1.5 * 2^23 (the code sits in the low mantissa
         // bits), with v / s as v * (1 / s).  A zero row (s = 0) gets all-zero
@@ -460,6 +486,10 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
             }
             w[k >> 1] = h[0] | (h[1] << 16);
           }
+          // xor_order signs back: flip the sign bit of each E4M3 byte of the
+          // flagged words (a zero code may come out as E4M3 -0, 0x80)
+#pragma unroll
+          for (int q = 0; q < 8; ++q) w[q] ^= (0u - ((flip_words >> q) & 1u)) & 0x80808080u;
           uint4* qrow = reinterpret_cast<uint4*>(a.Q + static_cast<size_t>(row) * K + seg * 32);
           qrow[0] = make_uint4(w[0], w[1], w[2], w[3]);
           qrow[1] = make_uint4(w[4], w[5], w[6], w[7]);
