@@ -20,7 +20,7 @@
 //     done on the way in with mixed-precision add / sub (one 16-bit operand,
 //     one fp32 operand, fp32 result).  For the symmetric E4M3 output each
 //     lane group reads its segment in the order position ^ m (m a multiple
-//     of 4 that differs between neighbouring lane groups), which spreads the
+//     of 8 that differs between neighbouring lane groups), which spreads the
 //     lanes' 16-bit loads over the shared-memory banks (a swap vector is
 //     mostly ascending, so in natural order the lanes of a warp hit the same
 //     banks); see xor_order below for why the result only changes sign;
@@ -222,11 +222,14 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
   // cross-lane stages share m, so the signs factor out of those stages too.
   // The row maximum ignores signs; the codes get them back when stored (for
   // m a multiple of 4 the sign is the same for the 4 codes of one 32-bit
-  // word: bit q of flip_words).  Only the symmetric E4M3 path uses it.
-  const bool xor_order = a.e4m3 == 1 && !CLIP && !SPLIT && !ASYM && lb >= 3 &&
+  // word: bit q of flip_words).  Only the symmetric E4M3 path uses it, with
+  // m a multiple of 8 (b >= 16): measured faster than multiples of 4, 16 or
+  // masks with low bits, which break up the 4-byte bank words that adjacent
+  // columns share.
+  const bool xor_order = a.e4m3 == 1 && !CLIP && !SPLIT && !ASYM && lb >= 4 &&
                          (reinterpret_cast<uintptr_t>(a.perm) & 15u) == 0;
-  const int xm = xor_order ? ((4 * (lane >> (lb > 5 ? lb - 5 : 0))) &
-                              ((1 << (lb < 5 ? lb : 5)) - 4))
+  const int xm = xor_order ? ((8 * (lane >> (lb > 5 ? lb - 5 : 0))) &
+                              ((1 << (lb < 5 ? lb : 5)) - 8))
                            : 0;
   uint32_t flip_words = 0;
 #pragma unroll
