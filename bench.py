@@ -772,19 +772,37 @@ def main():
 
     # ---- context (not part of value): the other path, fp16 cuBLAS on the
     # same layer shapes and rotated inputs, measured peak rates ----
-    def time_steps(fn, n):
+    def time_steps(fn, n, graph=None):
+        """ms per call of fn(k, s_ptr) over n calls, launched the way the
+        value is (one CUDA graph of the n calls, or eager with --no-graph)."""
+        graph = not args.no_graph if graph is None else graph
         for k in range(3):
-            fn(k)
+            fn(k, None)
         torch.cuda.synchronize()
+        g = None
+        if graph:
+            cs = torch.cuda.Stream(device=dev)
+            cs.wait_stream(stream)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=cs):
+                for k in range(n):
+                    fn(k, cs.cuda_stream)
+            torch.cuda.synchronize()
+            g.replay()
+            torch.cuda.synchronize()
         a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        for k in range(n):
-            fn(k)
+        if g is not None:
+            g.replay()
+        else:
+            for k in range(n):
+                fn(k, None)
         z.record(stream)
         torch.cuda.synchronize()
         return a.elapsed_time(z) / n
 
-    other_ms = time_steps(lambda k: step(k, fused=not args.fused), args.steps)
+    other_ms = time_steps(lambda k, s_ptr: step(k, fused=not args.fused, s_ptr=s_ptr),
+                          args.steps)
 
     # Each kernel of the separate path alone, K launches back to back per
     # layer (events around the K launches only): its duration with
@@ -795,11 +813,12 @@ def main():
         def rq_only(i):
             _, K, N, lay = layers[i]
 
-            def f(k):
+            def f(k, s_ptr):
                 x = xsets[k % nsets][i]
                 st = clq.clq_rotate_quant_act(x.data_ptr(), clq._dt(x), M, K, K,
                                               lay.perm.data_ptr(), b, clq.CLQ_CODES_E4M3,
-                                              xq[i].data_ptr(), sx[i].data_ptr(), None, sp)
+                                              xq[i].data_ptr(), sx[i].data_ptr(), None,
+                                              sp if s_ptr is None else s_ptr)
                 if st:
                     raise clq.ClqError(st, "clq_rotate_quant_act")
             return f
@@ -807,12 +826,13 @@ def main():
         def gm_only(i):
             _, K, N, lay = layers[i]
 
-            def f(k):
+            def f(k, s_ptr):
                 st = clq.clq_w4a4_linear(xq[i].data_ptr(), clq.CLQ_CODES_E4M3,
                                          sx[i].data_ptr(), lay.We.data_ptr(),
                                          clq.CLQ_CODES_E4M3, lay.s_w.data_ptr(),
                                          lay.bias.data_ptr(), M, N, K, b,
-                                         clq._dt(ys[i]), ys[i].data_ptr(), None, sp)
+                                         clq._dt(ys[i]), ys[i].data_ptr(), None,
+                                         sp if s_ptr is None else s_ptr)
                 if st:
                     raise clq.ClqError(st, "clq_w4a4_linear")
             return f
@@ -820,12 +840,15 @@ def main():
         rq_b2b = [time_steps(rq_only(i), args.steps) for i in range(nlay)]
         gm_b2b = [time_steps(gm_only(i), args.steps) for i in range(nlay)]
 
-    def cublas_step(si):
+    def cublas_step(si, s_ptr=None):
         xs = xsets[si % nsets]
         for i, (w, bias) in enumerate(w_dense):
             torch.addmm(bias, xs[i], w.t(), out=ys[i])
 
-    cublas_ms = time_steps(cublas_step, args.steps)
+    # cuBLAS gets its faster launch mode (measured: graph capture slows its
+    # kernels here)
+    cublas_ms = min(time_steps(cublas_step, args.steps, graph=False),
+                    time_steps(cublas_step, args.steps, graph=True))
     measured = clq.measure_peaks()
     status = clq.device_status()
     if status != 0:
