@@ -39,6 +39,13 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars.tmem_slot;
+  // The tensor maps are kernel parameters, not outputs of the previous kernel:
+  // fetch them while it finishes (measured +0.25 % on the PixArt step).
+  if (threadIdx.x == WARP_TMA * 32) {
+    prefetch_tensor_map(&mapA);
+    prefetch_tensor_map(&mapB);
+    if (use_tma_store) prefetch_tensor_map(&mapY);
+  }
   // Barriers and TMEM are set up; global inputs are read only from here on.
   pdl_wait();
   pdl_launch_dependents();
