@@ -75,13 +75,16 @@ def _check_rq(x_t, x32, perm, b):
     check_rot(grot, orot)
     check_scales(gs, os_)
     check_codes(_codes(gq, K), oc, orot, os_)
-    # both layouts carry the same codes and scales
+    # both layouts carry the same codes and scales; the E4M3 path (for b >= 16
+    # it reads each segment in an XOR order and restores the output signs)
+    # gives the same rotation too
     assert np.array_equal(_codes(eq, K), _codes(gq, K)) and np.array_equal(es, gs)
+    check_rot(erot, orot)
     return gq, gs
 
 
 # ------------------------------------------------------------ rotate-quant --
-@pytest.mark.parametrize("b", [1, 2, 8, 32, 64, 128, 256])
+@pytest.mark.parametrize("b", [1, 2, 8, 16, 32, 64, 128, 256])
 @pytest.mark.parametrize("dtype", ["f16", "bf16"])
 def test_rotate_quant_block_sizes(b, dtype):
     K = 512
