@@ -345,10 +345,12 @@ clq_status clq_clip_search(const void* W, clq_dtype dtype, int32_t N, int32_t K,
 size_t clq_fused_linear_workspace_size(int32_t M, int32_t K);
 
 /*
- * The whole layer in one persistent kernel: every CTA first rotates and
- * quantizes its share of token rows into `workspace` (which stays in L2 for
- * the layer sizes of the paper's models), then runs GEMM tiles, each of which
- * starts as soon as the rows of its token block are published.  Same
+ * The whole layer in one persistent kernel: every CTA rotates and quantizes
+ * token rows into `workspace` (which stays in L2 for the layer sizes of the
+ * paper's models) and runs GEMM tiles, each of which starts as soon as the
+ * rows of its token block are published.  With E4M3 weights and K <= 9216
+ * the two run side by side in every CTA; otherwise each CTA first finishes
+ * its rows, then turns to the GEMM.  Same
  * arithmetic and results as clq_rotate_quant_act followed by
  * clq_w4a4_linear.  X: device [M][ldx] of `dtype`; Y: device [M][N] of
  * `dtype`; bias: device [N] of `dtype` or NULL; W / w_codes as for

@@ -56,6 +56,9 @@ struct GemmArgs {
 // ([rows][K/2]), CLQ_CODES_E4M3 ([rows][K]) or, for 8-bit codes,
 // CLQ_CODES_E4M3_SPLIT ([rows][2][K]; A split with B E4M3 or split); TMA maps
 // are built here.
+// Output-channel tile width (192 or 256) of the E4M3 x E4M3 GEMM for an
+// M x N product on `sms` SMs.
+int gemm_tile_n(int M, int N, int sms);
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st);
 

@@ -56,10 +56,13 @@ constexpr int MAX_STAGES = 6;
 // PA / PB: E4M3 planes per operand, 1 for 4-bit codes, 2 for 8-bit codes
 // split as q = 16 h + l (plane 0 holds 16 h, plane 1 holds l; both E4M3
 // values, so the MMAs of the two planes add up to q in one accumulator).
-template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1>
+// EW: epilogue warps (0: 4 with unpack warps, else 8); SMAX: stage cap, for
+// a CTA that keeps shared memory for other work.
+template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1, int EW = 0,
+          int SMAX = MAX_STAGES>
 struct Cfg {
   static constexpr bool UNPACK = APACK || BPACK;
-  static constexpr int EPI_WARPS = UNPACK ? 4 : 8;
+  static constexpr int EPI_WARPS = EW != 0 ? EW : (UNPACK ? 4 : 8);
   static constexpr int THREADS = UNPACK ? MIN_THREADS : 320;
   static constexpr int EPI_THREADS = 32 * EPI_WARPS;
   static constexpr int EPI_NBUF = 8 / EPI_WARPS;  // staging buffers per warp
@@ -70,7 +73,7 @@ struct Cfg {
   static constexpr int STAGE = AU + BU + (APACK ? A_P : 0) + (BPACK ? BP : 0);
   static constexpr int FIXED = EPI_TOTAL + 6 * BNT * 4;
   static constexpr int S0 = (222 * 1024 - FIXED) / STAGE;
-  static constexpr int S = S0 > MAX_STAGES ? MAX_STAGES : S0;  // pipeline stages
+  static constexpr int S = S0 > SMAX ? SMAX : S0;  // pipeline stages
   static constexpr size_t OFF_UA = 0;                           // E4M3 operands
   static constexpr size_t OFF_UB = OFF_UA + S * AU;
   static constexpr size_t OFF_PA = OFF_UB + S * BU;             // packed staging
@@ -85,6 +88,8 @@ struct Cfg {
   static_assert(S >= 2, "pipeline needs two stages");
   static_assert((PA == 1 || PA == 2) && (PB == 1 || PB == 2), "one or two planes");
   static_assert(!UNPACK || (PA == 1 && PB == 1), "8-bit planes come as E4M3 only");
+  static_assert(EPI_WARPS == 4 || (EPI_WARPS == 8 && !UNPACK), "4 or 8 epilogue warps");
+  static_assert(SMAX <= MAX_STAGES, "barrier arrays hold MAX_STAGES stages");
 };
 
 struct __align__(8) Barriers {
@@ -118,9 +123,10 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 
 // Barrier init (thread 0) and TMEM allocation (warp WARP_MMA); the caller
 // follows with tcgen05 fences around a CTA barrier.
-template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1>
+template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1, int EW = 0,
+          int SMAX = MAX_STAGES>
 __device__ __forceinline__ void setup(Barriers* bars) {
-  using C = Cfg<APACK, BPACK, BNT, PA, PB>;
+  using C = Cfg<APACK, BPACK, BNT, PA, PB, EW, SMAX>;
   constexpr int S = C::S;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -162,11 +168,12 @@ __device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, ui
 // EPI_PREFETCH: let the epilogue prefetch TMEM (taken only in the 320-thread
 // configuration, where registers allow it).
 // ASYM: asymmetric activation codes (zero-point epilogue, g.lo / g.wsum).
+// EW / SMAX: as in Cfg (the same values as the setup() call).
 template <typename OutT, bool APACK, bool BPACK, int BNT = BN, bool EPI_PREFETCH = true,
-          int PA = 1, int PB = 1, bool ASYM = false>
+          int PA = 1, int PB = 1, bool ASYM = false, int EW = 0, int SMAX = MAX_STAGES>
 __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
                                          Barriers* bars, uint32_t tmem, const uint32_t* ready) {
-  using C = Cfg<APACK, BPACK, BNT, PA, PB>;
+  using C = Cfg<APACK, BPACK, BNT, PA, PB, EW, SMAX>;
   constexpr int S = C::S;
   volatile int32_t* abort = &bars->abort;
 

@@ -271,27 +271,28 @@ bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows
                                CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
+// Tile width of the E4M3 x E4M3 GEMM: an SM's intake from L2 bounds the
+// kernel, so a tile costs about its operand bytes per K step (A 16 KB + B
+// BN/8 KB), and the CTAs walk ceil(tiles / SMs) rounds.  256 wins unless 192
+// splits N into whole tiles with no more rounds (N = 1152: 6 x 192 instead of
+// 4.5 x 256).  128 measured slower everywhere.
+int gemm_tile_n(int M, int N, int sms) {
+  const long mt = (M + BM - 1) / BM;
+  auto cost = [&](int w) {
+    const long rounds = (mt * ((N + w - 1) / w) + sms - 1) / sms;
+    return rounds * (16.0 + w / 8.0);
+  };
+  return cost(192) < cost(256) ? 192 : BN;
+}
+
 cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, int w_codes,
                              const GemmArgs& g, int out_dtype, cudaStream_t st) {
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
   const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
   const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
-  // Tile width: an SM's intake from L2 bounds the kernel, so a tile costs
-  // about its operand bytes per K step (A 16 KB + B BN/8 KB), and the CTAs
-  // walk ceil(tiles / SMs) rounds.  256 wins unless 192 splits N into whole
-  // tiles with no more rounds (N = 1152: 6 x 192 instead of 4.5 x 256).  128
-  // measured slower everywhere.
   const bool split = x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT;
-  int bn = BN;
-  if (!apack && !bpack && !split && g.lo == nullptr) {
-    const long mt = (g.M + BM - 1) / BM;
-    auto cost = [&](int w) {
-      const long rounds = (mt * ((g.N + w - 1) / w) + sms - 1) / sms;
-      return rounds * (16.0 + w / 8.0);
-    };
-    if (cost(192) < cost(256)) bn = 192;
-  }
+  const int bn = (!apack && !bpack && !split && g.lo == nullptr) ? gemm_tile_n(g.M, g.N, sms) : BN;
   MapSet m;
   if (!encode_codes_map(&m.A, Xq, x_codes, g.M, g.K, BM, 0) ||
       !encode_codes_map(&m.B, W, w_codes, g.N, g.K, bn, 0))
