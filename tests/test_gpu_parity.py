@@ -383,7 +383,12 @@ def test_prepared_linear_state_roundtrip(tmp_path):
                                            (300, 600, 1152, 128, "bf16"),
                                            (129, 264, 4608, 256, "f16"),
                                            (64, 256, 12288, 128, "bf16"),
-                                           (40, 128, 16384, 64, "f16")])
+                                           (40, 128, 16384, 64, "f16"),
+                                           # the widest rows of the concurrent form
+                                           # (one row a tile) and the first K of
+                                           # the sequential form with E4M3 weights
+                                           (130, 200, 9216, 128, "f16"),
+                                           (70, 130, 9248, 32, "bf16")])
 def test_fused_matches_separate_and_oracle(M, N, K, b, dtype):
     x_t, x32 = _inputs(M, K, dtype, seed=M + K)
     rng = np.random.default_rng(K)
