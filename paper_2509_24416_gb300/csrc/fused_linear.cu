@@ -36,42 +36,49 @@ namespace {
 
 using namespace gemm;
 
-constexpr int FT = 512;  // threads: the RQ phase uses all, the GEMM phase up to 448
+// Threads per CTA.  Sequential form: rotate-quant on all of them, then the
+// GEMM pipeline on up to 448.  Concurrent form: GEMM warps 0-5 beside
+// rotate-quant warps 6-15.
+constexpr int FT = 512;
+
+// Adds the rows [row0, row0 + rows) to the ready counters of the 128-token
+// blocks they fall in (a tile of rows may straddle two blocks); RELEASE: each
+// add is a release at GPU scope, else relaxed (the caller fences first).
+template <bool RELEASE>
+__device__ __forceinline__ void count_rows(uint32_t* ready, int row0, int rows) {
+  int r = row0;
+  const int end = row0 + rows;
+  while (r < end) {
+    const int mb = r / BM;
+    const int stop = min(end, (mb + 1) * BM);
+    const unsigned n = static_cast<unsigned>(stop - r);
+    if (RELEASE)
+      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(ready + mb), "r"(n)
+                   : "memory");
+    else
+      atomicAdd(ready + mb, n);
+    r = stop;
+  }
+}
 
 struct PublishRows {
   uint32_t* ready;
   rq::Team team;  // the threads that stored the rows
+  // Every team thread, once its stores of the tile are issued: proxy fence,
+  // team barrier, then one thread publishes (fence at GPU scope, adds).
   __device__ void operator()(int row0, int rows) const {
     fence_proxy_async_global();
     team.sync();
     if (team.rank() == 0) {
       __threadfence();
-      int r = row0;
-      const int end = row0 + rows;
-      while (r < end) {
-        const int mb = r / BM;
-        const int stop = min(end, (mb + 1) * BM);
-        atomicAdd(ready + mb, static_cast<unsigned>(stop - r));
-        r = stop;
-      }
+      count_rows<false>(ready, row0, rows);
     }
   }
   // Loader mode: the compute threads have fenced their stores for the async
   // proxy and signalled them on a CTA barrier this thread has waited on; a
   // release add at GPU scope makes them visible to every CTA that acquires
   // the counter.
-  __device__ void release(int row0, int rows) const {
-    int r = row0;
-    const int end = row0 + rows;
-    while (r < end) {
-      const int mb = r / BM;
-      const int stop = min(end, (mb + 1) * BM);
-      asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(ready + mb),
-                   "r"(static_cast<unsigned>(stop - r))
-                   : "memory");
-      r = stop;
-    }
-  }
+  __device__ void release(int row0, int rows) const { count_rows<true>(ready, row0, rows); }
 };
 
 // Rotate-quant stage geometry of the fused kernel: its shared memory is sized
