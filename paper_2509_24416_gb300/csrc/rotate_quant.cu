@@ -38,7 +38,9 @@ __global__ void outlier_scores_kernel(const uint16_t* calib, int B, int Tn, int 
 // on GB300 (M up to 65536 tokens): a CTA takes about max(1.2, 0.1 + 0.121 W)
 // us per tile when W warps share the SM (a latency floor, then issue-bound),
 // every CTA walks ceil(tiles / CTAs) tiles, and the first tile's arrival adds
-// about 0.7 us per 2304-byte row; a lone CTA per SM pays 1.35x per tile.  Few
+// about 0.25 us per 2304-byte row (refit after the XOR-ordered gather: a sweep
+// of rows per tile over the benchmark shapes); a lone CTA per SM pays 1.35x
+// per tile.  Few
 // rows per tile win when M is small (more CTAs share the work), many when M
 // is large.
 void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads,
@@ -62,7 +64,7 @@ void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads
     // (measured: 1.35x per tile at K = 4608).
     const double alone = ctas == 1 ? 1.35 : 1.0;
     const double cost = rounds * alone * std::max(1.2, 0.1 + 0.121 * ctas * warps) +
-                        0.7 * r * (2.0 * K) / 2304.0;
+                        0.25 * r * (2.0 * K) / 2304.0;
     if (cost < best_cost - 1e-9) {
       best_cost = cost;
       best_r = r;
