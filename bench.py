@@ -91,6 +91,23 @@ KERNEL_SOURCES = {
 }
 
 
+ACT_CODE_BYTES = 1.0  # bytes per activation code in the layout the timed path writes
+
+
+def rq_algorithmic_bytes(M, K):
+    """HBM bytes one rotate-quant launch must move, whatever code layout it
+    writes: the 16-bit input (2 B an element), the packed INT4 codes (0.5 B an
+    element) and one fp32 scale a row: M (2.5 K + 4).  The roofline fraction
+    of the kernel is taken on these bytes."""
+    return M * (2.5 * K + 4)
+
+
+def rq_layout_bytes(M, K, code_bytes):
+    """Bytes the launch actually moves with `code_bytes` bytes a code (1 for
+    the E4M3 layout, 0.75 for E2M3, 0.5 packed, 2 for split 8-bit planes)."""
+    return M * ((2.0 + code_bytes) * K + 4)
+
+
 SM_INTAKE_BYTES_PER_CLK = 64.0  # measured per-SM L2 -> SM ceiling (profiles/peaks_gb300.md)
 
 
@@ -404,7 +421,8 @@ def run_sweep(args):
                 cell.update({
                     "valid": True,
                     "rotate_quant_us": round(rq_us, 2),
-                    "rotate_quant_GBps": round(M * (3.0 * K + 4) / (rq_us * 1e-6) / 1e9, 1),
+                    "rotate_quant_GBps": round(rq_algorithmic_bytes(M, K) / (rq_us * 1e-6) / 1e9,
+                                               1),
                     "separate_us": round(sep_us, 2),
                     "separate_TOPS": round(ops / (sep_us * 1e-6) / 1e12, 1),
                     "fused_us": round(fu_us, 2),
@@ -534,7 +552,9 @@ def run_bits(args):
             rq = sum(e[3 * i].elapsed_time(e[3 * i + 1]) for e in evs) / args.steps
             gm = sum(e[3 * i + 1].elapsed_time(e[3 * i + 2]) for e in evs) / args.steps
             K, N = d["K"], d["N"]
-            rq_bytes = M * (2.0 * K + width * K + (8 if asym else 4))
+            # algorithmic bytes at this activation width: 16-bit input, packed
+            # codes (bits / 8 B a code), the per-row scale (and minimum)
+            rq_bytes = M * (2.0 * K + (width / 2.0) * K + (8 if asym else 4))
             y = ys[i][:ERR_ROWS].double().cpu().numpy()
             err = float(((y - refs[i]) ** 2).sum() ** 0.5 / (refs[i] ** 2).sum() ** 0.5)
             per_layer.append({
@@ -871,7 +891,7 @@ def main():
     for i, (name, K, N, _) in enumerate(layers):
         rq_us = 1e3 * rq_ms[i] / args.steps
         gm_us = 1e3 * gm_ms[i] / args.steps
-        rq_bytes = M * (3.0 * K + 4)  # fp16 in, one E4M3 code byte out, scale
+        rq_bytes = rq_algorithmic_bytes(M, K)
         per_layer.append({
             "layer": name, "K": K, "N": N,
             "us": round(rq_us + gm_us, 2),
@@ -887,7 +907,8 @@ def main():
     rq_total_s = rq_ms.sum() * 1e-3 / args.steps
     gemm_kernel = "fused_linear" if args.fused else "w4a4_gemm"
     achieved = gemm_flops / gm_total_s / 1e12
-    rq_bytes_all = sum(M * (3.0 * K + 4) for K in K_list)
+    rq_bytes_all = sum(rq_algorithmic_bytes(M, K) for K in K_list)
+    rq_layout_all = sum(rq_layout_bytes(M, K, ACT_CODE_BYTES) for K in K_list)
     roofline = {"kernel": gemm_kernel, "bound": "tensor", "achieved": round(achieved, 1),
                 "peak": fp8_peak, "unit": "TFLOP/s", "frac": round(achieved / fp8_peak, 4),
                 "frac_of_measured_tcgen05_e4m3": round(achieved / measured["tcgen05_e4m3_tflops"], 4),
@@ -912,6 +933,11 @@ def main():
         rq_roof = {"kernel": "rotate_quant", "bound": "hbm", "achieved": round(rq_ach, 1),
                    "peak": hbm_peak, "unit": "GB/s", "frac": round(rq_ach / hbm_peak, 4),
                    "frac_of_8TBps": round(rq_ach / 8000.0, 4),
+                   "algorithmic_bytes_per_step": int(rq_bytes_all),
+                   "bytes_note": "2.5 B/element + 4 B/row (16-bit input, packed INT4 codes, "
+                                 "fp32 scale)",
+                   "layout_bytes_per_step": int(rq_layout_all),
+                   "layout_GBps": round(rq_layout_all / rq_total_s / 1e9, 1),
                    "traffic": recorded_traffic("rotate_quant", args.workload)}
         if rq_b2b is not None:
             rq_b2b_ach = rq_bytes_all / (sum(rq_b2b) * 1e-3) / 1e9

@@ -601,9 +601,13 @@ class PreparedLinear:
         clip = errors = best = None
         if clip_grid is not None and w_bits == 4:
             Xcal = calib.reshape(-1, K).contiguous()
-            Yref = Xcal.float() @ W.float().t()
+            # The search's target, the layer's full-precision output: taken in
+            # fp64 and rounded once to fp32, so that no matmul setting of the
+            # caller (TF32, reduced-precision reductions) changes the objective.
+            Yref = Xcal.double() @ W.double().t()
             if bias is not None:
-                Yref = Yref + bias.float()[None, :]
+                Yref = Yref + bias.double()[None, :]
+            Yref = Yref.float().contiguous()
             clip, errors, best = clip_search(W.contiguous(), perm, b, Xcal, Yref, bias,
                                              grid=clip_grid, stream=stream)
         layer = cls.from_weight(W, perm, b, bias=bias, clip=clip, a_bits=a_bits,

@@ -384,6 +384,44 @@ clq_status clq_weight_code_sums(const uint8_t* W, clq_codes w_codes, int32_t N, 
       clq::launch_code_sums(W, w_codes, N, K, wsum, static_cast<cudaStream_t>(stream)));
 }
 
+}  // extern "C"
+
+namespace clq {
+
+// Host checks of clq_fused_linear's arguments other than its workspace, in
+// the order that call makes them; *noop is set when M or N is 0.
+int32_t fused_linear_check(const void* X, int32_t dtype, int32_t M, int32_t K, int32_t ldx,
+                           const int32_t* perm, int32_t b, const uint8_t* W, int32_t w_codes,
+                           const float* s_w, const void* bias, int32_t N, const void* Y,
+                           bool* noop) {
+  *noop = false;
+  if (!valid_dtype(dtype) || !valid_codes(w_codes) || M < 0 || N < 0)
+    return CLQ_ERR_INVALID_ARG;
+  clq_status st = check_k_b(K, b);
+  if (st != CLQ_OK) return st;
+  if (ldx < K) return CLQ_ERR_SHAPE;
+  if (ldx % 8 != 0) return CLQ_ERR_ALIGN;
+  if (M == 0 || N == 0) {
+    *noop = true;
+    return CLQ_OK;
+  }
+  if (X == nullptr || perm == nullptr || W == nullptr || s_w == nullptr || Y == nullptr)
+    return CLQ_ERR_INVALID_ARG;
+  if (!aligned(X, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(perm, 4) ||
+      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)))
+    return CLQ_ERR_ALIGN;
+  return CLQ_OK;
+}
+
+int32_t device_check() {
+  int32_t* status = nullptr;
+  return device_setup(&status);
+}
+
+}  // namespace clq
+
+extern "C" {
+
 size_t clq_fused_linear_workspace_size(int32_t M, int32_t K) {
   if (M < 0 || K < 32 || K > 16384 || K % 32 != 0) return 0;
   return clq::fused_workspace_layout(M, K).bytes;
@@ -393,21 +431,14 @@ clq_status clq_fused_linear(const void* X, clq_dtype dtype, int32_t M, int32_t K
                             const int32_t* perm, int32_t b, const uint8_t* W,
                             clq_codes w_codes, const float* s_w, const void* bias, int32_t N,
                             void* Y, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!valid_dtype(dtype) || !valid_codes(w_codes) || M < 0 || N < 0)
-    return CLQ_ERR_INVALID_ARG;
-  clq_status st = check_k_b(K, b);
-  if (st != CLQ_OK) return st;
-  if (ldx < K) return CLQ_ERR_SHAPE;
-  if (ldx % 8 != 0) return CLQ_ERR_ALIGN;
-  if (M == 0 || N == 0) return CLQ_OK;
-  if (X == nullptr || perm == nullptr || W == nullptr || s_w == nullptr || Y == nullptr ||
-      workspace == nullptr)
-    return CLQ_ERR_INVALID_ARG;
+  bool noop = false;
+  clq_status st =
+      clq::fused_linear_check(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w, bias, N, Y, &noop);
+  if (st != CLQ_OK || noop) return st;
+  if (workspace == nullptr) return CLQ_ERR_INVALID_ARG;
   const clq::FusedWorkspace ws = clq::fused_workspace_layout(M, K);
   if (workspace_bytes < ws.bytes) return CLQ_ERR_INVALID_ARG;
-  if (!aligned(X, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(perm, 4) ||
-      !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)) || !aligned(workspace, 256))
-    return CLQ_ERR_ALIGN;
+  if (!aligned(workspace, 256)) return CLQ_ERR_ALIGN;
   int32_t* status = nullptr;
   st = device_setup(&status);
   if (st != CLQ_OK) return st;

@@ -93,6 +93,15 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq, const uint8_t* W, int
                                 const GemmArgs& g, int logb, int dtype, uint32_t* ready,
                                 cudaStream_t st);
 
+// Host checks of clq_fused_linear's arguments other than its workspace, in
+// the order that call makes them (a clq_status; *noop set when M or N is 0),
+// and the check that the current device is an sm_103 GPU.
+int32_t fused_linear_check(const void* X, int32_t dtype, int32_t M, int32_t K, int32_t ldx,
+                           const int32_t* perm, int32_t b, const uint8_t* W, int32_t w_codes,
+                           const float* s_w, const void* bias, int32_t N, const void* Y,
+                           bool* noop);
+int32_t device_check();
+
 // Bounded-wait self test (one CTA, one mbarrier nothing arrives at).
 cudaError_t launch_wait_selftest(uint64_t timeout_ns, int32_t* status, cudaStream_t st);
 

@@ -9,6 +9,7 @@
 #include <cuda_runtime.h>
 
 #include "../../include/clq.h"
+#include "clq_kernels.h"
 
 namespace {
 
@@ -31,8 +32,10 @@ clq_status scratch_address(void** out) {
   void* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
   if (p == nullptr) {
     void* q = nullptr;
-    if (cudaGetSymbolAddress(&q, g_noalloc_scratch) != cudaSuccess || q == nullptr)
+    if (cudaGetSymbolAddress(&q, g_noalloc_scratch) != cudaSuccess || q == nullptr) {
+      cudaGetLastError();  // leave no error behind for the caller's next check
       return CLQ_ERR_CUDA;
+    }
     g_scratch_ptr[dev].store(q, std::memory_order_release);
     p = q;
   }
@@ -48,16 +51,22 @@ extern "C" clq_status clq_fused_linear_noalloc(const void* X, clq_dtype dtype, i
                                                clq_codes w_codes, const float* s_w,
                                                const void* bias, int32_t N, void* Y,
                                                void* stream) {
-  if (M > 0 && K >= 32 && K <= 16384 && K % 32 == 0 &&
-      clq_fused_linear_workspace_size(M, K) > CLQ_NOALLOC_SCRATCH_BYTES)
+  // The same checks, in the same order, as clq_fused_linear; an empty problem
+  // is a no-op whatever its size.
+  bool noop = false;
+  clq_status st = clq::fused_linear_check(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w, bias,
+                                          N, Y, &noop);
+  if (st != CLQ_OK || noop) return st;
+  if (clq_fused_linear_workspace_size(M, K) > CLQ_NOALLOC_SCRATCH_BYTES)
     return CLQ_ERR_SCRATCH_LIMIT;
+  // An unsupported device is reported as such before the symbol is looked up.
+  st = clq::device_check();
+  if (st != CLQ_OK) return st;
   void* scratch = nullptr;
-  if (M > 0 && N > 0) {
-    const clq_status st = scratch_address(&scratch);
-    if (st != CLQ_OK) return st;
-  }
-  // The forwarded call validates every other argument, clears the counters
-  // it needs in the scratch array and launches on `stream`.
+  st = scratch_address(&scratch);
+  if (st != CLQ_OK) return st;
+  // The forwarded call clears the counters it needs in the scratch array and
+  // launches on `stream`.
   return clq_fused_linear(X, dtype, M, K, ldx, perm, b, W, w_codes, s_w, bias, N, Y, scratch,
                           CLQ_NOALLOC_SCRATCH_BYTES, stream);
 }

@@ -109,7 +109,8 @@ def test_prepared_linear_calibrate_runs_the_offline_steps(metric):
     assert torch.equal(info["perm"].cpu(), perm)
     K = W.shape[1]
     Xcal = calib.reshape(-1, K).contiguous()
-    Yref = Xcal.float() @ W.float().t() + bias.float()[None, :]
+    # the target calibrate() uses: fp64 product rounded once to fp32
+    Yref = (Xcal.double() @ W.double().t() + bias.double()[None, :]).float()
     clip, errors, best = clq.clip_search(W, perm.to(DEV), b, Xcal, Yref, bias)
     assert best == info["best"] and torch.equal(clip, info["clip"])
     ref = clq.PreparedLinear.from_weight(W, perm.to(DEV), b, bias=bias, clip=clip)
