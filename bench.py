@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--impl", default="clq", choices=["clq", "reference"])
     p.add_argument("--workload", default="pixart_1024")
     p.add_argument("--fused", action="store_true")
+    p.add_argument("--codes", default="auto", choices=["auto", "e4m3", "e2m3"],
+                   help="execution layout of the 4-bit codes (auto: the layer's default)")
     p.add_argument("--sweep", action="store_true",
                    help="time the 100-cell M x (K, N) x b grid, one JSON line per cell")
     p.add_argument("--bits", action="store_true",
@@ -91,7 +93,7 @@ KERNEL_SOURCES = {
 }
 
 
-ACT_CODE_BYTES = 1.0  # bytes per activation code in the layout the timed path writes
+CODES = {"auto": None, "e4m3": 1, "e2m3": 3}  # clq.CLQ_CODES_E4M3 / CLQ_CODES_E2M3
 
 
 def rq_algorithmic_bytes(M, K):
@@ -108,18 +110,17 @@ def rq_layout_bytes(M, K, code_bytes):
     return M * ((2.0 + code_bytes) * K + 4)
 
 
-SM_INTAKE_BYTES_PER_CLK = 64.0  # measured per-SM L2 -> SM ceiling (profiles/peaks_gb300.md)
-
-
-def gemm_intake_bound(M, shapes, sms, sm_mhz):
-    """The GEMM's structural ceiling on this part: every SM takes at most
-    SM_INTAKE_BYTES_PER_CLK from L2 per clock, and each 128 x w output tile
-    brings (128 + w) K operand bytes in and sends 2 x 128 w output bytes out
-    through the same port.  Tiles are those the launcher picks (w = 192 when
-    it covers N in whole tiles with no more rounds, else 256), dealt round-
-    robin, so a layer takes ceil(tiles / SMs) tile-times.  Returns TFLOP/s
-    over the layer set."""
-    rate = SM_INTAKE_BYTES_PER_CLK * sm_mhz * 1e6
+def gemm_intake_bound(M, shapes, sms, sm_mhz, bytes_per_clk):
+    """The GEMM's structural ceiling on this part: TMA fills each SM's shared
+    memory with at most `bytes_per_clk` operand bytes per clock (measured in
+    the same run by clq_peak_operand_stream, counted in shared-memory bytes,
+    which are 128 per row and K step for E4M3 and E2M3 alike), and each 128 x w
+    output tile brings (128 + w) K operand bytes in and sends 2 x 128 w output
+    bytes out through the same engine.  Tiles are those the launcher picks
+    (w = 192 when it covers N in whole tiles with no more rounds, else 256),
+    dealt round-robin, so a layer takes ceil(tiles / SMs) tile-times.  Returns
+    TFLOP/s over the layer set."""
+    rate = bytes_per_clk * sm_mhz * 1e6
     mt = (M + 127) // 128
     t_total, ops = 0.0, 0.0
     for (K, N) in shapes:
@@ -264,20 +265,81 @@ def run_oracle(workload, rows, reps):
                 os.environ[k] = v
 
 
+def _oracle_slice_worker(workload, rows, w, nworkers, barrier, out):
+    """One process of the all-core oracle run: token rows [w rows, (w + 1) rows)
+    of a batch of rows * nworkers tokens, prepared untimed, then timed once
+    after every worker has reached the barrier."""
+    import oracle
+    from paper_2509_24416_gb300 import synth
+    cfg = synth.WORKLOADS[workload]
+    prepared = []
+    for li in range(len(cfg["layers"])):
+        d = synth.layer_inputs(cfg, li, M=rows * nworkers)
+        perm = oracle.build_permutation(oracle.outlier_scores(d["calib"]))
+        Wq, s_w, _, _ = oracle.prepare_weights(d["W32"], perm, cfg["b"])
+        prepared.append((d["X32"][w * rows:(w + 1) * rows], perm, Wq, s_w, d["bias32"]))
+    barrier.wait()
+    t0 = time.perf_counter()
+    for (x, perm, Wq, s_w, bias) in prepared:
+        Xq, s_x, _, _ = oracle.rotate_quant_act(x, perm, cfg["b"])
+        oracle.w4a4_linear(Xq, s_x, Wq, s_w, cfg["b"], bias)
+    out.put((w, t0, time.perf_counter()))
+
+
+def run_oracle_all_cores(workload, rows, nworkers):
+    """The oracle on `nworkers` single-threaded spawned processes at once,
+    each on its own slice of `rows` tokens; returns the wall time from the
+    first start to the last end (perf_counter is system-wide monotonic)."""
+    import multiprocessing as mp
+    env = {"OMP_NUM_THREADS": "1", "OPENBLAS_NUM_THREADS": "1",
+           "MKL_NUM_THREADS": "1"}
+    old = {k: os.environ.get(k) for k in env}
+    os.environ.update(env)
+    try:
+        ctx = mp.get_context("spawn")
+        barrier = ctx.Barrier(nworkers)
+        out = ctx.Queue()
+        procs = [ctx.Process(target=_oracle_slice_worker,
+                             args=(workload, rows, w, nworkers, barrier, out))
+                 for w in range(nworkers)]
+        for p in procs:
+            p.start()
+        res = [out.get() for _ in procs]
+        for p in procs:
+            p.join()
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    return max(r[2] for r in res) - min(r[1] for r in res)
+
+
 def cpu_baseline(workload, budget_s=20.0):
+    """The oracle as it stands on the host cores: one core (a spawned
+    single-threaded process, best of 2) and every core (`os.cpu_count()`
+    single-threaded processes on disjoint token slices, one pass)."""
     from paper_2509_24416_gb300 import synth
     cfg = synth.WORKLOADS[workload]
     probe_rows = 16
     t = run_oracle(workload, probe_rows, 1)[0]
     rows = int(max(16, min(cfg["M"], probe_rows * budget_s / max(t, 1e-3) / 2)))
     times = run_oracle(workload, rows, 2)
-    sec = min(times)
-    ops = sum(layer_ops(cfg, rows))
-    return {"value": ops / sec / 1e12, "unit": "TOPS", "cores": 1,
+    sec1 = min(times)
+    one = sum(layer_ops(cfg, rows)) / sec1 / 1e12
+    ncores = os.cpu_count() or 1
+    rows_w = int(max(1, min(cfg["M"] // ncores, rows)))
+    sec_n = run_oracle_all_cores(workload, rows_w, ncores)
+    alln = sum(layer_ops(cfg, rows_w * ncores)) / sec_n / 1e12
+    return {"value": alln, "unit": "TOPS", "cores": ncores, "nproc": ncores,
             "kind": "oracle",
-            "sample": "%d of %d tokens per layer, all %d layers, rotate-quant + "
-                      "int64 GEMM + fp64 epilogue, numpy single-threaded, best of 2"
-                      % (rows, cfg["M"], len(cfg["layers"]))}
+            "sample": "%d tokens per core (%d in all) of %d per layer, all %d layers, "
+                      "rotate-quant + int64 GEMM + fp64 epilogue, numpy, %d single-threaded "
+                      "processes at once, one pass" % (rows_w, rows_w * ncores, cfg["M"],
+                                                       len(cfg["layers"]), ncores),
+            "single_core": {"value": one, "unit": "TOPS", "cores": 1,
+                            "sample": "%d of %d tokens per layer, best of 2" % (rows, cfg["M"])}}
 
 
 def reference_arm(args):
@@ -376,7 +438,7 @@ def run_sweep(args):
                 xs.append(x.half())
                 del x
             Y = torch.empty((M, N), dtype=torch.float16, device=dev)
-            xq = torch.empty((M, K), dtype=torch.uint8, device=dev)
+            xq = torch.empty((M, K), dtype=torch.uint8, device=dev)  # widest 4-bit layout
             s_x = torch.empty(M, dtype=torch.float32, device=dev)
             ws = clq.fused_workspace(M, K, dev)
             ops = 2.0 * M * N * K
@@ -392,15 +454,15 @@ def run_sweep(args):
 
                 def rq(k):
                     st = clq.clq_rotate_quant_act(xs[k % nsets].data_ptr(), clq.CLQ_F16, M, K, K,
-                                                  perm.data_ptr(), b, clq.CLQ_CODES_E4M3,
+                                                  perm.data_ptr(), b, lay.act_codes,
                                                   xq.data_ptr(), s_x.data_ptr(), None, sp)
                     if st:
                         raise clq.ClqError(st, "clq_rotate_quant_act")
 
                 def sep(k):
                     rq(k)
-                    st = clq.clq_w4a4_linear(xq.data_ptr(), clq.CLQ_CODES_E4M3, s_x.data_ptr(),
-                                             lay.We.data_ptr(), clq.CLQ_CODES_E4M3,
+                    st = clq.clq_w4a4_linear(xq.data_ptr(), lay.act_codes, s_x.data_ptr(),
+                                             lay.We.data_ptr(), lay.w_codes,
                                              lay.s_w.data_ptr(), lay.bias.data_ptr(), M, N, K, b,
                                              clq.CLQ_F16, Y.data_ptr(), None, sp)
                     if st:
@@ -409,7 +471,7 @@ def run_sweep(args):
                 def fused(k):
                     st = clq.clq_fused_linear(xs[k % nsets].data_ptr(), clq.CLQ_F16, M, K, K,
                                               perm.data_ptr(), b, lay.We.data_ptr(),
-                                              clq.CLQ_CODES_E4M3, lay.s_w.data_ptr(),
+                                              lay.w_codes, lay.s_w.data_ptr(),
                                               lay.bias.data_ptr(), N, Y.data_ptr(),
                                               ws.data_ptr(), ws.numel(), sp)
                     if st:
@@ -481,18 +543,20 @@ def run_bits(args):
         x64 = d["X32"][:ERR_ROWS].astype("float64")
         refs.append(x64 @ d["W32"].astype("float64").T + d["bias32"].astype("float64")[None, :])
     for name, a_bits, w_bits, asym in BIT_SETTINGS:
+        # asymmetric 4-bit codes reach -8, which only the E4M3 layout holds
+        w4 = clq.CLQ_CODES_E4M3 if asym and w_bits == 4 else None
         lays = [clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b, bias=d["bias"].to(dev),
-                                               a_bits=a_bits, w_bits=w_bits)
+                                               a_bits=a_bits, w_bits=w_bits, w_codes=w4)
                 for d, perm in data]
         wsums = [clq.weight_code_sums(lay.We, d["K"]) for lay, (d, _) in zip(lays, data)]
-        width = 2 if a_bits == 8 else 1
-        xq = [torch.empty((M, width * d["K"]), dtype=torch.uint8, device=dev) for d, _ in data]
+        x_codes = lays[0].act_codes
+        w_codes = lays[0].w_codes
+        xq = [torch.empty((M, clq.codes_width(x_codes, d["K"])), dtype=torch.uint8, device=dev)
+              for d, _ in data]
         sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in data]
         los = [torch.empty(M, dtype=torch.float32, device=dev) for _ in data]
         ys = [torch.empty((M, d["N"]), dtype=td, device=dev) for d, _ in data]
 
-        x_codes = clq.CLQ_CODES_E4M3_SPLIT if a_bits == 8 else clq.CLQ_CODES_E4M3
-        w_codes = clq.CLQ_CODES_E4M3_SPLIT if w_bits == 8 else clq.CLQ_CODES_E4M3
         sp = stream.cuda_stream
         dt = clq._dt(xsets[0][0])
 
@@ -554,7 +618,7 @@ def run_bits(args):
             K, N = d["K"], d["N"]
             # algorithmic bytes at this activation width: 16-bit input, packed
             # codes (bits / 8 B a code), the per-row scale (and minimum)
-            rq_bytes = M * (2.0 * K + (width / 2.0) * K + (8 if asym else 4))
+            rq_bytes = M * (2.0 * K + (a_bits / 8.0) * K + (8 if asym else 4))
             y = ys[i][:ERR_ROWS].double().cpu().numpy()
             err = float(((y - refs[i]) ** 2).sum() ** 0.5 / (refs[i] ** 2).sum() ** 0.5)
             per_layer.append({
@@ -671,14 +735,15 @@ def main():
         calib = torch.from_numpy(d["calib"]).to(td).to(dev)
         perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
         lay = clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b,
-                                             bias=d["bias"].to(dev))
+                                             bias=d["bias"].to(dev), w_codes=CODES[args.codes])
         layers.append((d["name"], d["K"], d["N"], lay))
         xs_host.append(d["X"])
         w_dense.append((d["W"].to(dev), d["bias"].to(dev)))  # fp16 cuBLAS comparator
     set_bytes = sum(x.numel() * 2 for x in xs_host)
     nsets = max(2, math.ceil(2 * L2_BYTES / set_bytes) + 1)
     xsets = [[x.to(dev) for x in xs_host] for _ in range(nsets)]
-    xq = [torch.empty((M, K), dtype=torch.uint8, device=dev) for (_, K, _, _) in layers]
+    xq = [torch.empty((M, clq.codes_width(lay.act_codes, K)), dtype=torch.uint8, device=dev)
+          for (_, K, _, lay) in layers]
     sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in layers]
     ys = [torch.empty((M, N), dtype=td, device=dev) for (_, _, N, _) in layers]
     wss = [clq.fused_workspace(M, K, dev) for (_, K, _, _) in layers]
@@ -699,23 +764,23 @@ def main():
             if fused:
                 st = clq.clq_fused_linear(xs[i].data_ptr(), clq._dt(xs[i]), M, K, K,
                                           lay.perm.data_ptr(), b, lay.We.data_ptr(),
-                                          clq.CLQ_CODES_E4M3, lay.s_w.data_ptr(),
+                                          lay.w_codes, lay.s_w.data_ptr(),
                                           lay.bias.data_ptr(), N, ys[i].data_ptr(),
                                           wss[i].data_ptr(), wss[i].numel(), sp_)
                 if st:
                     raise clq.ClqError(st, "clq_fused_linear")
             else:
                 st = clq.clq_rotate_quant_act(xs[i].data_ptr(), clq._dt(xs[i]), M, K, K,
-                                              lay.perm.data_ptr(), b, clq.CLQ_CODES_E4M3,
+                                              lay.perm.data_ptr(), b, lay.act_codes,
                                               xq[i].data_ptr(), sx[i].data_ptr(), None, sp_)
                 if st:
                     raise clq.ClqError(st, "clq_rotate_quant_act")
                 if ev is not None:
                     ev[4 * i + 1].record(stream)
                     ev[4 * i + 2].record(stream)
-                st = clq.clq_w4a4_linear(xq[i].data_ptr(), clq.CLQ_CODES_E4M3,
+                st = clq.clq_w4a4_linear(xq[i].data_ptr(), lay.act_codes,
                                          sx[i].data_ptr(), lay.We.data_ptr(),
-                                         clq.CLQ_CODES_E4M3,
+                                         lay.w_codes,
                                          lay.s_w.data_ptr(), lay.bias.data_ptr(), M, N, K, b,
                                          clq._dt(ys[i]), ys[i].data_ptr(), None, sp_)
                 if st:
@@ -782,6 +847,28 @@ def main():
     if world > 1:
         dist.barrier()
     total_ms = t_start.elapsed_time(t_end)
+    # Steady state: the same K steps repeated until at least 200 ms have run
+    # (at least 3 repeats), events around each repeat; the median per-step
+    # time of the repeats is reported beside the value.
+    reps = max(3, int(math.ceil(200.0 / max(total_ms, 1e-3))))
+    rep_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+    torch.cuda.synchronize()
+    for a_ev, z_ev in rep_ev:
+        a_ev.record(stream)
+        if graph is not None:
+            graph.replay()
+        else:
+            for k in range(args.steps):
+                step(k)
+        z_ev.record(stream)
+    torch.cuda.synchronize()
+    rep_ms = [a_ev.elapsed_time(z_ev) for a_ev, z_ev in rep_ev]
+    steady = {"repeats": reps, "steps_per_repeat": args.steps,
+              "region_ms": round(float(np.sum(rep_ms)), 2),
+              "ms_per_step_median": round(float(np.median(rep_ms)) / args.steps, 5),
+              "ms_per_step_min": round(float(np.min(rep_ms)) / args.steps, 5),
+              "ms_per_step_max": round(float(np.max(rep_ms)) / args.steps, 5)}
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4 * nlay)]
            for _ in range(args.steps)]
     torch.cuda.synchronize()
@@ -836,7 +923,7 @@ def main():
             def f(k, s_ptr):
                 x = xsets[k % nsets][i]
                 st = clq.clq_rotate_quant_act(x.data_ptr(), clq._dt(x), M, K, K,
-                                              lay.perm.data_ptr(), b, clq.CLQ_CODES_E4M3,
+                                              lay.perm.data_ptr(), b, lay.act_codes,
                                               xq[i].data_ptr(), sx[i].data_ptr(), None,
                                               sp if s_ptr is None else s_ptr)
                 if st:
@@ -847,9 +934,9 @@ def main():
             _, K, N, lay = layers[i]
 
             def f(k, s_ptr):
-                st = clq.clq_w4a4_linear(xq[i].data_ptr(), clq.CLQ_CODES_E4M3,
+                st = clq.clq_w4a4_linear(xq[i].data_ptr(), lay.act_codes,
                                          sx[i].data_ptr(), lay.We.data_ptr(),
-                                         clq.CLQ_CODES_E4M3, lay.s_w.data_ptr(),
+                                         lay.w_codes, lay.s_w.data_ptr(),
                                          lay.bias.data_ptr(), M, N, K, b,
                                          clq._dt(ys[i]), ys[i].data_ptr(), None,
                                          sp if s_ptr is None else s_ptr)
@@ -908,7 +995,8 @@ def main():
     gemm_kernel = "fused_linear" if args.fused else "w4a4_gemm"
     achieved = gemm_flops / gm_total_s / 1e12
     rq_bytes_all = sum(rq_algorithmic_bytes(M, K) for K in K_list)
-    rq_layout_all = sum(rq_layout_bytes(M, K, ACT_CODE_BYTES) for K in K_list)
+    rq_layout_all = sum(rq_layout_bytes(M, K, clq.codes_width(lay.act_codes, K) / K)
+                        for (_, K, _, lay) in layers)
     roofline = {"kernel": gemm_kernel, "bound": "tensor", "achieved": round(achieved, 1),
                 "peak": fp8_peak, "unit": "TFLOP/s", "frac": round(achieved / fp8_peak, 4),
                 "frac_of_measured_tcgen05_e4m3": round(achieved / measured["tcgen05_e4m3_tflops"], 4),
@@ -919,14 +1007,25 @@ def main():
         ach_b2b = gemm_flops / (sum(gm_b2b) * 1e-3) / 1e12
         roofline["achieved_back_to_back"] = round(ach_b2b, 1)
         roofline["frac_back_to_back"] = round(ach_b2b / fp8_peak, 4)
+    lay_codes = "e2m3" if layers[0][3].w_codes == clq.CLQ_CODES_E2M3 else "e4m3"
+    mainloop = measured.get("mainloop_%s_tflops" % lay_codes)
+    if mainloop:
+        roofline["mainloop_tflops"] = mainloop
+        roofline["frac_of_mainloop"] = round(achieved / mainloop, 4)
+        roofline["mainloop_note"] = ("clq_peak_operand_stream: the GEMM's TMA + MMA loop on "
+                                     "128 x 256 tiles of L2-resident %s codes, no epilogue, "
+                                     "this run" % lay_codes)
     if not args.fused:
         sm_mhz = (clocks or {}).get("sm_mhz") or 2070.0
         sms = torch.cuda.get_device_properties(dev).multi_processor_count
-        bound = gemm_intake_bound(M, list(zip(K_list, N_list)), sms, sm_mhz)
+        fill = measured["operand_stream_%s_smem_gbs" % lay_codes] * 1e9 / sms / (sm_mhz * 1e6)
+        bound = gemm_intake_bound(M, list(zip(K_list, N_list)), sms, sm_mhz, fill)
         roofline["intake_bound"] = {
             "tflops": round(bound, 1), "frac": round(achieved / bound, 4),
-            "model": "per-SM L2 intake %.0f B/clk (measured) at the median SM clock, output "
-                     "writes on the same port, the launcher's tiles" % SM_INTAKE_BYTES_PER_CLK}
+            "bytes_per_clk_per_sm": round(fill, 2),
+            "model": "TMA fill of shared memory per SM measured in this run "
+                     "(clq_peak_operand_stream, no MMA) at the median SM clock, output "
+                     "writes through the same engine, the launcher's tiles"}
     rq_roof = None
     if not args.fused:
         rq_ach = rq_bytes_all / rq_total_s / 1e9
@@ -981,7 +1080,11 @@ def main():
             "metric": METRIC, "value": round(value, 2), "unit": "TOPS",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3-int4/f32",
+            "steady_state": dict(steady, value_median=round(
+                ops_step * world / (steady["ms_per_step_median"] * 1e-3) / 1e12, 2)),
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": "int4 codes on %s tcgen05 operands, f32 accumulate" % (
+                "e2m3" if layers[0][3].act_codes == clq.CLQ_CODES_E2M3 else "e4m3"),
             "data": "synthetic (seeded Philox, DiT-shaped; no model weights)",
             "config": config_dict(cfg, args), "roofline": roofline,
             "roofline_rotate_quant": rq_roof, "per_layer": per_layer,

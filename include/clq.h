@@ -71,6 +71,8 @@ typedef int32_t clq_status;
 #define CLQ_ERR_DEVICE_INDEX 7 /* perm held an index outside [0, K)        */
 #define CLQ_ERR_SCRATCH_LIMIT 8 /* problem needs more than the static     */
                                 /* scratch of clq_fused_linear_noalloc     */
+#define CLQ_ERR_DEVICE_CODE 9  /* a code array held a value outside the   */
+                               /* INT4 range [-7, 7] (clq_convert_codes)   */
 
 typedef int32_t clq_dtype;
 #define CLQ_F16 0
@@ -88,8 +90,23 @@ typedef int32_t clq_dtype;
  *                         tensor-core GEMM loads with TMA directly, without
  *                         expanding nibbles in every CTA.  A zero code may
  *                         be written as either E4M3 zero (0x00 or 0x80).
- * The codes are the same INT4 values in both layouts and every call gives
- * identical results for either.  The 8-bit layout (the W4A8 and W8A8 bit
+ *  CLQ_CODES_E2M3         [rows][3K/4] bytes: each group of 16 consecutive
+ *                         codes is one little-endian 96-bit field (12
+ *                         bytes), code i of the group in bits 6i .. 6i + 5
+ *                         holding the code's exact E2M3 encoding (sign bit
+ *                         5, two exponent bits with bias 1, three mantissa
+ *                         bits: 0..7 are 0x00, 0x08, 0x10, 0x14, 0x18, 0x1A,
+ *                         0x1C, 0x1E; every integer in [-7, 7] is an E2M3
+ *                         value).  The tensor-core GEMM's tensor maps pad
+ *                         each 12-byte group to 16 bytes on the way into
+ *                         shared memory, the layout 6-bit MMA operands take,
+ *                         so this execution layout needs 3/4 of E4M3's
+ *                         bytes.  Requires K % 128 == 0 and 32-byte aligned
+ *                         arrays.  A zero code may be written as either E2M3
+ *                         zero (0x00 or 0x20).  The GEMM takes it for both
+ *                         operands together.
+ * The codes are the same INT4 values in every layout and every call gives
+ * identical results for any of them.  The 8-bit layout (the W4A8 and W8A8 bit
  * settings of Sec. 4.1; codes q in [-127, 127], s = r / 127):
  *  CLQ_CODES_E4M3_SPLIT   [rows][2][K] bytes: for each row, plane 0 holds the
  *                         E4M3 encoding of 16 h and plane 1 that of l, where
@@ -102,6 +119,7 @@ typedef int32_t clq_codes;
 #define CLQ_CODES_INT4_PACKED 0
 #define CLQ_CODES_E4M3 1
 #define CLQ_CODES_E4M3_SPLIT 2
+#define CLQ_CODES_E2M3 3
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char* clq_status_string(clq_status status);
@@ -180,7 +198,8 @@ clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N,
 
 /*
  * clq_prepare_weights in any code layout (`w_codes`): 4-bit codes (qmax 7)
- * for CLQ_CODES_INT4_PACKED ([N][K/2]) or CLQ_CODES_E4M3 ([N][K]), 8-bit
+ * for CLQ_CODES_INT4_PACKED ([N][K/2]), CLQ_CODES_E4M3 ([N][K]) or
+ * CLQ_CODES_E2M3 ([N][3K/4], K % 128 == 0, Wq 32-byte aligned), 8-bit
  * codes (qmax 127, the W8A8 setting) for CLQ_CODES_E4M3_SPLIT ([N][2][K]).
  * The clip bound caps max_k |W~[n][k]| as above.
  */
@@ -198,7 +217,8 @@ clq_status clq_prepare_weights_codes(const void* W, clq_dtype dtype, int32_t N,
  * qmax = 7 for the 4-bit layouts and 127 for CLQ_CODES_E4M3_SPLIT.
  * One HBM pass over X.  X: device [M][ldx] of `dtype`.  perm: device int32
  * [K].  Xq: device uint8 codes in layout `x_codes` ([M][K/2] packed,
- * [M][K] E4M3 or [M][2][K] split).  s_x: device fp32 [M].  x_rot_dbg:
+ * [M][K] E4M3, [M][3K/4] E2M3 with K % 128 == 0 and Xq 32-byte aligned, or
+ * [M][2][K] split).  s_x: device fp32 [M].  x_rot_dbg:
  * device fp32 [M][K] or NULL (receives X~).
  */
 clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M,
@@ -218,14 +238,33 @@ clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K,
                               uint8_t* We, void* stream);
 
 /*
+ * A code array of `rows` x K INT4 codes from one 4-bit layout to another
+ * (CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3, CLQ_CODES_E2M3, in any direction,
+ * the same layout included).  The codes are unchanged; this is how the
+ * storage format (packed nibbles) and the execution layouts are turned into
+ * one another, offline.  src: device, [rows][width(src_codes)] bytes; dst:
+ * device, [rows][width(dst_codes)] bytes, not overlapping src; width is K/2,
+ * K or 3K/4.  Requires rows >= 0, K % 32 == 0, K <= 16384 (K % 128 == 0 when
+ * either side is E2M3); arrays 16-byte aligned (32 for E2M3).  A source code
+ * outside [-7, 7] (packed -8, or an E4M3 / E2M3 field that holds no integer
+ * in that range) is written as 0 and reported as CLQ_ERR_DEVICE_CODE in the
+ * device status word.
+ */
+clq_status clq_convert_codes(const uint8_t* src, clq_codes src_codes,
+                             uint8_t* dst, clq_codes dst_codes, int32_t rows,
+                             int32_t K, void* stream);
+
+/*
  * INT4 x INT4 product with the dequant + bias epilogue:
  * Y[i][n] = out_dtype(acc[i][n] * s_x[i] * s_w[n] / b + bias[n]).
- * Xq: device activation codes in layout `x_codes` ([M][K/2] or [M][K]);
- * s_x: device fp32 [M]; W: device weight codes in layout `w_codes`
- * ([N][K/2] or [N][K]); s_w: device fp32 [N]; bias: device [N] of
- * `out_dtype` or NULL; Y: device [M][N] of `out_dtype`.  acc_dbg: device
- * int32 [M][N] or NULL; when given it receives the exact integer
- * accumulators.  All four layout combinations give identical results.
+ * Xq: device activation codes in layout `x_codes` ([M][K/2], [M][K] or
+ * [M][3K/4]); s_x: device fp32 [M]; W: device weight codes in layout
+ * `w_codes` ([N][K/2], [N][K] or [N][3K/4]); s_w: device fp32 [N]; bias:
+ * device [N] of `out_dtype` or NULL; Y: device [M][N] of `out_dtype`.
+ * acc_dbg: device int32 [M][N] or NULL; when given it receives the exact
+ * integer accumulators.  Packed and E4M3 operands combine in all four ways;
+ * CLQ_CODES_E2M3 goes with CLQ_CODES_E2M3 only (other pairings with it return
+ * CLQ_ERR_UNSUPPORTED).  Every combination gives identical results.
  */
 clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes,
                            const float* s_x, const uint8_t* W,
@@ -241,12 +280,11 @@ clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes,
  *  W4A4  x_codes and w_codes 4-bit layouts (as clq_w4a4_linear);
  *  W4A8  x_codes CLQ_CODES_E4M3_SPLIT, w_codes CLQ_CODES_E4M3;
  *  W8A8  both CLQ_CODES_E4M3_SPLIT.
- * Other combinations return CLQ_ERR_UNSUPPORTED.  W4A4 and W4A8
- * accumulators are exact integers for every K <= 16384; W8A8 accumulators
- * are exact while every partial sum stays below 2^24 in magnitude (always
- * for K <= 896) and carry fp32 rounding beyond.  acc_dbg (int32 [M][N] or
- * NULL) receives the accumulators rounded to integers.  Arguments otherwise
- * as for clq_w4a4_linear.
+ * Other combinations return CLQ_ERR_UNSUPPORTED.  The accumulators are
+ * exact integers for every K <= 16384 at every setting (W8A8 keeps its plane
+ * products in three accumulators and adds them as integers).  acc_dbg (int32
+ * [M][N] or NULL) receives them.  Arguments otherwise as for
+ * clq_w4a4_linear.
  */
 clq_status clq_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x,
                       const uint8_t* W, clq_codes w_codes, const float* s_w,
@@ -353,8 +391,10 @@ size_t clq_fused_linear_workspace_size(int32_t M, int32_t K);
  * its rows, then turns to the GEMM.  Same
  * arithmetic and results as clq_rotate_quant_act followed by
  * clq_w4a4_linear.  X: device [M][ldx] of `dtype`; Y: device [M][N] of
- * `dtype`; bias: device [N] of `dtype` or NULL; W / w_codes as for
- * clq_w4a4_linear; workspace: device, 256-byte aligned, at least
+ * `dtype`; bias: device [N] of `dtype` or NULL; W / w_codes: weights in any
+ * 4-bit layout, as for clq_w4a4_linear (the activation codes in the
+ * workspace then take E2M3 beside E2M3 weights, else E4M3); workspace:
+ * device, 256-byte aligned, at least
  * clq_fused_linear_workspace_size(M, K) bytes, owned by the caller and
  * overwritten by the call.
  */
@@ -425,10 +465,24 @@ clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream);
  *   (1 .. 1e6) rounds of 4 independent MMAs per warp, 32 warps per SM.
  * clq_peak_hbm_read: reads `bytes` (a multiple of 16, buf 16-byte aligned)
  *   once; *ops = bytes.
+ * clq_peak_operand_stream: the W4A4 GEMM's main loop without its epilogue,
+ *   one CTA per SM walking `tiles` (1 .. 1e5) 128 x 256 output tiles of
+ *   K / 128 steps: a TMA producer fills a ring of four stages with the
+ *   GEMM's operand boxes (A 128 rows, B 256 rows, 128 codes a row, 48 KB of
+ *   shared memory a step in either layout) taken from `buf`, a device code
+ *   array of `rows` x K codes in layout `codes` (CLQ_CODES_E4M3 or
+ *   CLQ_CODES_E2M3; rows a multiple of 256, K a multiple of 128, buf 32-byte
+ *   aligned).  mma = 0: each stage is released as soon as it lands, *ops =
+ *   the shared-memory bytes filled (the rate an SM takes operands in);
+ *   mma = 1: the GEMM's four 128 x 256 x 32 MMAs run on each stage, *ops =
+ *   the multiply-accumulates.
  */
 clq_status clq_peak_tcgen05_e4m3(int32_t iters, int64_t* ops, void* stream);
 clq_status clq_peak_mma_sync(int32_t kind, int32_t iters, int64_t* ops, void* stream);
 clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void* stream);
+clq_status clq_peak_operand_stream(const uint8_t* buf, int32_t rows, int32_t K,
+                                   clq_codes codes, int32_t mma, int32_t tiles,
+                                   int64_t* ops, void* stream);
 
 #ifdef __cplusplus
 }

@@ -20,11 +20,11 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libclq.so")
 
 CLQ_F16, CLQ_BF16 = 0, 1
-CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3, CLQ_CODES_E4M3_SPLIT = 0, 1, 2
+CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3, CLQ_CODES_E4M3_SPLIT, CLQ_CODES_E2M3 = 0, 1, 2, 3
 STATUS = {0: "CLQ_OK", 1: "CLQ_ERR_INVALID_ARG", 2: "CLQ_ERR_SHAPE",
           3: "CLQ_ERR_ALIGN", 4: "CLQ_ERR_UNSUPPORTED", 5: "CLQ_ERR_CUDA",
           6: "CLQ_ERR_TIMEOUT", 7: "CLQ_ERR_DEVICE_INDEX",
-          8: "CLQ_ERR_SCRATCH_LIMIT"}
+          8: "CLQ_ERR_SCRATCH_LIMIT", 9: "CLQ_ERR_DEVICE_CODE"}
 EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_build_permutation", "clq_prepare_weights",
            "clq_rotate_quant_act", "clq_expand_weights", "clq_w4a4_linear",
@@ -36,7 +36,7 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_prepare_weights_codes", "clq_linear",
            "clq_rotate_quant_act_asym", "clq_weight_code_sums",
            "clq_linear_asym", "clq_clip_search_workspace_size",
-           "clq_clip_search")
+           "clq_clip_search", "clq_convert_codes", "clq_peak_operand_stream")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -53,6 +53,7 @@ _SIGS = {
     "clq_rotate_quant_act": (_I, [_P, _I, _I, _I, _I, _P, _I, _I, _P, _P, _P,
                                   _P]),
     "clq_expand_weights": (_I, [_P, _I, _I, _P, _P]),
+    "clq_convert_codes": (_I, [_P, _I, _P, _I, _I, _I, _P]),
     "clq_w4a4_linear": (_I, [_P, _I, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I,
                              _P, _P, _P]),
     "clq_fused_linear_workspace_size": (_Z, [_I, _I]),
@@ -65,6 +66,7 @@ _SIGS = {
     "clq_peak_tcgen05_e4m3": (_I, [_I, _P, _P]),
     "clq_peak_mma_sync": (_I, [_I, _I, _P, _P]),
     "clq_peak_hbm_read": (_I, [_P, ctypes.c_uint64, _P, _P]),
+    "clq_peak_operand_stream": (_I, [_P, _I, _I, _I, _I, _I, _P, _P]),
     "clq_prepare_weights_codes": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I,
                                        _P, _P, _P, _P]),
     "clq_linear": (_I, [_P, _I, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P,
@@ -179,6 +181,10 @@ def clq_expand_weights(Wq, N, K, We, stream):
     return load().clq_expand_weights(Wq, N, K, We, stream)
 
 
+def clq_convert_codes(src, src_codes, dst, dst_codes, rows, K, stream):
+    return load().clq_convert_codes(src, src_codes, dst, dst_codes, rows, K, stream)
+
+
 def clq_w4a4_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M, N, K, b,
                     out_dtype, Y, acc_dbg, stream):
     return load().clq_w4a4_linear(Xq, x_codes, s_x, W, w_codes, s_w, bias, M,
@@ -220,6 +226,10 @@ def clq_peak_tcgen05_e4m3(iters, ops, stream):
 
 def clq_peak_mma_sync(kind, iters, ops, stream):
     return load().clq_peak_mma_sync(kind, iters, ops, stream)
+
+
+def clq_peak_operand_stream(buf, rows, K, codes, mma, tiles, ops, stream):
+    return load().clq_peak_operand_stream(buf, rows, K, codes, mma, tiles, ops, stream)
 
 
 def clq_peak_hbm_read(buf, nbytes, ops, stream):
@@ -300,7 +310,17 @@ def build_permutation(scores):
 def codes_width(codes, K):
     """Bytes per row of K codes in layout `codes`."""
     return {CLQ_CODES_INT4_PACKED: K // 2, CLQ_CODES_E4M3: K,
-            CLQ_CODES_E4M3_SPLIT: 2 * K}[codes]
+            CLQ_CODES_E4M3_SPLIT: 2 * K, CLQ_CODES_E2M3: K // 4 * 3}[codes]
+
+
+def exec_layout(K):
+    """The default 4-bit execution layout for K input channels: E4M3, one
+    byte a code, the layout the W4A4 step runs fastest with (measured: the
+    GEMM's TMA fills shared memory with the same padded bytes for E2M3, and
+    its 16-code groups cost the rotate-quant store extra work).  E2M3
+    (0.75 B a code, K % 128 == 0) is the layout to pass as ``w_codes`` when
+    resident weight memory matters more."""
+    return CLQ_CODES_E4M3
 
 
 def prepare_weights(W, perm, b, clip=None, with_rot=False, stream=None,
@@ -414,8 +434,24 @@ def codes_layout(t, K):
         return CLQ_CODES_INT4_PACKED
     if t.shape[1] == 2 * K:
         return CLQ_CODES_E4M3_SPLIT
-    raise ValueError("codes must be [rows, K/2] packed, [rows, K] E4M3 or "
-                     "[rows, 2K] split")
+    if 4 * t.shape[1] == 3 * K:
+        return CLQ_CODES_E2M3
+    raise ValueError("codes must be [rows, K/2] packed, [rows, K] E4M3, "
+                     "[rows, 3K/4] E2M3 or [rows, 2K] split")
+
+
+def convert_codes(src, K, dst_codes, dst=None, stream=None):
+    """A 4-bit code array in any layout -> the same codes in layout
+    `dst_codes` (uint8 [rows, width])."""
+    rows = src.shape[0]
+    width = codes_width(dst_codes, K)
+    if dst is None:
+        dst = torch.empty((rows, width), dtype=torch.uint8, device=src.device)
+    else:
+        _buffer(dst, (rows, width), torch.uint8, src.device, "dst")
+    _check(clq_convert_codes(_ptr(src), codes_layout(src, K), _ptr(dst), dst_codes,
+                             rows, K, _stream(stream)), "clq_convert_codes")
+    return dst
 
 
 def w4a4_linear(Xq, s_x, W, s_w, b, K, bias=None, out_dtype=torch.float16,
@@ -520,7 +556,7 @@ def fused_workspace(M, K, device):
 def fused_linear(X, perm, b, W, s_w, bias=None, Y=None, workspace=None,
                  stream=None):
     """X [M, K] -> Y [M, N] in X's dtype, rotate-quant and GEMM in one
-    kernel.  W is packed [N, K/2] or E4M3 [N, K]."""
+    kernel.  W is packed [N, K/2], E4M3 [N, K] or E2M3 [N, 3K/4]."""
     _row_major(X, "X")
     M, K = X.shape
     N = W.shape[0]
@@ -551,38 +587,79 @@ def selftest_bounded_wait(timeout_ns=1000000, stream=None):
 
 
 class PreparedLinear:
-    """A quantized linear layer: the prepared-weight package (Wq, s_w, perm,
-    b, bias) of Sec. 3.3, where the swap vector is the only stored part of G.
+    """A quantized linear layer: the prepared-weight package (codes, s_w,
+    perm, b, bias) of Sec. 3.3, where the swap vector is the only stored part
+    of G.
 
-    At W4A4 and W4A8, Wq holds the packed INT4 codes (the storage format,
-    4 bits per weight) and We the same codes in the E4M3 execution layout the
-    GEMM loads directly.  At W8A8, Wq holds the 8-bit codes as split planes
-    ([N, 2K], which is also the execution layout).  Activation codes are
-    produced in an execution layout too (they are transient): E4M3 for
-    4-bit, split planes for 8-bit activations (a_bits).
-    ``state_dict()`` keeps only the storage codes; ``from_state_dict()``
-    expands them again.  Calling the object runs the separate rotate-quant
-    and GEMM kernels (``fused=False``) or, at W4A4, the fused kernel.
+    Only one copy of the weight codes is resident on the device, ``We``, in
+    the execution layout the GEMM loads directly (``w_codes``): at W4A4 E4M3
+    (1 B a weight) by default, or E2M3 (12 bytes per 16 codes, 0.75 B a
+    weight, K % 128 == 0) on request; at W4A8 E4M3 (the 8-bit activation
+    planes pair with E4M3 weights); at W8A8 the split 8-bit planes.  ``Wq`` gives the
+    storage format (packed INT4 nibbles, 4 bits a weight, the format the
+    paper's memory figure counts; the split planes at W8A8), converted from
+    ``We`` on demand.  Activation codes are produced in an execution layout
+    too (they are transient): the 4-bit layout of the weights, or split
+    planes for 8-bit activations (a_bits).  ``state_dict()`` keeps the
+    storage codes; ``from_state_dict()`` converts them back.  Calling the
+    object runs the separate rotate-quant and GEMM kernels (``fused=False``)
+    or, at W4A4, the fused kernel.
     """
 
-    def __init__(self, Wq, s_w, perm, b, bias=None, We=None, a_bits=4):
-        self.Wq, self.s_w, self.perm, self.b, self.bias = Wq, s_w, perm, b, bias
+    def __init__(self, Wq, s_w, perm, b, bias=None, We=None, a_bits=4, w_codes=None):
+        """Wq: weight codes in any layout (packed storage codes, an
+        execution layout, or split planes for 8-bit weights); they are
+        converted to the execution layout unless ``We`` already holds it."""
+        self.s_w, self.perm, self.b, self.bias = s_w, perm, b, bias
         K = perm.numel()
-        self.w_bits = 8 if Wq.shape[1] == 2 * K else 4
+        self.K = K
+        src = We if We is not None else Wq
+        self.w_bits = 8 if codes_layout(src, K) == CLQ_CODES_E4M3_SPLIT else 4
         if a_bits not in (4, 8) or (self.w_bits == 8 and a_bits != 8):
             raise ValueError("bit settings are W4A4, W4A8 and W8A8")
         self.a_bits = a_bits
         if self.w_bits == 8:
-            self.We = Wq
+            self.w_codes = CLQ_CODES_E4M3_SPLIT
+        elif w_codes is not None:
+            self.w_codes = w_codes
         else:
-            self.We = expand_weights(Wq) if We is None else We
+            self.w_codes = exec_layout(K) if a_bits == 4 else CLQ_CODES_E4M3
+        if codes_layout(src, K) == self.w_codes:
+            self.We = src
+        else:
+            self.We = convert_codes(src, K, self.w_codes)
+
+    @property
+    def Wq(self):
+        """Storage codes: packed INT4 nibbles [N, K/2] (4-bit weights), or the
+        split planes [N, 2K] (8-bit weights), converted from ``We``."""
+        if self.w_bits == 8:
+            return self.We
+        if self.w_codes == CLQ_CODES_INT4_PACKED:
+            return self.We
+        return convert_codes(self.We, self.K, CLQ_CODES_INT4_PACKED)
+
+    def resident_bytes(self):
+        """Device bytes the layer keeps: weight codes, scales, swap vector,
+        bias."""
+        n = self.We.numel() + self.s_w.numel() * 4 + self.perm.numel() * 4
+        if self.bias is not None:
+            n += self.bias.numel() * self.bias.element_size()
+        return n
 
     @classmethod
-    def from_weight(cls, W, perm, b, bias=None, clip=None, a_bits=4, w_bits=4):
+    def from_weight(cls, W, perm, b, bias=None, clip=None, a_bits=4, w_bits=4,
+                    w_codes=None):
         perm = perm.to(W.device, torch.int32).contiguous()
-        codes = CLQ_CODES_E4M3_SPLIT if w_bits == 8 else CLQ_CODES_INT4_PACKED
-        Wq, s_w = prepare_weights(W.contiguous(), perm, b, clip, codes=codes)
-        return cls(Wq, s_w, perm, b, bias, a_bits=a_bits)
+        K = W.shape[1]
+        if w_bits == 8:
+            codes = CLQ_CODES_E4M3_SPLIT
+        elif w_codes is not None:
+            codes = w_codes
+        else:
+            codes = exec_layout(K) if a_bits == 4 else CLQ_CODES_E4M3
+        We, s_w = prepare_weights(W.contiguous(), perm, b, clip, codes=codes)
+        return cls(None, s_w, perm, b, bias, We=We, a_bits=a_bits, w_codes=codes)
 
     @classmethod
     def calibrate(cls, W, calib, b, bias=None, metric="absmax", clip_grid=None,
@@ -614,6 +691,15 @@ class PreparedLinear:
                                 w_bits=w_bits)
         return layer, dict(scores=scores, perm=perm, clip=clip, errors=errors, best=best)
 
+    @property
+    def act_codes(self):
+        """Layout of the activation codes the separate path writes: split
+        planes for 8-bit activations, else the 4-bit layout of the weights
+        (E2M3 with E2M3, E4M3 otherwise)."""
+        if self.a_bits == 8:
+            return CLQ_CODES_E4M3_SPLIT
+        return CLQ_CODES_E2M3 if self.w_codes == CLQ_CODES_E2M3 else CLQ_CODES_E4M3
+
     def state_dict(self):
         d = dict(Wq=self.Wq, s_w=self.s_w, perm=self.perm,
                  b=torch.tensor(self.b), a_bits=torch.tensor(self.a_bits))
@@ -638,7 +724,7 @@ class PreparedLinear:
                 raise ValueError("the fused kernel runs W4A4 only")
             return fused_linear(X, self.perm, self.b, self.We, self.s_w,
                                 self.bias, Y=Y, workspace=workspace, stream=stream)
-        codes = CLQ_CODES_E4M3_SPLIT if self.a_bits == 8 else CLQ_CODES_E4M3
+        codes = self.act_codes
         Xq, s_x = rotate_quant_act(X, self.perm, self.b, codes,
                                    Xq=Xq, s_x=s_x, stream=stream)
         if self.a_bits == 4:
@@ -667,7 +753,7 @@ class HostPipeline:
         dev = torch.device(device)
         self.xd = [torch.empty((M, K), dtype=dtype, device=dev) for (_, M, K, _) in layers]
         self.yd = [torch.empty((M, N), dtype=dtype, device=dev) for (_, M, _, N) in layers]
-        self.xq = [torch.empty((M, K * (2 if lay.a_bits == 8 else 1)), dtype=torch.uint8,
+        self.xq = [torch.empty((M, codes_width(lay.act_codes, K)), dtype=torch.uint8,
                                device=dev)
                    for (lay, M, K, _) in layers]
         self.sx = [torch.empty(M, dtype=torch.float32, device=dev) for (_, M, _, _) in layers]
@@ -716,7 +802,9 @@ def measure_peaks(stream=None, reps=5):
     """Measured peak rates on the current device (best of `reps`, CUDA events
     on `stream` around each microbenchmark launch): tcgen05 E4M3 and
     mma.sync s8 / s4 / e4m3 in TFLOP/s (2 ops per multiply-accumulate) and
-    the HBM read bandwidth in GB/s."""
+    the HBM read bandwidth in GB/s; the GEMM's operand stream into shared
+    memory (GB/s of shared-memory bytes, all SMs, operands L2-resident) and
+    its main loop with the MMAs (TFLOP/s), for E4M3 and E2M3 operands."""
     s = torch.cuda.current_stream() if stream is None else stream
     sp = s.cuda_stream
     dev = torch.device("cuda", torch.cuda.current_device())
@@ -747,5 +835,16 @@ def measure_peaks(stream=None, reps=5):
     out["hbm_read_gbs"] = 1e-9 * timed(lambda: _check(
         clq_peak_hbm_read(buf.data_ptr(), buf.numel(), ctypes.byref(ops), sp),
         "clq_peak_hbm_read"))
+    # operands of a 4096 x 1152 code array (L2-resident, like the GEMM's)
+    rows, K, tiles = 4096, 1152, 48
+    for codes, tag in ((CLQ_CODES_E4M3, "e4m3"), (CLQ_CODES_E2M3, "e2m3")):
+        for mma in (0, 1):
+            r = 1e-9 * timed(lambda: _check(
+                clq_peak_operand_stream(buf.data_ptr(), rows, K, codes, mma, tiles,
+                                        ctypes.byref(ops), sp), "clq_peak_operand_stream"))
+            if mma:
+                out["mainloop_%s_tflops" % tag] = 2e-3 * r
+            else:
+                out["operand_stream_%s_smem_gbs" % tag] = r
     del buf
     return {k: round(v, 1) for k, v in out.items()}

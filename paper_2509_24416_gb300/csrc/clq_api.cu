@@ -71,7 +71,18 @@ clq_status check_k_b(int K, int b) {
 bool valid_dtype(int d) { return d == CLQ_F16 || d == CLQ_BF16; }
 
 // 4-bit layouts (W4A4 entry points) and every layout (rotate-quant, clq_linear).
-bool valid_codes(int f) { return f == CLQ_CODES_INT4_PACKED || f == CLQ_CODES_E4M3; }
+bool valid_codes(int f) {
+  return f == CLQ_CODES_INT4_PACKED || f == CLQ_CODES_E4M3 || f == CLQ_CODES_E2M3;
+}
+
+// Extra rules of the E2M3 layout: whole 128-code groups (the GEMM's tensor
+// maps take 128 codes a row per box) and 32-byte aligned arrays.
+clq_status check_e2m3(int codes, int K, const void* p) {
+  if (codes != CLQ_CODES_E2M3) return CLQ_OK;
+  if (K % 128 != 0) return CLQ_ERR_SHAPE;
+  if (p != nullptr && (reinterpret_cast<uintptr_t>(p) % 32) != 0) return CLQ_ERR_ALIGN;
+  return CLQ_OK;
+}
 bool valid_any_codes(int f) { return valid_codes(f) || f == CLQ_CODES_E4M3_SPLIT; }
 
 // Launch of the fused kernel on a workspace laid out as `ws` (validated).
@@ -111,8 +122,11 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
                                uint8_t* Q, float* S, float* rot, void* stream,
                                float* lo = nullptr) {
   if (!valid_dtype(dtype) || !valid_any_codes(codes) || M < 0) return CLQ_ERR_INVALID_ARG;
+  // centered asymmetric codes reach -8, which E2M3 does not hold
+  if (lo != nullptr && codes == CLQ_CODES_E2M3) return CLQ_ERR_UNSUPPORTED;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
+  if (codes == CLQ_CODES_E2M3 && K % 128 != 0) return CLQ_ERR_SHAPE;
   if (ld < K) return CLQ_ERR_SHAPE;
   if (ld % 8 != 0) return CLQ_ERR_ALIGN;
   if (M == 0) return CLQ_OK;
@@ -121,6 +135,8 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
       (rot != nullptr && !aligned(rot, 16)) || (clip != nullptr && !aligned(clip, 4)) ||
       (lo != nullptr && !aligned(lo, 4)))
     return CLQ_ERR_ALIGN;
+  st = check_e2m3(codes, K, Q);
+  if (st != CLQ_OK) return st;
   int32_t* status = nullptr;
   st = device_setup(&status);
   if (st != CLQ_OK) return st;
@@ -137,7 +153,10 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   a.lo = lo;
   a.status = status;
   a.logb = log2i(b);
-  a.e4m3 = codes == CLQ_CODES_E4M3 ? 1 : codes == CLQ_CODES_E4M3_SPLIT ? 2 : 0;
+  a.e4m3 = codes == CLQ_CODES_E4M3         ? 1
+           : codes == CLQ_CODES_E4M3_SPLIT ? 2
+           : codes == CLQ_CODES_E2M3       ? 3
+                                           : 0;
   return from_cuda(
       clq::launch_rotate_quant(a, dtype, log2i(b), static_cast<cudaStream_t>(stream)));
 }
@@ -156,8 +175,13 @@ clq_status linear_common(const uint8_t* Xq, int x_codes, const float* s_x, const
       !(x_codes == CLQ_CODES_E4M3_SPLIT &&
         (w_codes == CLQ_CODES_E4M3 || w_codes == CLQ_CODES_E4M3_SPLIT)))
     return CLQ_ERR_UNSUPPORTED;
+  // E2M3 operands pair with each other only, symmetric codes only.
+  if ((x_codes == CLQ_CODES_E2M3) != (w_codes == CLQ_CODES_E2M3) ||
+      (x_codes == CLQ_CODES_E2M3 && lo != nullptr))
+    return CLQ_ERR_UNSUPPORTED;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
+  if (x_codes == CLQ_CODES_E2M3 && K % 128 != 0) return CLQ_ERR_SHAPE;
   if (M == 0 || N == 0) return CLQ_OK;
   if (Xq == nullptr || s_x == nullptr || W == nullptr || s_w == nullptr || Y == nullptr)
     return CLQ_ERR_INVALID_ARG;
@@ -166,6 +190,8 @@ clq_status linear_common(const uint8_t* Xq, int x_codes, const float* s_x, const
       (acc_dbg != nullptr && !aligned(acc_dbg, 4)) || (lo != nullptr && !aligned(lo, 4)) ||
       (wsum != nullptr && !aligned(wsum, 4)))
     return CLQ_ERR_ALIGN;
+  if ((st = check_e2m3(x_codes, K, Xq)) != CLQ_OK || (st = check_e2m3(w_codes, K, W)) != CLQ_OK)
+    return st;
   int32_t* status = nullptr;
   st = device_setup(&status);
   if (st != CLQ_OK) return st;
@@ -239,6 +265,8 @@ const char* clq_status_string(clq_status s) {
     case CLQ_ERR_CUDA: return "CLQ_ERR_CUDA: a CUDA runtime call failed";
     case CLQ_ERR_TIMEOUT: return "CLQ_ERR_TIMEOUT: a bounded device-side wait ran out";
     case CLQ_ERR_DEVICE_INDEX: return "CLQ_ERR_DEVICE_INDEX: perm index outside [0, K)";
+    case CLQ_ERR_DEVICE_CODE:
+      return "CLQ_ERR_DEVICE_CODE: a code array held a value outside [-7, 7]";
     case CLQ_ERR_SCRATCH_LIMIT:
       return "CLQ_ERR_SCRATCH_LIMIT: M x K needs more than the static scratch of "
              "clq_fused_linear_noalloc";
@@ -246,7 +274,7 @@ const char* clq_status_string(clq_status s) {
   }
 }
 
-int32_t clq_version(void) { return 100; }
+int32_t clq_version(void) { return 101; }
 
 clq_status clq_build_permutation(const float* host_scores, int32_t K, int32_t* host_perm) {
   if (host_scores == nullptr || host_perm == nullptr || K < 1) return CLQ_ERR_INVALID_ARG;
@@ -340,6 +368,25 @@ clq_status clq_expand_weights(const uint8_t* Wq, int32_t N, int32_t K, uint8_t* 
   return from_cuda(clq::launch_expand_weights(Wq, N, K, We, static_cast<cudaStream_t>(stream)));
 }
 
+clq_status clq_convert_codes(const uint8_t* src, clq_codes src_codes, uint8_t* dst,
+                             clq_codes dst_codes, int32_t rows, int32_t K, void* stream) {
+  if (!valid_codes(src_codes) || !valid_codes(dst_codes) || rows < 0 || K < 0)
+    return CLQ_ERR_INVALID_ARG;
+  if (K < 32 || K > 16384 || K % 32 != 0) return CLQ_ERR_SHAPE;
+  if ((src_codes == CLQ_CODES_E2M3 || dst_codes == CLQ_CODES_E2M3) && K % 128 != 0)
+    return CLQ_ERR_SHAPE;
+  if (rows == 0) return CLQ_OK;
+  if (src == nullptr || dst == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (!aligned(src, 16) || !aligned(dst, 16)) return CLQ_ERR_ALIGN;
+  clq_status st = check_e2m3(src_codes, K, src);
+  if (st != CLQ_OK || (st = check_e2m3(dst_codes, K, dst)) != CLQ_OK) return st;
+  int32_t* status = nullptr;
+  st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  return from_cuda(clq::launch_convert_codes(src, src_codes, dst, dst_codes, rows, K, status,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
 clq_status clq_w4a4_linear(const uint8_t* Xq, clq_codes x_codes, const float* s_x,
                            const uint8_t* W, clq_codes w_codes, const float* s_w,
                            const void* bias, int32_t M, int32_t N, int32_t K, int32_t b,
@@ -374,11 +421,14 @@ clq_status clq_weight_code_sums(const uint8_t* W, clq_codes w_codes, int32_t N, 
                                 float* wsum, void* stream) {
   if (!valid_any_codes(w_codes) || N < 0) return CLQ_ERR_INVALID_ARG;
   if (K < 32 || K > 16384 || K % 32 != 0) return CLQ_ERR_SHAPE;
+  if (w_codes == CLQ_CODES_E2M3 && K % 128 != 0) return CLQ_ERR_SHAPE;
   if (N == 0) return CLQ_OK;
   if (W == nullptr || wsum == nullptr) return CLQ_ERR_INVALID_ARG;
   if (!aligned(W, 16) || !aligned(wsum, 4)) return CLQ_ERR_ALIGN;
+  clq_status st = check_e2m3(w_codes, K, W);
+  if (st != CLQ_OK) return st;
   int32_t* status = nullptr;
-  clq_status st = device_setup(&status);
+  st = device_setup(&status);
   if (st != CLQ_OK) return st;
   return from_cuda(
       clq::launch_code_sums(W, w_codes, N, K, wsum, static_cast<cudaStream_t>(stream)));
@@ -399,6 +449,7 @@ int32_t fused_linear_check(const void* X, int32_t dtype, int32_t M, int32_t K, i
     return CLQ_ERR_INVALID_ARG;
   clq_status st = check_k_b(K, b);
   if (st != CLQ_OK) return st;
+  if (w_codes == CLQ_CODES_E2M3 && K % 128 != 0) return CLQ_ERR_SHAPE;
   if (ldx < K) return CLQ_ERR_SHAPE;
   if (ldx % 8 != 0) return CLQ_ERR_ALIGN;
   if (M == 0 || N == 0) {
@@ -410,7 +461,7 @@ int32_t fused_linear_check(const void* X, int32_t dtype, int32_t M, int32_t K, i
   if (!aligned(X, 16) || !aligned(W, 16) || !aligned(Y, 16) || !aligned(perm, 4) ||
       !aligned(s_w, 4) || (bias != nullptr && !aligned(bias, 2)))
     return CLQ_ERR_ALIGN;
-  return CLQ_OK;
+  return check_e2m3(w_codes, K, W);
 }
 
 int32_t device_check() {
@@ -504,6 +555,26 @@ clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void
   if (st != CLQ_OK) return st;
   st = from_cuda(clq::launch_peak_hbm_read(buf, bytes, status, static_cast<cudaStream_t>(stream)));
   *ops = static_cast<int64_t>(bytes);
+  return st;
+}
+
+clq_status clq_peak_operand_stream(const uint8_t* buf, int32_t rows, int32_t K,
+                                   clq_codes codes, int32_t mma, int32_t tiles, int64_t* ops,
+                                   void* stream) {
+  if (ops == nullptr || buf == nullptr || (codes != CLQ_CODES_E4M3 && codes != CLQ_CODES_E2M3) ||
+      (mma != 0 && mma != 1) || tiles < 1 || tiles > 100000)
+    return CLQ_ERR_INVALID_ARG;
+  if (rows < 256 || rows % 256 != 0 || K < 128 || K > 16384 || K % 128 != 0)
+    return CLQ_ERR_SHAPE;
+  if (reinterpret_cast<uintptr_t>(buf) % 32 != 0) return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  long long bytes = 0, macs = 0;
+  st = from_cuda(clq::launch_peak_operand_stream(buf, rows, K, codes, mma, tiles, status,
+                                                 static_cast<cudaStream_t>(stream), &bytes,
+                                                 &macs));
+  *ops = mma ? macs : bytes;
   return st;
 }
 

@@ -214,13 +214,24 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t smem_byte_addr) {
   return d;
 }
 
-// Instruction descriptor: E4M3 A and B, F32 accumulate, both K-major.
-__host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t M, uint32_t N) {
+// Operand formats of kind::f8f6f4 in the instruction descriptor.
+constexpr uint32_t kFmtE4M3 = 0;
+constexpr uint32_t kFmtE2M3 = 3;
+
+// Instruction descriptor of kind::f8f6f4: A and B formats, F32 accumulate,
+// both K-major.
+__host__ __device__ constexpr uint32_t idesc_f8f6f4_f32(uint32_t M, uint32_t N, uint32_t afmt,
+                                                        uint32_t bfmt) {
   return (1u << 4)                // D format F32
-         | (0u << 7)              // A format E4M3
-         | (0u << 10)             // B format E4M3
+         | (afmt << 7)            // A format
+         | (bfmt << 10)           // B format
          | ((N >> 3) << 17)       // N / 8
          | ((M >> 4) << 24);      // M / 16
+}
+
+// E4M3 A and B.
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t M, uint32_t N) {
+  return idesc_f8f6f4_f32(M, N, kFmtE4M3, kFmtE4M3);
 }
 
 // --------------------------------------------------------------- numbers ---

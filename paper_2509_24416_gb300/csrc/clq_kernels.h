@@ -23,7 +23,8 @@ struct RotateQuantArgs {
   int32_t* status;       // device status word
   int32_t logb;          // log2(b)
   int32_t e4m3;          // codes layout: 0 packed nibbles, 1 one E4M3 byte each,
-                         // 2 8-bit codes as two E4M3 planes (16 h, l)
+                         // 2 8-bit codes as two E4M3 planes (16 h, l), 3 E2M3
+                         // (16 codes in 12 bytes)
 };
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
@@ -80,6 +81,10 @@ cudaError_t launch_code_sums(const uint8_t* W, int codes, int N, int K, float* w
                              cudaStream_t st);
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st);
+// rows x K codes from one 4-bit layout to another (K % 16 == 0; E2M3 needs
+// K % 128 == 0 only for the GEMM's tensor maps).
+cudaError_t launch_convert_codes(const uint8_t* src, int src_codes, uint8_t* dst, int dst_codes,
+                                 int rows, int K, int32_t* status, cudaStream_t st);
 
 // Workspace of the fused kernel: codes, scales, per-token-block row counters.
 struct FusedWorkspace {
@@ -127,6 +132,13 @@ cudaError_t launch_peak_tcgen05(int iters, int32_t* status, cudaStream_t st, lon
 cudaError_t launch_peak_mma_sync(int kind, int iters, int32_t* sink, cudaStream_t st,
                                  long long* macs);
 cudaError_t launch_peak_hbm_read(const void* buf, size_t bytes, int32_t* sink, cudaStream_t st);
+// The GEMM's operand stream (peaks.cu): `tiles` 128 x 256 tiles a CTA, one
+// CTA per SM, from a rows x K code array (E4M3 or E2M3); with `mma` the MMAs
+// too.  *smem_bytes / *macs receive the shared-memory bytes filled and the
+// multiply-accumulates.
+cudaError_t launch_peak_operand_stream(const uint8_t* buf, int rows, int K, int codes, int mma,
+                                       int tiles, int32_t* status, cudaStream_t st,
+                                       long long* smem_bytes, long long* macs);
 // Raise `func`'s dynamic shared-memory limit to the device maximum once per
 // device, and (per_sm != null) return its occupancy for (threads, smem),
 // cached, so that launches make no per-call attribute queries.

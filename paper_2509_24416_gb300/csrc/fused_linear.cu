@@ -27,6 +27,8 @@
 // rows in the shared memory the GEMM leaves free, and warp 15 claims their
 // tiles, loads and publishes them (rq::run's loader mode).  The GEMM of a
 // token block starts as soon as its rows are published.
+#include <type_traits>
+
 #include "gemm_pipeline.cuh"
 #include "rq_device.cuh"
 
@@ -103,7 +105,9 @@ struct Conc {
   static constexpr size_t RQ_OFF = (C::BYTES + 1023) & ~static_cast<size_t>(1023);
 };
 
-template <typename T, bool BPACK, int BNT>
+// F6 (both forms): the workspace codes and the weights are E2M3, loaded by
+// 16U6 tensor maps (gemm::pipeline's F6 mode).
+template <typename T, bool BPACK, int BNT, bool F6>
 __global__ void __launch_bounds__(FT, 1)
     fused_linear_kernel(const __grid_constant__ CUtensorMap mapA,
                         const __grid_constant__ CUtensorMap mapB,
@@ -124,13 +128,14 @@ __global__ void __launch_bounds__(FT, 1)
   __syncthreads();
 
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr};
-  pipeline<T, false, BPACK, BNT, false>(maps, g, smem, &bars, tmem, ready);
+  pipeline<T, false, BPACK, BNT, false, 1, 1, false, 0, MAX_STAGES, F6>(maps, g, smem, &bars,
+                                                                        tmem, ready);
   tc_fence_before();
   __syncthreads();
   teardown(tmem, Cfg<false, BPACK, BNT>::TMEM);
 }
 
-template <typename T, int BNT>
+template <typename T, int BNT, bool F6>
 __global__ void __launch_bounds__(FT, 1)
     fused_concurrent_kernel(const __grid_constant__ CUtensorMap mapA,
                             const __grid_constant__ CUtensorMap mapB,
@@ -157,33 +162,33 @@ __global__ void __launch_bounds__(FT, 1)
         rq, smem + Conc<BNT>::RQ_OFF, tile_counter, PublishRows{ready, team}, team);
   } else {
     const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr, nullptr, nullptr};
-    pipeline<T, false, false, BNT, false, 1, 1, false, 4, kConcGemmStages>(maps, g, smem, &bars,
-                                                                          tmem, ready);
+    pipeline<T, false, false, BNT, false, 1, 1, false, 4, kConcGemmStages, F6>(maps, g, smem,
+                                                                              &bars, tmem, ready);
   }
   tc_fence_before();
   __syncthreads();
   teardown(tmem, C::TMEM);
 }
 
-template <typename T, int BNT>
+template <typename T, int BNT, bool F6>
 cudaError_t launch_conc(const CUtensorMap& mapA, const CUtensorMap& mapB,
                         const CUtensorMap& mapY, const RotateQuantArgs& rq, const GemmArgs& g,
                         uint32_t* ready, int use_tma_store, size_t smem, int grid,
                         cudaStream_t st) {
   uint32_t* tile_counter = ready + (g.M + BM - 1) / BM;
-  auto k = fused_concurrent_kernel<T, BNT>;
+  auto k = fused_concurrent_kernel<T, BNT, F6>;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, FT, nullptr);
   if (e != cudaSuccess) return e;
   k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store);
   return cudaGetLastError();
 }
 
-template <typename T, bool BPACK, int BNT>
+template <typename T, bool BPACK, int BNT, bool F6>
 cudaError_t launch_t(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapY,
                      const RotateQuantArgs& rq, const GemmArgs& g, uint32_t* ready,
                      int use_tma_store, size_t smem, int grid, cudaStream_t st) {
   uint32_t* tile_counter = ready + (g.M + BM - 1) / BM;
-  auto k = fused_linear_kernel<T, BPACK, BNT>;
+  auto k = fused_linear_kernel<T, BPACK, BNT, F6>;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, FT, nullptr);
   if (e != cudaSuccess) return e;
   k<<<grid, FT, smem, st>>>(mapA, mapB, mapY, rq, g, ready, tile_counter, use_tma_store);
@@ -214,7 +219,9 @@ cudaError_t launch_concurrent(const RotateQuantArgs& rq_in, const uint8_t* W, in
                               cudaStream_t st) {
   RotateQuantArgs rq = rq_in;
   rq.logb = logb;
-  rq.e4m3 = 1;
+  const bool f6 = w_codes == CLQ_CODES_E2M3;
+  const int a_codes = f6 ? CLQ_CODES_E2M3 : CLQ_CODES_E4M3;  // the weights' family
+  rq.e4m3 = f6 ? 3 : 1;
   const int segs = rq.K / 32;
   const int R = std::min(kTeamCompute / segs, kConcStride / (2 * rq.K));
   if (R < 1) return cudaErrorInvalidValue;
@@ -229,7 +236,7 @@ cudaError_t launch_concurrent(const RotateQuantArgs& rq_in, const uint8_t* W, in
       cudaMemsetAsync(ready, 0, sizeof(uint32_t) * (static_cast<size_t>(tiles_m) + 1), st);
   if (e != cudaSuccess) return e;
   CUtensorMap mapA, mapB, mapY;
-  if (!encode_codes_map(&mapA, rq.Q, CLQ_CODES_E4M3, g.M, g.K, BM, 0) ||
+  if (!encode_codes_map(&mapA, rq.Q, a_codes, g.M, g.K, BM, 0) ||
       !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn, 0))
     return cudaErrorInvalidValue;
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
@@ -238,15 +245,19 @@ cudaError_t launch_concurrent(const RotateQuantArgs& rq_in, const uint8_t* W, in
   } else {
     mapY = mapA;  // unused
   }
-  if (dtype == CLQ_F16)
-    return bn == 192 ? launch_conc<__half, 192>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                                smem, sms, st)
-                     : launch_conc<__half, 256>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                                smem, sms, st);
-  return bn == 192 ? launch_conc<__nv_bfloat16, 192>(mapA, mapB, mapY, rq, g, ready,
-                                                     use_tma_store, smem, sms, st)
-                   : launch_conc<__nv_bfloat16, 256>(mapA, mapB, mapY, rq, g, ready,
-                                                     use_tma_store, smem, sms, st);
+  auto go = [&](auto f6_tag) {
+    constexpr bool F6 = decltype(f6_tag)::value;
+    if (dtype == CLQ_F16)
+      return bn == 192 ? launch_conc<__half, 192, F6>(mapA, mapB, mapY, rq, g, ready,
+                                                      use_tma_store, smem, sms, st)
+                       : launch_conc<__half, 256, F6>(mapA, mapB, mapY, rq, g, ready,
+                                                      use_tma_store, smem, sms, st);
+    return bn == 192 ? launch_conc<__nv_bfloat16, 192, F6>(mapA, mapB, mapY, rq, g, ready,
+                                                           use_tma_store, smem, sms, st)
+                     : launch_conc<__nv_bfloat16, 256, F6>(mapA, mapB, mapY, rq, g, ready,
+                                                           use_tma_store, smem, sms, st);
+  };
+  return f6 ? go(std::true_type()) : go(std::false_type());
 }
 
 }  // namespace
@@ -266,7 +277,10 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   // raw stage holds.
   RotateQuantArgs rq = rq_in;
   rq.logb = logb;
-  rq.e4m3 = 1;  // the workspace holds the codes in the GEMM's operand layout
+  // the workspace holds the codes in the GEMM's operand layout: E2M3 beside
+  // E2M3 weights, else E4M3
+  const bool f6 = w_codes == CLQ_CODES_E2M3;
+  rq.e4m3 = f6 ? 3 : 1;
   const int segs = rq.K / 32;
   const int R = std::max(1, std::min(FT / segs, kRqStride / (2 * rq.K)));
   const size_t rq_bytes = rq::smem_bytes(R, kRqStride, kRqStages);
@@ -280,7 +294,7 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
   if (e != cudaSuccess) return e;
 
   CUtensorMap mapA, mapB, mapY;
-  if (!encode_codes_map(&mapA, rq.Q, CLQ_CODES_E4M3, g.M, g.K, BM, 0) ||
+  if (!encode_codes_map(&mapA, rq.Q, f6 ? CLQ_CODES_E2M3 : CLQ_CODES_E4M3, g.M, g.K, BM, 0) ||
       !encode_codes_map(&mapB, W, w_codes, g.N, g.K, bn, 0))
     return cudaErrorInvalidValue;
   const int use_tma_store = (g.N % 8 == 0) ? 1 : 0;
@@ -290,15 +304,21 @@ cudaError_t launch_fused_linear(const RotateQuantArgs& rq_in, const uint8_t* W, 
     mapY = mapA;  // unused
   }
   const int grid = sms;
-  if (dtype == CLQ_F16)
-    return bpack ? launch_t<__half, true, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                              smem, grid, st)
-                 : launch_t<__half, false, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
-                                               smem, grid, st);
-  return bpack ? launch_t<__nv_bfloat16, true, BN>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
+  if (f6)
+    return dtype == CLQ_F16
+               ? launch_t<__half, false, BN, true>(mapA, mapB, mapY, rq, g, ready, use_tma_store,
                                                    smem, grid, st)
-               : launch_t<__nv_bfloat16, false, BN>(mapA, mapB, mapY, rq, g, ready,
-                                                    use_tma_store, smem, grid, st);
+               : launch_t<__nv_bfloat16, false, BN, true>(mapA, mapB, mapY, rq, g, ready,
+                                                          use_tma_store, smem, grid, st);
+  if (dtype == CLQ_F16)
+    return bpack ? launch_t<__half, true, BN, false>(mapA, mapB, mapY, rq, g, ready,
+                                                     use_tma_store, smem, grid, st)
+                 : launch_t<__half, false, BN, false>(mapA, mapB, mapY, rq, g, ready,
+                                                      use_tma_store, smem, grid, st);
+  return bpack ? launch_t<__nv_bfloat16, true, BN, false>(mapA, mapB, mapY, rq, g, ready,
+                                                          use_tma_store, smem, grid, st)
+               : launch_t<__nv_bfloat16, false, BN, false>(mapA, mapB, mapY, rq, g, ready,
+                                                           use_tma_store, smem, grid, st);
 }
 
 }  // namespace clq

@@ -205,7 +205,11 @@ __device__ __forceinline__ void epilogue_block(const uint32_t (&r)[32], int c, i
 // processed, so its latency hides behind the arithmetic and the store (32
 // more registers a thread).  `store_count` counts this warp's stores (it
 // selects the staging buffer).
-template <typename OutT, int NCOL, int NBUF, bool PREFETCH, bool ASYM = false>
+//
+// SEP3 > 0: the accumulator is the sum of three TMEM accumulators SEP3
+// columns apart, each an exact integer in fp32 (the W8A8 plane products); they
+// are added as int32 and the block goes on with that (exact) sum.
+template <typename OutT, int NCOL, int NBUF, bool PREFETCH, bool ASYM = false, int SEP3 = 0>
 __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, int col0,
                                               int lane, int m0, int n0, int M, int N, float sx,
                                               const float* col_scale, const float* col_bias,
@@ -215,6 +219,38 @@ __device__ __forceinline__ void epilogue_part(uint32_t tmem_acc, int quarter, in
   static_assert(NCOL % EPI_COLS == 0, "column share must be whole 32-column blocks");
   const uint32_t lane_base = tmem_acc + (static_cast<uint32_t>(quarter * 32) << 16);
   if (n0 + col0 >= N) return;
+  if constexpr (SEP3 > 0) {
+    const int row = m0 + quarter * 32 + lane;
+#pragma unroll 1
+    for (int c = col0; c < col0 + NCOL && n0 + c < N; c += EPI_COLS) {
+      uint32_t r[32], r1[32];
+      tmem_ld32(lane_base + c, r);
+      tmem_ld32(lane_base + SEP3 + c, r1);
+      tmem_ld_wait_tie(r);
+      tmem_ld_wait_tie(r1);
+      int32_t isum[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        isum[j] = __float2int_rn(__uint_as_float(r[j])) + __float2int_rn(__uint_as_float(r1[j]));
+      tmem_ld32(lane_base + 2 * SEP3 + c, r1);
+      tmem_ld_wait_tie(r1);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        isum[j] += __float2int_rn(__uint_as_float(r1[j]));
+        r[j] = __float_as_uint(static_cast<float>(isum[j]));
+      }
+      if (acc_dbg != nullptr && row < M) {
+        int32_t* arow = acc_dbg + static_cast<size_t>(row) * N + n0 + c;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (n0 + c + j < N) arow[j] = isum[j];
+      }
+      epilogue_block<OutT, NBUF, ASYM>(r, c, quarter, lane, m0, n0, M, N, sx, col_scale,
+                                       col_bias, zm, col_zw, staging, mapY, Y, nullptr,
+                                       store_count);
+    }
+    return;
+  }
   if (!PREFETCH) {
 #pragma unroll 1
     for (int c = col0; c < col0 + NCOL && n0 + c < N; c += EPI_COLS) {

@@ -9,11 +9,11 @@
 // integer accumulators come out exact as long as the fp32 sums are exact
 // (checked bit for bit against the int64 oracle, +-7 codes at K = 16384).
 // 8-bit codes (W4A8, W8A8) arrive as two E4M3 planes, 16 h and l with
-// q = 16 h + l, and every pair of planes is multiplied into the same
-// accumulator.  Every partial sum of W4A8 stays below 2^24 for K <= 16384
-// (at most (128 + 8) * 7 per code pair), so it is exact too; W8A8 is exact
-// while the partial sums stay below 2^24 (any codes at K <= 896: at most
-// (128 + 8)^2 per code pair) and takes fp32 rounding beyond.
+// q = 16 h + l.  W4A8 multiplies both activation planes into one
+// accumulator: every partial sum stays below 2^24 for K <= 16384 (at most
+// (128 + 8) * 7 per code pair), so it is exact too.  W8A8 keeps three
+// accumulators (SEP below) that are each exact and are added as integers.
+// E2M3 operands (F6) take the same MMA with 6-bit formats.
 //
 // Persistent: one CTA per SM walks 128 (M) x 256 (N) tiles in a static
 // round-robin order, K step 128 codes.  Each operand arrives either as E4M3
@@ -58,8 +58,11 @@ constexpr int MAX_STAGES = 6;
 // values, so the MMAs of the two planes add up to q in one accumulator).
 // EW: epilogue warps (0: 4 with unpack warps, else 8); SMAX: stage cap, for
 // a CTA that keeps shared memory for other work.
+// SEP (8-bit x 8-bit codes, PA = PB = 2): the plane products go to three
+// accumulators (16 h x 16 h, the two cross terms, l x l) of one buffer, so
+// that each stays exact in fp32 (see pipeline()); 3 BNT TMEM columns.
 template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1, int EW = 0,
-          int SMAX = MAX_STAGES>
+          int SMAX = MAX_STAGES, bool SEP = false>
 struct Cfg {
   static constexpr bool UNPACK = APACK || BPACK;
   static constexpr int EPI_WARPS = EW != 0 ? EW : (UNPACK ? 4 : 8);
@@ -84,12 +87,14 @@ struct Cfg {
   static constexpr uint32_t TX = (APACK ? A_P : AU) + (BPACK ? BP : BU);
   // two accumulators of BNT columns, 2 * BNT rounded up to the power of two
   // tcgen05.alloc takes
-  static constexpr uint32_t TMEM = 2 * BNT <= 256 ? 256u : 512u;
+  static constexpr uint32_t TMEM = SEP ? 512u : (2 * BNT <= 256 ? 256u : 512u);
+  static constexpr int NBUF = SEP ? 1 : 2;  // accumulator buffers (tiles in flight)
   static_assert(S >= 2, "pipeline needs two stages");
   static_assert((PA == 1 || PA == 2) && (PB == 1 || PB == 2), "one or two planes");
   static_assert(!UNPACK || (PA == 1 && PB == 1), "8-bit planes come as E4M3 only");
   static_assert(EPI_WARPS == 4 || (EPI_WARPS == 8 && !UNPACK), "4 or 8 epilogue warps");
   static_assert(SMAX <= MAX_STAGES, "barrier arrays hold MAX_STAGES stages");
+  static_assert(!SEP || (PA == 2 && PB == 2 && 3 * BNT <= 512), "SEP: 8-bit x 8-bit, 3 BNT <= 512");
 };
 
 struct __align__(8) Barriers {
@@ -124,9 +129,9 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 // Barrier init (thread 0) and TMEM allocation (warp WARP_MMA); the caller
 // follows with tcgen05 fences around a CTA barrier.
 template <bool APACK, bool BPACK, int BNT = BN, int PA = 1, int PB = 1, int EW = 0,
-          int SMAX = MAX_STAGES>
+          int SMAX = MAX_STAGES, bool SEP = false>
 __device__ __forceinline__ void setup(Barriers* bars) {
-  using C = Cfg<APACK, BPACK, BNT, PA, PB, EW, SMAX>;
+  using C = Cfg<APACK, BPACK, BNT, PA, PB, EW, SMAX, SEP>;
   constexpr int S = C::S;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -169,12 +174,29 @@ __device__ __forceinline__ bool wait_rows_ready(const uint32_t* ready, int m, ui
 // configuration, where registers allow it).
 // ASYM: asymmetric activation codes (zero-point epilogue, g.lo / g.wsum).
 // EW / SMAX: as in Cfg (the same values as the setup() call).
+// F6: both operands are E2M3 codes, 16 codes in 12 bytes in global memory;
+// the tensor maps (type 16U6_ALIGN16B) pad every 12-byte group to 16 bytes on
+// the way into shared memory, which is the layout tcgen05.mma kind::f8f6f4
+// reads for 6-bit operands, so a stage holds the same 128 bytes per row and K
+// step as with E4M3 while only 96 of them cross from L2 (the copies complete
+// that many transaction bytes).
+//
+// SEP (W8A8): plane 0 holds 16 h and plane 1 l of each 8-bit code (q = 16 h
+// + l), so q_x q_w = (16 h_x)(16 h_w) + [(16 h_x) l_w + l_x (16 h_w)] + l_x l_w.
+// One fp32 accumulator would round once partial sums pass 2^24 (K > 896 at
+// +-127).  Kept apart, each stays exact to K = 16384: the first sums
+// multiples of 256 below 2^28 (exact up to 2^32), the second multiples of 16
+// below 2^25 (exact up to 2^28), the third integers below 2^20.  The
+// epilogue adds them as int32 (|q_x q_w| K <= 2^28).
 template <typename OutT, bool APACK, bool BPACK, int BNT = BN, bool EPI_PREFETCH = true,
-          int PA = 1, int PB = 1, bool ASYM = false, int EW = 0, int SMAX = MAX_STAGES>
+          int PA = 1, int PB = 1, bool ASYM = false, int EW = 0, int SMAX = MAX_STAGES,
+          bool F6 = false, bool SEP = false>
 __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, uint8_t* smem,
                                          Barriers* bars, uint32_t tmem, const uint32_t* ready) {
-  using C = Cfg<APACK, BPACK, BNT, PA, PB, EW, SMAX>;
+  using C = Cfg<APACK, BPACK, BNT, PA, PB, EW, SMAX, SEP>;
   constexpr int S = C::S;
+  static_assert(!F6 || (!C::UNPACK && PA == 1 && PB == 1), "E2M3 operands come one plane each");
+  constexpr uint32_t TX = F6 ? C::TX / 4 * 3 : C::TX;
   volatile int32_t* abort = &bars->abort;
 
   const int warp = threadIdx.x >> 5;
@@ -212,7 +234,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&bars->tma_full[s], C::TX);
+          mbar_arrive_expect_tx(&bars->tma_full[s], TX);
           if (APACK)
             tma_load_2d(smem + C::OFF_PA + s * A_P, maps.A, kb * BKP, m0, &bars->tma_full[s]);
           else
@@ -237,12 +259,14 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
     }
   } else if (warp == WARP_MMA) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_e4m3_f32(BM, BNT);
+      constexpr uint32_t idesc = F6 ? idesc_f8f6f4_f32(BM, BNT, kFmtE2M3, kFmtE2M3)
+                                    : idesc_e4m3_f32(BM, BNT);
       int it = 0, tc = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tc) {
-        const int buf = tc & 1;
-        if (!mbar_wait_bounded(&bars->acc_empty[buf], ((tc >> 1) & 1) ^ 1, abort, g.status,
+        const int buf = SEP ? 0 : (tc & 1);
+        const uint32_t use = SEP ? tc : (tc >> 1);  // this buffer's earlier tiles
+        if (!mbar_wait_bounded(&bars->acc_empty[buf], (use & 1) ^ 1, abort, g.status,
                                kWaitLimitNs)) {
           ok = false;
           break;
@@ -264,10 +288,15 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
 #pragma unroll
             for (int pb = 0; pb < PB; ++pb)
 #pragma unroll
-              for (int k = 0; k < BK / 32; ++k)
-                mma_e4m3(d, sw128_desc(a0 + pa * A_U + k * 32),
-                         sw128_desc(b0 + pb * BNT * BK + k * 32), idesc,
-                         (kb | pa | pb | k) != 0 ? 1u : 0u);
+              for (int k = 0; k < BK / 32; ++k) {
+                // SEP: accumulator 0 (16h x 16h), 1 (cross terms), 2 (l x l); the
+                // cross terms' second product always accumulates
+                const int acc_i = SEP ? (pa + pb) : 0;
+                const bool first = SEP ? ((kb | k) == 0 && !(pa == 1 && pb == 0))
+                                       : (kb | pa | pb | k) == 0;
+                mma_e4m3(d + acc_i * BNT, sw128_desc(a0 + pa * A_U + k * 32),
+                         sw128_desc(b0 + pb * BNT * BK + k * 32), idesc, first ? 0u : 1u);
+              }
           mma_commit(&bars->mma_done[s]);
         }
         if (ok) mma_commit(&bars->acc_full[buf]);
@@ -286,7 +315,8 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tc) {
       const int m0 = (t / tiles_n) * BM;
       const int n0 = (t % tiles_n) * BNT;
-      const int buf = tc & 1;
+      const int buf = SEP ? 0 : (tc & 1);
+      const uint32_t use = SEP ? tc : (tc >> 1);
       // Column data of this tile into the buffer of its parity; the buffer of
       // the other parity may still be read by slower warps (previous tile).
       float* col_scale = reinterpret_cast<float*>(smem + C::OFF_COL) + buf * 3 * BNT;
@@ -303,7 +333,7 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
         col_bias[j] = bi;
         if (ASYM) col_zw[j] = col < g.N ? g.wsum[col] * sc : 0.f;
       }
-      bool ok = mbar_wait_bounded(&bars->acc_full[buf], (tc >> 1) & 1, abort, g.status,
+      bool ok = mbar_wait_bounded(&bars->acc_full[buf], use & 1, abort, g.status,
                                   kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok);
       named_bar_sync(kEpiBarrier, C::EPI_THREADS);  // column data of this tile written
@@ -315,7 +345,8 @@ __device__ __forceinline__ void pipeline(const Maps& maps, const GemmArgs& g, ui
       const float sx = row < g.M ? __ldcg(g.s_x + row) : 0.f;
       // asymmetric codes: the value of code 0 is min + 2^(n-1) delta
       const float zm = ASYM && row < g.M ? fmaf(g.zp_shift, sx, __ldcg(g.lo + row)) : 0.f;
-      epilogue_part<OutT, C::EPI_NCOL, C::EPI_NBUF, EPI_PREFETCH && !C::UNPACK, ASYM>(
+      epilogue_part<OutT, C::EPI_NCOL, C::EPI_NBUF, EPI_PREFETCH && !C::UNPACK && !SEP, ASYM,
+                    SEP ? BNT : 0>(
           tmem + buf * BNT, quarter, part * C::EPI_NCOL, lane, m0, n0, g.M, g.N, sx, col_scale,
           col_bias, zm, col_zw, staging, maps.Y, g.Y, g.acc_dbg, stores);
       tc_fence_before();

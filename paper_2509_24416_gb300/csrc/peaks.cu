@@ -8,7 +8,13 @@
 //  * mma.sync (warp-level MMA, the only INT8 / INT4 tensor path sm_103a
 //    has): s8 m16n8k32, s4 m16n8k64 and, for comparison, e4m3 m16n8k32,
 //    8 warps per CTA, 4 CTAs per SM, 4 independent accumulators per warp;
-//  * HBM read: every byte of a caller buffer read once with 16-byte loads.
+//  * HBM read: every byte of a caller buffer read once with 16-byte loads;
+//  * operand stream: the W4A4 GEMM's main loop without its epilogue, one CTA
+//    per SM: a TMA producer fills a ring of four 48 KB stages with the GEMM's
+//    boxes (A 128 rows, B 256 rows, 128 codes a row, E4M3 or E2M3 layout)
+//    from a caller code array, and a consumer either releases each stage at
+//    once (the rate at which an SM takes operands in) or issues the GEMM's
+//    four 128 x 256 x 32 MMAs on it (the rate of the main loop).
 #include "clq_device.cuh"
 #include "clq_kernels.h"
 
@@ -109,7 +115,128 @@ __global__ void peak_hbm_read_kernel(const uint4* __restrict__ p, size_t n, int3
   if (x == 0x9E3779B9u) sink[0] = static_cast<int32_t>(x);
 }
 
+constexpr int kStreamStages = 4;
+constexpr int kStreamA = 128 * 128;  // smem bytes of one A box (E4M3 or padded E2M3)
+constexpr int kStreamB = 256 * 128;
+
+// F6: E2M3 boxes (0.75 of the smem bytes cross from L2); MMA: issue the MMAs.
+template <bool F6, bool MMA>
+__global__ void __launch_bounds__(128, 1)
+    peak_stream_kernel(const __grid_constant__ CUtensorMap mapA,
+                       const __grid_constant__ CUtensorMap mapB, int rows, int K, int tiles,
+                       int32_t* status) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full[kStreamStages], empty[kStreamStages], done;
+  __shared__ uint32_t slot;
+  __shared__ int32_t abort;
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStreamStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&done, 1);
+    abort = 0;
+    fence_mbarrier_init();
+  }
+  if (MMA && warp == 1) {
+    tmem_alloc(&slot, 256);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const int nk = K / 128, mt = rows / 128, nt = rows / 256;
+  constexpr uint32_t TX = F6 ? (kStreamA + kStreamB) / 4 * 3 : kStreamA + kStreamB;
+  const int steps = tiles * nk;
+  if (warp == 0 && lane == 0) {
+    prefetch_tensor_map(&mapA);
+    prefetch_tensor_map(&mapB);
+    for (int it = 0; it < steps; ++it) {
+      const int s = it % kStreamStages;
+      const int t = static_cast<int>(blockIdx.x) + (it / nk) * static_cast<int>(gridDim.x);
+      const int kb = it % nk;
+      if (!mbar_wait_bounded(&empty[s], ((it / kStreamStages) & 1) ^ 1, &abort, status,
+                             kWaitLimitNs))
+        break;
+      mbar_arrive_expect_tx(&full[s], TX);
+      uint8_t* st = smem + s * (kStreamA + kStreamB);
+      tma_load_2d(st, &mapA, kb * 128, (t % mt) * 128, &full[s]);
+      tma_load_2d(st + kStreamA, &mapB, kb * 128, ((t / mt) % nt) * 256, &full[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t idesc = F6 ? idesc_f8f6f4_f32(128, 256, kFmtE2M3, kFmtE2M3)
+                                  : idesc_e4m3_f32(128, 256);
+    bool ok = true;
+    for (int it = 0; it < steps && ok; ++it) {
+      const int s = it % kStreamStages;
+      ok = mbar_wait_bounded(&full[s], (it / kStreamStages) & 1, &abort, status, kWaitLimitNs);
+      if (!ok) break;
+      if (MMA) {
+        tc_fence_after();
+        const uint32_t a0 = smem_addr(smem + s * (kStreamA + kStreamB));
+        const uint32_t b0 = a0 + kStreamA;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_e4m3(slot, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                   (it | k) != 0 ? 1u : 0u);
+        mma_commit(&empty[s]);
+      } else {
+        mbar_arrive(&empty[s]);
+      }
+    }
+    if (MMA) {
+      mma_commit(&done);
+      mbar_wait_bounded(&done, 0, nullptr, nullptr, 100000000ull);
+    }
+    if (!ok) {  // copies already issued land before the CTA exits
+      for (int s = 0; s < kStreamStages; ++s)
+        for (int ph = 0; ph < 2; ++ph)
+          mbar_wait_bounded(&full[s], ph, nullptr, nullptr, 10000000ull);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (MMA && warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(slot, 256);
+  }
+}
+
+template <bool F6, bool MMA>
+cudaError_t launch_stream_t(const CUtensorMap& a, const CUtensorMap& b, int rows, int K,
+                            int tiles, int32_t* status, int sms, cudaStream_t st) {
+  auto k = peak_stream_kernel<F6, MMA>;
+  const size_t smem = kStreamStages * (kStreamA + kStreamB) + 1024;
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, 128, nullptr);
+  if (e != cudaSuccess) return e;
+  k<<<sms, 128, smem, st>>>(a, b, rows, K, tiles, status);
+  return cudaGetLastError();
+}
+
 }  // namespace
+
+cudaError_t launch_peak_operand_stream(const uint8_t* buf, int rows, int K, int codes, int mma,
+                                       int tiles, int32_t* status, cudaStream_t st,
+                                       long long* smem_bytes, long long* macs) {
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  CUtensorMap a, b;
+  if (!encode_codes_map(&a, buf, codes, rows, K, 128, 0) ||
+      !encode_codes_map(&b, buf, codes, rows, K, 256, 0))
+    return cudaErrorInvalidValue;
+  const long long steps = static_cast<long long>(sms) * tiles * (K / 128);
+  *smem_bytes = steps * (kStreamA + kStreamB);
+  *macs = mma ? steps * 128LL * 256 * 128 : 0;
+  const bool f6 = codes == CLQ_CODES_E2M3;
+  if (f6)
+    return mma ? launch_stream_t<true, true>(a, b, rows, K, tiles, status, sms, st)
+               : launch_stream_t<true, false>(a, b, rows, K, tiles, status, sms, st);
+  return mma ? launch_stream_t<false, true>(a, b, rows, K, tiles, status, sms, st)
+             : launch_stream_t<false, false>(a, b, rows, K, tiles, status, sms, st);
+}
 
 cudaError_t launch_peak_tcgen05(int iters, int32_t* status, cudaStream_t st, long long* macs) {
   const int sms = sm_count();

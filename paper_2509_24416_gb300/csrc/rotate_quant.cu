@@ -7,6 +7,11 @@ namespace clq {
 
 namespace {
 
+// Cost-model constants of the paired kernel (us, elements per us per SM).
+constexpr double kPairFloorUs = 1.0;
+constexpr double kPairRate = 10000.0;
+constexpr double kPairFirstUs = 0.25;
+
 // Outlier score (Sec. 3.3): S = fp32 batch mean (sequential sum over the
 // batch, then / B), score[k] = max_t |S[t][k]|.  Threads own channels;
 // blockIdx.y owns a slice of tokens; slices combine with an integer atomicMax
@@ -75,6 +80,79 @@ void rotate_quant_config(int M, int K, int sms, int* rows_per_tile, int* threads
   *smem = rq::smem_bytes(best_r, stride, stages);
 }
 
+// Paired-row kernel (rq_pair.cuh): RH rows per half-stage, chosen by the same
+// kind of model: an SM runs a round of its resident CTAs' tiles in about
+// max(floor, elements / (rate * min(1, warps / 12))) us (issue-bound with
+// enough warps, latency-bound below), the CTAs walk ceil(tiles / CTAs)
+// rounds, and the first tile's arrival adds its bytes' share of latency.
+void rotate_quant_pair_config(int M, int K, int sms, int* rows_half, int* threads, size_t* smem,
+                              int* half) {
+  const int row = 2 * K;
+  const int hb = row <= rq::kPairHalfSmall ? rq::kPairHalfSmall : rq::kPairHalfLarge;
+  const int segs = K >> 5;
+  const int rh_max = std::max(1, std::min(hb / row, 512 / segs));
+  const int regs_warps = 65536 / (32 * rq::kPairMaxRegs);
+  int best = 1;
+  double best_cost = 1e300;
+  for (int rh = 1; rh <= rh_max; ++rh) {
+    const int warps = (rh * segs + 31) / 32;
+    const size_t bytes = rq::pair_smem_bytes(rh, hb, rq::kPairStages);
+    const int ctas = std::min(regs_warps / warps, static_cast<int>((227u * 1024u) / (bytes + 1024u)));
+    if (ctas < 1) continue;
+    const long tiles = (static_cast<long>(M) + 2 * rh - 1) / (2 * rh);
+    const long total = static_cast<long>(ctas) * std::max(sms, 1);
+    const long rounds = (tiles + total - 1) / total;
+    const double elems = static_cast<double>(ctas) * 2 * rh * K;
+    const double occ = std::min(1.0, ctas * warps / 12.0);
+    const double round_us = std::max(kPairFloorUs, elems / (kPairRate * occ));
+    const double cost = rounds * round_us + kPairFirstUs * (2.0 * rh * row) / 4608.0;
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = rh;
+    }
+  }
+  *rows_half = best;
+  *threads = ((best * segs) + 31) & ~31;
+  *smem = rq::pair_smem_bytes(best, hb, rq::kPairStages);
+  *half = hb;
+}
+
+// Wide-segment kernel (rq_wide.cuh): RH rows a tile, one thread per 64
+// positions of a row, stage STAGE bytes; the same model as the paired
+// kernel with the register cap of the wide loop.
+void rotate_quant_wide_config(int M, int K, int sms, int* rows, int* threads, size_t* smem,
+                              int* stage) {
+  const int row = 2 * K;
+  const int sb = row <= rq::kPairHalfSmall ? rq::kPairHalfSmall : rq::kPairHalfLarge;
+  const int segs = K >> 6;
+  const int rh_max = std::max(1, std::min(sb / row, 512 / segs));
+  const int regs_warps = 65536 / (32 * rq::kWideMaxRegs);
+  int best = 1;
+  double best_cost = 1e300;
+  for (int rh = 1; rh <= rh_max; ++rh) {
+    const int warps = (rh * segs + 31) / 32;
+    const size_t bytes = rq::wide_smem_bytes(rh, sb, rq::kPairStages);
+    const int ctas = std::min(regs_warps / warps, static_cast<int>((227u * 1024u) / (bytes + 1024u)));
+    if (ctas < 1) continue;
+    const long tiles = (static_cast<long>(M) + rh - 1) / rh;
+    const long total = static_cast<long>(ctas) * std::max(sms, 1);
+    const long rounds = (tiles + total - 1) / total;
+    // idle lanes of a partial last warp cost like working ones
+    const double elems = static_cast<double>(ctas) * warps * 32 * 64;
+    const double occ = std::min(1.0, ctas * warps / 12.0);
+    const double round_us = std::max(kPairFloorUs, elems / (kPairRate * occ));
+    const double cost = rounds * round_us + kPairFirstUs * (rh * row) / 4608.0;
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = rh;
+    }
+  }
+  *rows = best;
+  *threads = ((best * segs) + 31) & ~31;
+  *smem = rq::wide_smem_bytes(best, sb, rq::kPairStages);
+  *stage = sb;
+}
+
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
                                 cudaStream_t st) {
   RotateQuantArgs args = a;
@@ -82,6 +160,31 @@ cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
   size_t smem = 0;
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
+  // Symmetric 4-bit activation codes in the E4M3 or E2M3 layout: the wide
+  // kernel for b = 64 (K % 64 == 0; measured 10 % faster in the PixArt step
+  // than the paired kernel, which wins at b = 128 and 256), the paired-row
+  // kernel for 32 <= b <= 256 otherwise.
+  const bool hot = a.lo == nullptr && a.clip == nullptr && (a.e4m3 == 1 || a.e4m3 == 3);
+  if (hot && logb == 6 && a.K % 64 == 0) {
+    int stage = 0;
+    rotate_quant_wide_config(a.M, a.K, sms, &args.rows_per_tile, &threads, &smem, &stage);
+    const bool e2 = a.e4m3 == 3;
+    if (dtype == CLQ_F16)
+      return e2 ? launch_rotate_quant_wide_f16_e2m3(args, logb, stage, threads, smem, sms, st)
+                : launch_rotate_quant_wide_f16_e4m3(args, logb, stage, threads, smem, sms, st);
+    return e2 ? launch_rotate_quant_wide_bf16_e2m3(args, logb, stage, threads, smem, sms, st)
+              : launch_rotate_quant_wide_bf16_e4m3(args, logb, stage, threads, smem, sms, st);
+  }
+  if (hot && logb >= 5) {
+    int half = 0;
+    rotate_quant_pair_config(a.M, a.K, sms, &args.rows_per_tile, &threads, &smem, &half);
+    const bool e2 = a.e4m3 == 3;
+    if (dtype == CLQ_F16)
+      return e2 ? launch_rotate_quant_pair_f16_e2m3(args, logb, half, threads, smem, sms, st)
+                : launch_rotate_quant_pair_f16_e4m3(args, logb, half, threads, smem, sms, st);
+    return e2 ? launch_rotate_quant_pair_bf16_e2m3(args, logb, half, threads, smem, sms, st)
+              : launch_rotate_quant_pair_bf16_e4m3(args, logb, half, threads, smem, sms, st);
+  }
   rotate_quant_config(a.M, a.K, sms, &args.rows_per_tile, &threads, &smem);
   if (dtype == CLQ_F16) return launch_rotate_quant_f16(args, logb, threads, smem, sms, st);
   return launch_rotate_quant_bf16(args, logb, threads, smem, sms, st);

@@ -7,6 +7,11 @@
 // (ASYM) asymmetrically with the row's min and max as bounds (Eq. 1 with
 // dynamic l and r), stored as centered codes q - 2^(n-1).
 //
+// The standalone activation path with symmetric 4-bit codes in the E4M3 or
+// E2M3 layout and b >= 32 runs the specialized loops of rq_pair.cuh and
+// rq_wide.cuh; this general loop serves every other setting (packed codes,
+// b < 32, 8-bit and asymmetric codes, clipped weights) and the fused kernel.
+//
 // Every thread of the CTA takes part.  The CTA walks tiles of R rows.  Raw
 // rows stream into a ring of STAGES shared-memory buffers (STRIDE bytes
 // apart, both compile-time, so that a stage's address is an immediate
@@ -310,7 +315,7 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
     // m a multiple of 8 (b >= 16): measured faster than multiples of 4, 16 or
     // masks with low bits, which break up the 4-byte bank words that adjacent
     // columns share.
-    const bool xor_order = a.e4m3 == 1 && !CLIP && !SPLIT && !ASYM && lb >= 4 &&
+    const bool xor_order = (a.e4m3 == 1 || a.e4m3 == 3) && !CLIP && !SPLIT && !ASYM && lb >= 4 &&
                            (reinterpret_cast<uintptr_t>(a.perm) & 15u) == 0;
     const int xm = xor_order ? ((8 * (lane >> (lb > 5 ? lb - 5 : 0))) &
                                 ((1 << (lb < 5 ? lb : 5)) - 8))
@@ -563,6 +568,35 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
             qh[1] = make_uint4(wh[4], wh[5], wh[6], wh[7]);
             ql[0] = make_uint4(wl[0], wl[1], wl[2], wl[3]);
             ql[1] = make_uint4(wl[4], wl[5], wl[6], wl[7]);
+          } else if (a.e4m3 == 3) {
+            // E2M3 codes, 16 to 12 bytes: each group of 16 consecutive codes
+            // is one little-endian 96-bit field, code i in bits 6i .. 6i + 5.
+            // cvt gives each code's 6-bit encoding in a byte (sign bit 5); four
+            // of those bytes c = b0 | b1 << 8 | b2 << 16 | b3 << 24 close up to
+            // 24 bits by two subtractions: c - 3 (b1 << 6 | b3 << 22) moves b1
+            // and b3 down two bits, t - 15 (hi << 12) moves the upper 12-bit
+            // pair down four.
+            uint32_t g[8];
+#pragma unroll
+            for (int k = 0; k < 16; k += 2) {
+              uint32_t h[2];
+#pragma unroll
+              for (int j = 0; j < 2; ++j) {
+                const float2 q = __fadd2_rn(v[k + j], make_float2(-12582912.0f, -12582912.0f));
+                uint16_t e;
+                asm("cvt.rn.satfinite.e2m3x2.f32 %0, %1, %2;" : "=h"(e) : "f"(q.y), "f"(q.x));
+                h[j] = e;
+              }
+              uint32_t c = h[0] | (h[1] << 16);
+              c ^= (0u - ((flip_words >> (k >> 1)) & 1u)) & 0x20202020u;  // xor_order signs
+              const uint32_t t = c - 3u * ((c >> 2) & 0x0FC00FC0u);
+              g[k >> 1] = t - 15u * ((t >> 4) & 0x00FFF000u);
+            }
+            uint2* qrow = reinterpret_cast<uint2*>(a.Q + static_cast<size_t>(row) * (3 * K / 4) +
+                                                   seg * 24);
+            qrow[0] = make_uint2(g[0] | (g[1] << 24), (g[1] >> 8) | (g[2] << 16));
+            qrow[1] = make_uint2((g[2] >> 16) | (g[3] << 8), g[4] | (g[5] << 24));
+            qrow[2] = make_uint2((g[5] >> 8) | (g[6] << 16), (g[6] >> 16) | (g[7] << 8));
           } else if (a.e4m3) {
             // one byte per code: the E4M3 encoding of the integer code
             uint32_t w[8];

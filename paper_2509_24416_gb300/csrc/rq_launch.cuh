@@ -6,6 +6,8 @@
 #include <algorithm>
 
 #include "rq_device.cuh"
+#include "rq_pair.cuh"
+#include "rq_wide.cuh"
 
 namespace clq {
 
@@ -15,6 +17,24 @@ cudaError_t launch_rotate_quant_f16(const RotateQuantArgs& a, int logb, int thre
                                     int sms, cudaStream_t st);
 cudaError_t launch_rotate_quant_bf16(const RotateQuantArgs& a, int logb, int threads,
                                      size_t smem, int sms, cudaStream_t st);
+// Wide-segment kernel per input type and code layout (rotate_quant_pair_*.cu).
+cudaError_t launch_rotate_quant_wide_f16_e4m3(const RotateQuantArgs& a, int logb, int stage,
+                                              int threads, size_t smem, int sms, cudaStream_t st);
+cudaError_t launch_rotate_quant_wide_f16_e2m3(const RotateQuantArgs& a, int logb, int stage,
+                                              int threads, size_t smem, int sms, cudaStream_t st);
+cudaError_t launch_rotate_quant_wide_bf16_e4m3(const RotateQuantArgs& a, int logb, int stage,
+                                               int threads, size_t smem, int sms, cudaStream_t st);
+cudaError_t launch_rotate_quant_wide_bf16_e2m3(const RotateQuantArgs& a, int logb, int stage,
+                                               int threads, size_t smem, int sms, cudaStream_t st);
+// Paired-row kernel per input type and code layout (rotate_quant_pair_*.cu).
+cudaError_t launch_rotate_quant_pair_f16_e4m3(const RotateQuantArgs& a, int logb, int half,
+                                              int threads, size_t smem, int sms, cudaStream_t st);
+cudaError_t launch_rotate_quant_pair_f16_e2m3(const RotateQuantArgs& a, int logb, int half,
+                                              int threads, size_t smem, int sms, cudaStream_t st);
+cudaError_t launch_rotate_quant_pair_bf16_e4m3(const RotateQuantArgs& a, int logb, int half,
+                                               int threads, size_t smem, int sms, cudaStream_t st);
+cudaError_t launch_rotate_quant_pair_bf16_e2m3(const RotateQuantArgs& a, int logb, int half,
+                                               int threads, size_t smem, int sms, cudaStream_t st);
 
 namespace rq {
 
@@ -41,6 +61,84 @@ template <typename T, int LOGB, bool CLIP, bool SPLIT = false, bool ASYM = false
 cudaError_t launch_b(const RotateQuantArgs& a, int threads, size_t smem, int sms,
                      cudaStream_t st) {
   return launch_geom<T, LOGB, CLIP, kStride, kStages, SPLIT, ASYM>(a, threads, smem, sms, st);
+}
+
+// Paired-row kernel (rq_pair.cuh): a.rows_per_tile = rows of one half.
+template <typename T, int LOGB, int CODES, int HALF, bool ROT>
+cudaError_t launch_pair_geom(const RotateQuantArgs& a, int threads, size_t smem, int sms,
+                             cudaStream_t st) {
+  auto kern = rotate_quant_pair_kernel<T, LOGB, CODES, HALF, kPairStages, ROT>;
+  int per_sm = 0;
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(kern), smem, threads, &per_sm);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  const int tiles = (a.M + 2 * a.rows_per_tile - 1) / (2 * a.rows_per_tile);
+  const int g = std::min(tiles, sms * per_sm);
+  return launch_pdl(kern, g, threads, smem, st, a);
+}
+
+template <typename T, int CODES, int HALF, bool ROT>
+cudaError_t launch_pair_b(const RotateQuantArgs& a, int logb, int threads, size_t smem, int sms,
+                          cudaStream_t st) {
+  switch (logb) {
+    case 5: return launch_pair_geom<T, 5, CODES, HALF, ROT>(a, threads, smem, sms, st);
+    case 6: return launch_pair_geom<T, 6, CODES, HALF, ROT>(a, threads, smem, sms, st);
+    case 7: return launch_pair_geom<T, 7, CODES, HALF, ROT>(a, threads, smem, sms, st);
+    default: return launch_pair_geom<T, 8, CODES, HALF, ROT>(a, threads, smem, sms, st);
+  }
+}
+
+template <typename T, int CODES, bool ROT>
+cudaError_t launch_pair_h(const RotateQuantArgs& a, int logb, int half, int threads, size_t smem,
+                          int sms, cudaStream_t st) {
+  return half == kPairHalfSmall
+             ? launch_pair_b<T, CODES, kPairHalfSmall, ROT>(a, logb, threads, smem, sms, st)
+             : launch_pair_b<T, CODES, kPairHalfLarge, ROT>(a, logb, threads, smem, sms, st);
+}
+
+// The paired kernel for CODES (1 E4M3, 3 E2M3), 32 <= b <= 256; `half` is the
+// half-stage size rotate_quant_pair_config chose.
+template <typename T, int CODES>
+cudaError_t launch_rotate_quant_pair_t(const RotateQuantArgs& a, int logb, int half, int threads,
+                                       size_t smem, int sms, cudaStream_t st) {
+  if (a.rot != nullptr)
+    return launch_pair_h<T, CODES, true>(a, logb, half, threads, smem, sms, st);
+  return launch_pair_h<T, CODES, false>(a, logb, half, threads, smem, sms, st);
+}
+
+// Wide-segment kernel (rq_wide.cuh): a.rows_per_tile = rows of a tile.
+template <typename T, int LOGB, int CODES, int STAGE, bool ROT>
+cudaError_t launch_wide_geom(const RotateQuantArgs& a, int threads, size_t smem, int sms,
+                             cudaStream_t st) {
+  auto kern = rotate_quant_wide_kernel<T, LOGB, CODES, STAGE, kPairStages, ROT>;
+  int per_sm = 0;
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(kern), smem, threads, &per_sm);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  const int tiles = (a.M + a.rows_per_tile - 1) / a.rows_per_tile;
+  const int g = std::min(tiles, sms * per_sm);
+  return launch_pdl(kern, g, threads, smem, st, a);
+}
+
+template <typename T, int CODES, int STAGE, bool ROT>
+cudaError_t launch_wide_b(const RotateQuantArgs& a, int logb, int threads, size_t smem, int sms,
+                          cudaStream_t st) {
+  (void)logb;  // b = 64 only
+  return launch_wide_geom<T, 6, CODES, STAGE, ROT>(a, threads, smem, sms, st);
+}
+
+// The wide kernel for CODES (1 E4M3, 3 E2M3), b = 64, K % 64 == 0; `stage`
+// is the stage size rotate_quant_wide_config chose.
+template <typename T, int CODES>
+cudaError_t launch_rotate_quant_wide_t(const RotateQuantArgs& a, int logb, int stage, int threads,
+                                       size_t smem, int sms, cudaStream_t st) {
+  if (a.rot != nullptr)
+    return stage == kPairHalfSmall
+               ? launch_wide_b<T, CODES, kPairHalfSmall, true>(a, logb, threads, smem, sms, st)
+               : launch_wide_b<T, CODES, kPairHalfLarge, true>(a, logb, threads, smem, sms, st);
+  return stage == kPairHalfSmall
+             ? launch_wide_b<T, CODES, kPairHalfSmall, false>(a, logb, threads, smem, sms, st)
+             : launch_wide_b<T, CODES, kPairHalfLarge, false>(a, logb, threads, smem, sms, st);
 }
 
 // log2(b) is a compile-time constant for b >= 16 on the 4-bit activation

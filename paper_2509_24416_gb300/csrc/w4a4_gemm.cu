@@ -16,14 +16,18 @@ namespace {
 
 using namespace gemm;
 
-template <bool APACK, bool BPACK, int BNT, int PA, int PB>
+// W8A8 tiles: three accumulators of 128 columns fill one TMEM allocation.
+constexpr int kSepBN = 128;
+
+template <bool APACK, bool BPACK, int BNT, int PA, int PB, bool SEP = false>
 constexpr size_t smem_bytes() {
-  return Cfg<APACK, BPACK, BNT, PA, PB>::BYTES + 1024;  // + alignment slack
+  return Cfg<APACK, BPACK, BNT, PA, PB, 0, MAX_STAGES, SEP>::BYTES + 1024;  // + alignment slack
 }
 
 // PA / PB = 2: the activation / weight codes are 8-bit, as two E4M3 planes
 // (mapA2 / mapB2 the second plane).
-template <typename OutT, bool APACK, bool BPACK, int BNT, int PA, int PB, bool ASYM>
+template <typename OutT, bool APACK, bool BPACK, int BNT, int PA, int PB, bool ASYM, bool F6,
+          bool SEP>
 __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap mapA,
                      const __grid_constant__ CUtensorMap mapB,
@@ -34,7 +38,7 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
   __shared__ Barriers bars;
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  setup<APACK, BPACK, BNT, PA, PB>(&bars);
+  setup<APACK, BPACK, BNT, PA, PB, 0, MAX_STAGES, SEP>(&bars);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -50,10 +54,11 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
   pdl_wait();
   pdl_launch_dependents();
   const Maps maps{&mapA, &mapB, use_tma_store ? &mapY : nullptr, &mapA2, &mapB2};
-  pipeline<OutT, APACK, BPACK, BNT, true, PA, PB, ASYM>(maps, g, smem, &bars, tmem, nullptr);
+  pipeline<OutT, APACK, BPACK, BNT, true, PA, PB, ASYM, 0, MAX_STAGES, F6, SEP>(
+      maps, g, smem, &bars, tmem, nullptr);
   tc_fence_before();
   __syncthreads();
-  teardown(tmem, Cfg<APACK, BPACK, BNT, PA, PB>::TMEM);
+  teardown(tmem, Cfg<APACK, BPACK, BNT, PA, PB, 0, MAX_STAGES, SEP>::TMEM);
 }
 
 // Packed INT4 weights -> E4M3 execution layout (one code per byte, the byte
@@ -80,12 +85,142 @@ __device__ __forceinline__ int e4m3_int(uint32_t byte) {
   return (byte & 0x80u) ? -i : i;
 }
 
+// Value of the 6-bit E2M3 field f (sign bit 5, exponent bits 4-3 with bias 1,
+// three mantissa bits) times 8, exact: an integer code q gives 8 q.
+__device__ __forceinline__ int e2m3_times8(uint32_t f) {
+  const int e = (f >> 3) & 0x3;
+  const int m = f & 0x7;
+  const int v = e == 0 ? m : (8 + m) << (e - 1);
+  return (f & 0x20u) ? -v : v;
+}
+
+// The 16 codes of group g (codes 16 g .. 16 g + 15) of a row in a 4-bit layout
+// (packed nibbles, E4M3 bytes or E2M3 fields), as integers; false if a field
+// holds no integer (only E2M3 and E4M3 fields can).
+__device__ __forceinline__ bool decode_group(const uint8_t* __restrict__ row, int codes, int g,
+                                             int (&c)[16]) {
+  bool ok = true;
+  if (codes == CLQ_CODES_INT4_PACKED) {
+    const uint8_t* p = row + 8 * g;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int lo = p[j] & 0xF, hi = p[j] >> 4;
+      c[2 * j] = lo >= 8 ? lo - 16 : lo;
+      c[2 * j + 1] = hi >= 8 ? hi - 16 : hi;
+    }
+  } else if (codes == CLQ_CODES_E2M3) {
+    const uint8_t* p = row + 12 * g;
+    uint64_t lo = 0, hi = 0;  // the 96-bit group, little-endian
+#pragma unroll
+    for (int j = 0; j < 8; ++j) lo |= static_cast<uint64_t>(p[j]) << (8 * j);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) hi |= static_cast<uint64_t>(p[8 + j]) << (8 * j);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int bit = 6 * i;
+      const uint32_t f = static_cast<uint32_t>(
+          (bit < 64 ? (lo >> bit) | (bit > 58 ? hi << (64 - bit) : 0ull) : hi >> (bit - 64)) &
+          0x3Full);
+      const int v8 = e2m3_times8(f);
+      ok &= (v8 & 7) == 0;
+      c[i] = v8 / 8;
+    }
+  } else {
+    const uint8_t* p = row + 16 * g;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) c[j] = e4m3_int(p[j]);
+  }
+  return ok;
+}
+
+// Bytes of one row of K codes in a layout.
+__host__ __device__ __forceinline__ size_t codes_row_bytes(int codes, int K) {
+  return codes == CLQ_CODES_INT4_PACKED ? static_cast<size_t>(K) / 2
+         : codes == CLQ_CODES_E2M3      ? static_cast<size_t>(K) / 4 * 3
+         : codes == CLQ_CODES_E4M3_SPLIT ? 2 * static_cast<size_t>(K)
+                                         : static_cast<size_t>(K);
+}
+
+// One group of 16 integer codes in [-7, 7] into a 4-bit layout.
+__device__ __forceinline__ void encode_group(uint8_t* __restrict__ row, int codes, int g,
+                                             const int (&c)[16]) {
+  if (codes == CLQ_CODES_INT4_PACKED) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      row[8 * g + j] = static_cast<uint8_t>((c[2 * j] & 0xF) | ((c[2 * j + 1] & 0xF) << 4));
+  } else if (codes == CLQ_CODES_E2M3) {
+    // E2M3 encodings of 0..7: exponent 0 for 0, else 1..3, mantissa in eighths
+    constexpr uint8_t kMag[8] = {0x00, 0x08, 0x10, 0x14, 0x18, 0x1A, 0x1C, 0x1E};
+    uint64_t lo = 0, hi = 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint64_t f = kMag[c[i] < 0 ? -c[i] : c[i]] | (c[i] < 0 ? 0x20u : 0u);
+      const int bit = 6 * i;
+      if (bit < 64) {
+        lo |= f << bit;
+        if (bit + 6 > 64) hi |= f >> (64 - bit);
+      } else {
+        hi |= f << (bit - 64);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) row[12 * g + j] = static_cast<uint8_t>(lo >> (8 * j));
+#pragma unroll
+    for (int j = 0; j < 4; ++j) row[12 * g + 8 + j] = static_cast<uint8_t>(hi >> (8 * j));
+  } else {
+    // E4M3 encodings of 0..7 (exponent bias 7), sign bit 7
+    constexpr uint8_t kMag[8] = {0x00, 0x38, 0x40, 0x44, 0x48, 0x4A, 0x4C, 0x4E};
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      row[16 * g + j] = kMag[c[j] < 0 ? -c[j] : c[j]] | (c[j] < 0 ? 0x80u : 0u);
+  }
+}
+
+// Code array in one 4-bit layout -> another, one thread a group of 16 codes.
+// A code outside [-7, 7] (packed -8) or a field that holds no integer is
+// written as 0 and reported.
+__global__ void convert_codes_kernel(const uint8_t* __restrict__ src, int src_codes,
+                                     uint8_t* __restrict__ dst, int dst_codes, int rows, int K,
+                                     int32_t* status) {
+  const int groups = K / 16;
+  const size_t n = static_cast<size_t>(rows) * groups;
+  const size_t sb = codes_row_bytes(src_codes, K), db = codes_row_bytes(dst_codes, K);
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t r = i / groups;
+    const int g = static_cast<int>(i - r * groups);
+    int c[16];
+    bool ok = decode_group(src + r * sb, src_codes, g, c);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const bool in = c[j] >= -7 && c[j] <= 7;
+      ok &= in;
+      if (!in) c[j] = 0;
+    }
+    if (!ok) record_status(status, CLQ_ERR_DEVICE_CODE);
+    encode_group(dst + r * db, dst_codes, g, c);
+  }
+}
+
 // sum_k q[n][k] of each row of a code array (any layout), one warp a row.
 __global__ void code_sums_kernel(const uint8_t* __restrict__ W, int codes, int N, int K,
                                  float* __restrict__ wsum) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= N) return;
+  if (codes == CLQ_CODES_E2M3) {
+    const uint8_t* row = W + static_cast<size_t>(warp) * codes_row_bytes(codes, K);
+    int acc = 0;
+    for (int gi = lane; gi < K / 16; gi += 32) {
+      int c[16];
+      decode_group(row, codes, gi, c);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) acc += c[j];
+    }
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) wsum[warp] = static_cast<float>(acc);
+    return;
+  }
   const int width = codes == CLQ_CODES_INT4_PACKED ? K / 2
                     : codes == CLQ_CODES_E4M3_SPLIT ? 2 * K : K;
   const uint4* row = reinterpret_cast<const uint4*>(W + static_cast<size_t>(warp) * width);
@@ -215,11 +350,12 @@ struct MapSet {
 };
 
 template <typename OutT, bool APACK, bool BPACK, int BNT, int PA = 1, int PB = 1,
-          bool ASYM = false>
+          bool ASYM = false, bool F6 = false>
 cudaError_t launch_gemm_t(const MapSet& m, const GemmArgs& g, int use_tma_store, int grid,
                           cudaStream_t st) {
-  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT, PA, PB, ASYM>;
-  constexpr size_t smem = smem_bytes<APACK, BPACK, BNT, PA, PB>();
+  constexpr bool SEP = PA == 2 && PB == 2;  // W8A8: exact plane accumulators
+  auto k = w4a4_gemm_kernel<OutT, APACK, BPACK, BNT, PA, PB, ASYM, F6, SEP>;
+  constexpr size_t smem = smem_bytes<APACK, BPACK, BNT, PA, PB, SEP>();
   constexpr int threads = Cfg<APACK, BPACK, BNT, PA, PB>::THREADS;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, threads, nullptr);
   if (e != cudaSuccess) return e;
@@ -231,17 +367,24 @@ cudaError_t launch_gemm_dt(const MapSet& m, const GemmArgs& g, int x_codes, int 
                            int use_tma_store, int grid, cudaStream_t st) {
   const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
   const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
+  if (x_codes == CLQ_CODES_E2M3) {  // both operands E2M3 (checked by the caller)
+    if (bn == 192)
+      return launch_gemm_t<OutT, false, false, 192, 1, 1, false, true>(m, g, use_tma_store, grid,
+                                                                        st);
+    return launch_gemm_t<OutT, false, false, BN, 1, 1, false, true>(m, g, use_tma_store, grid, st);
+  }
   if (g.lo != nullptr) {  // asymmetric activations: E4M3 / split operands only
     if (x_codes == CLQ_CODES_E4M3_SPLIT)
       return w_codes == CLQ_CODES_E4M3_SPLIT
-                 ? launch_gemm_t<OutT, false, false, BN, 2, 2, true>(m, g, use_tma_store, grid, st)
+                 ? launch_gemm_t<OutT, false, false, kSepBN, 2, 2, true>(m, g, use_tma_store,
+                                                                         grid, st)
                  : launch_gemm_t<OutT, false, false, BN, 2, 1, true>(m, g, use_tma_store, grid,
                                                                      st);
     return launch_gemm_t<OutT, false, false, BN, 1, 1, true>(m, g, use_tma_store, grid, st);
   }
   if (x_codes == CLQ_CODES_E4M3_SPLIT)
     return w_codes == CLQ_CODES_E4M3_SPLIT
-               ? launch_gemm_t<OutT, false, false, BN, 2, 2>(m, g, use_tma_store, grid, st)
+               ? launch_gemm_t<OutT, false, false, kSepBN, 2, 2>(m, g, use_tma_store, grid, st)
                : launch_gemm_t<OutT, false, false, BN, 2, 1>(m, g, use_tma_store, grid, st);
   if (apack)
     return bpack ? launch_gemm_t<OutT, true, true, BN>(m, g, use_tma_store, grid, st)
@@ -254,12 +397,19 @@ cudaError_t launch_gemm_dt(const MapSet& m, const GemmArgs& g, int x_codes, int 
 }  // namespace
 
 // TMA map of a code array (rows x K codes) in any layout: packed boxes of 64
-// bytes x box_rows (no swizzle, staged for unpacking) or E4M3 boxes of 128
-// bytes x box_rows with the 128-byte swizzle (MMA operand).  For the split
+// bytes x box_rows (no swizzle, staged for unpacking), E4M3 boxes of 128
+// bytes x box_rows with the 128-byte swizzle (MMA operand), or E2M3 boxes of
+// 128 codes x box_rows (96 bytes a row in global memory, 128 in shared
+// memory, 128-byte swizzle; K a multiple of 128).  For the split
 // layout ([rows][2][K]) the map covers plane `plane` of every row (row stride
 // 2K bytes); for the others `plane` must be 0.
 bool encode_codes_map(CUtensorMap* map, const uint8_t* base, int codes, int rows, int K,
                       int box_rows, int plane) {
+  if (codes == CLQ_CODES_E2M3)  // 16 codes in 12 bytes, each group padded to 16 in smem
+    return encode_tma_2d_strided(map, CU_TENSOR_MAP_DATA_TYPE_16U6_ALIGN16B, 1, base,
+                                 static_cast<uint64_t>(K), static_cast<uint64_t>(rows),
+                                 static_cast<uint64_t>(K) / 4 * 3, BK, box_rows,
+                                 CU_TENSOR_MAP_SWIZZLE_128B);
   if (codes == CLQ_CODES_INT4_PACKED)
     return encode_tma_2d_u8(map, base, static_cast<uint64_t>(K) / 2, static_cast<uint64_t>(rows),
                             BKP, box_rows);
@@ -292,7 +442,12 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   const bool apack = x_codes == CLQ_CODES_INT4_PACKED;
   const bool bpack = w_codes == CLQ_CODES_INT4_PACKED;
   const bool split = x_codes == CLQ_CODES_E4M3_SPLIT || w_codes == CLQ_CODES_E4M3_SPLIT;
-  const int bn = (!apack && !bpack && !split && g.lo == nullptr) ? gemm_tile_n(g.M, g.N, sms) : BN;
+  // The tile-width model weighs operand bytes per K step; E2M3 scales both
+  // widths' bytes by the same 3/4, so the choice is the same.
+  const bool w8a8 = x_codes == CLQ_CODES_E4M3_SPLIT && w_codes == CLQ_CODES_E4M3_SPLIT;
+  const int bn = w8a8 ? kSepBN
+                      : (!apack && !bpack && !split && g.lo == nullptr) ? gemm_tile_n(g.M, g.N, sms)
+                                                                         : BN;
   MapSet m;
   if (!encode_codes_map(&m.A, Xq, x_codes, g.M, g.K, BM, 0) ||
       !encode_codes_map(&m.B, W, w_codes, g.N, g.K, bn, 0))
@@ -314,6 +469,17 @@ cudaError_t launch_w4a4_gemm(const uint8_t* Xq, int x_codes, const uint8_t* W, i
   if (out_dtype == CLQ_F16)
     return launch_gemm_dt<__half>(m, g, x_codes, w_codes, bn, use_tma_store, grid, st);
   return launch_gemm_dt<__nv_bfloat16>(m, g, x_codes, w_codes, bn, use_tma_store, grid, st);
+}
+
+cudaError_t launch_convert_codes(const uint8_t* src, int src_codes, uint8_t* dst, int dst_codes,
+                                 int rows, int K, int32_t* status, cudaStream_t st) {
+  const size_t n = static_cast<size_t>(rows) * (K / 16);
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  const int blocks = static_cast<int>(std::min<size_t>((n + 255) / 256, 8u * sms));
+  convert_codes_kernel<<<std::max(blocks, 1), 256, 0, st>>>(src, src_codes, dst, dst_codes, rows,
+                                                            K, status);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_expand_weights(const uint8_t* Wq, int N, int K, uint8_t* We, cudaStream_t st) {

@@ -39,7 +39,7 @@ def test_all_symbols_exported(lib):
 def test_status_strings(lib):
     for code, name in clq.STATUS.items():
         assert lib.clq_status_string(code).decode().startswith(name)
-    assert lib.clq_version() == 100
+    assert lib.clq_version() == 101
 
 
 P = 1 << 20  # a fake, 16-byte aligned "device" address; never dereferenced
@@ -48,7 +48,9 @@ P = 1 << 20  # a fake, 16-byte aligned "device" address; never dereferenced
 @pytest.mark.parametrize("args,code", [
     # (X, dtype, M, K, ldx, perm, b, codes, Xq, s_x, rot) -> expected status
     ((P, 2, 4, 64, 64, P, 32, 0, P, P, None), 1),      # bad dtype
-    ((P, 0, 4, 64, 64, P, 32, 3, P, P, None), 1),      # bad code layout
+    ((P, 0, 4, 64, 64, P, 32, 4, P, P, None), 1),      # bad code layout
+    ((P, 0, 4, 64, 64, P, 32, 3, P, P, None), 2),      # E2M3 needs K % 128
+    ((P, 0, 4, 128, 128, P, 32, 3, P + 16, P, None), 3),  # E2M3 array 32-byte aligned
     ((P, 0, -1, 64, 64, P, 32, 0, P, P, None), 1),     # negative M
     ((P, 0, 4, 64, 64, P, 3, 0, P, P, None), 2),       # b not a power of two
     ((P, 0, 4, 64, 64, P, 512, 1, P, P, None), 2),     # b > 256
@@ -89,7 +91,12 @@ def test_w4a4_host_validation(lib, args, code):
     ((P, 2, P, P, 0, P, None, 4, 4, 64, 32, 0, P, None), 4),     # W4A8, packed W
     ((P, 0, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 4),     # W8A4
     ((P, 1, P, P, 2, P, None, 4, 4, 64, 32, 0, P, None), 4),     # W8A4
-    ((P, 3, P, P, 1, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad x layout
+    ((P, 5, P, P, 1, P, None, 4, 4, 64, 32, 0, P, None), 1),     # bad x layout
+    ((P, 3, P, P, 1, P, None, 4, 4, 128, 32, 0, P, None), 4),    # E2M3 with E4M3
+    ((P, 1, P, P, 3, P, None, 4, 4, 128, 32, 0, P, None), 4),    # E4M3 with E2M3
+    ((P, 3, P, P, 3, P, None, 4, 4, 64, 32, 0, P, None), 2),     # E2M3, K % 128
+    ((P, 3, P, P + 16, 3, P, None, 4, 4, 128, 32, 0, P, None), 3),  # E2M3 W alignment
+    ((None, 3, None, None, 3, None, None, 0, 4, 128, 32, 0, None, None), 0),
     ((P, 2, P, P, 2, P, None, 4, 4, 48, 16, 0, P, None), 2),     # K % 32
     ((P, 2, P, P, 1, P, None, 4, 4, 64, 32, 0, P + 2, None), 3), # misaligned Y
     ((None, 2, None, None, 2, None, None, 0, 4, 64, 32, 0, None, None), 0),
@@ -100,8 +107,10 @@ def test_linear_host_validation(lib, args, code):
 
 def test_prepare_weights_codes_host_validation(lib):
     # (W, dtype, N, K, ldw, perm, b, clip, w_codes, Wq, s_w, rot, stream)
-    assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 32, None, 3, P, P,
+    assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 32, None, 4, P, P,
                                          None, None) == 1
+    assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 32, None, 3, P, P,
+                                         None, None) == 2          # E2M3, K % 128
     assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 32, P + 2, 2, P,
                                          P, None, None) == 3
     assert clq.clq_prepare_weights_codes(P, 0, 4, 64, 64, P, 5, None, 2, P, P,
@@ -114,14 +123,17 @@ def test_asym_host_validation(lib):
     # rotate-quant asym: (X, dtype, M, K, ldx, perm, b, codes, Xq, delta, lo, rot, stream)
     assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 1, P, P, None, None,
                                          None) == 1                    # lo missing
-    assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 3, P, P, P, None,
+    assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 5, P, P, P, None,
                                          None) == 1                    # bad layout
+    assert clq.clq_rotate_quant_act_asym(P, 0, 4, 128, 128, P, 32, 3, P, P, P, None,
+                                         None) == 4                    # E2M3: no -8
     assert clq.clq_rotate_quant_act_asym(P, 0, 4, 64, 64, P, 32, 1, P, P, P + 2, None,
                                          None) == 3                    # misaligned lo
     assert clq.clq_rotate_quant_act_asym(None, 0, 0, 64, 64, None, 32, 1, None, None,
                                          None, None, None) == 0        # empty
     # code sums: (W, codes, N, K, wsum, stream)
-    assert clq.clq_weight_code_sums(P, 3, 4, 64, P, None) == 1
+    assert clq.clq_weight_code_sums(P, 5, 4, 64, P, None) == 1
+    assert clq.clq_weight_code_sums(P, 3, 4, 64, P, None) == 2     # E2M3, K % 128
     assert clq.clq_weight_code_sums(P, 1, 4, 48, P, None) == 2
     assert clq.clq_weight_code_sums(P, 1, 4, 64, P + 1, None) == 3
     assert clq.clq_weight_code_sums(None, 1, 0, 64, None, None) == 0
@@ -180,6 +192,18 @@ def test_fused_and_prepare_host_validation(lib):
                                 P + 16, 1 << 20, None) == 3  # 256-B alignment
     assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, 5, P, None, 4, P,
                                 P, 1 << 20, None) == 1    # bad w_format
+    assert clq.clq_fused_linear(P, 0, 4, 64, 64, P, 32, P, 3, P, None, 4, P,
+                                P, 1 << 20, None) == 2    # E2M3 weights, K % 128
+    assert clq.clq_fused_linear(P, 0, 4, 128, 128, P, 32, P + 16, 3, P, None, 4, P,
+                                P, 1 << 20, None) == 3    # E2M3 weights, alignment
+    # convert: (src, src_codes, dst, dst_codes, rows, K, stream)
+    assert clq.clq_convert_codes(P, 0, P, 5, 4, 128, None) == 1
+    assert clq.clq_convert_codes(P, 0, P, 3, 4, 64, None) == 2     # E2M3, K % 128
+    assert clq.clq_convert_codes(P, 0, P, 1, 4, 48, None) == 2     # K % 32
+    assert clq.clq_convert_codes(P, 0, P + 16, 3, 4, 128, None) == 3
+    assert clq.clq_convert_codes(P + 8, 0, P, 1, 4, 128, None) == 3
+    assert clq.clq_convert_codes(None, 0, None, 3, 0, 128, None) == 0
+    assert clq.clq_convert_codes(None, 0, P, 3, 4, 128, None) == 1
     assert clq.clq_prepare_weights(P, 0, 4, 64, 64, P, 32, P + 2, P, P, None,
                                    None) == 3
     assert clq.clq_expand_weights(P, 4, 48, P, None) == 2

@@ -183,22 +183,29 @@ def test_w4a8_carrier_exact_at_extremes(K):
     assert acc[0, 0] == 889 * K
 
 
-def test_w8a8_carrier_exact_to_896_and_rounded_beyond():
-    """W8A8 with every code at +-127: exact while 18496 K < 2^24 (K <= 896);
-    beyond, the fp32 accumulator rounds and stays within a few ulp."""
+@pytest.mark.parametrize("K", [896, 4096, 16384])
+def test_w8a8_carrier_exact_at_extremes(K):
+    """W8A8 with every code at +-127: |acc| reaches 16129 K (2.6e8 at
+    K = 16384), far past 2^24, and mixed rows rise to half of that and return
+    to 0.  The plane products are accumulated apart (multiples of 256, of 16
+    and plain integers) and added as integers, so the accumulators stay exact
+    at every K."""
     M, N = 130, 140
-    for K, exact in ((896, True), (4096, False)):
-        qx = np.full((M, K), 127, np.int16)
-        qw = np.full((N, K), 127, np.int16)
-        qw[1::2] = -127
-        ones_x = np.ones(M, np.float32)
-        ones_w = np.ones(N, np.float32)
-        _, gacc, _, acc, _ = _product_case(qx, qw, ones_x, ones_w, 32, 8, "bf16")
-        if exact:
-            assert np.array_equal(gacc, acc)
-        else:
-            rel = np.abs(gacc.astype(np.float64) - acc) / np.abs(acc)
-            assert rel.max() <= 1e-6, rel.max()
+    rng = np.random.default_rng(K)
+    qx = np.where(rng.random((M, K)) < 0.5, -127, 127).astype(np.int16)
+    qw = np.where(rng.random((N, K)) < 0.5, -127, 127).astype(np.int16)
+    qx[:8] = 127
+    qw[:8] = 127
+    qw[8:16] = -127
+    qx[8:16, : K // 2] = 127
+    qx[8:16, K // 2:] = -127
+    qx[16:24] = rng.integers(-127, 128, (8, K))   # every code value
+    ones_x = np.ones(M, np.float32)
+    ones_w = np.ones(N, np.float32)
+    y, gacc, y64, acc, _ = _product_case(qx, qw, ones_x, ones_w, 32, 8, "bf16")
+    assert np.array_equal(gacc, acc)
+    assert acc[0, 0] == 16129 * K
+    check_output_elementwise(y, y64, acc, ones_x, ones_w, 32, None, "bf16")
 
 
 @pytest.mark.parametrize("a_bits,w_bits", [(8, 4), (8, 8)])
@@ -254,7 +261,7 @@ def test_prepared_linear_bit_settings(a_bits, w_bits):
     layer = clq.PreparedLinear.from_weight(W.to(DEV), perm, b, a_bits=a_bits, w_bits=w_bits)
     assert layer.w_bits == w_bits and layer.a_bits == a_bits
     Y = layer(X)
-    codes = SPLIT if a_bits == 8 else clq.CLQ_CODES_E4M3
+    codes = layer.act_codes   # split planes at A8, else the weights' 4-bit layout
     Xq, s_x = clq.rotate_quant_act(X, perm, b, codes=codes)
     Y2 = clq.linear(Xq, s_x, layer.We, layer.s_w, b, K, out_dtype=X.dtype)
     again = clq.PreparedLinear.from_state_dict(layer.state_dict())(X)

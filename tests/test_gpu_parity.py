@@ -50,9 +50,49 @@ def _decode_e4m3(byte):
     return sign * val
 
 
+def _decode_e2m3(field):
+    """Value of a 6-bit E2M3 field (1 sign bit, 2 exponent bits with bias 1,
+    3 mantissa bits; exponent 0 is subnormal), from the format definition."""
+    f = np.asarray(field, np.int64)
+    sign = np.where(f & 0x20, -1.0, 1.0)
+    e = (f >> 3) & 0x3
+    m = f & 0x7
+    val = np.where(e == 0, m / 8.0, (1 + m / 8.0) * 2.0 ** (e - 1.0))
+    return sign * val
+
+
+def _e2m3_fields(Q, K):
+    """6-bit fields of an E2M3 code array [rows, 3K/4]: each 12-byte group is
+    one little-endian 96-bit field holding 16 codes, code i in bits 6i.."""
+    Q = np.ascontiguousarray(Q, np.uint8)
+    rows = Q.shape[0]
+    bits = np.unpackbits(Q.reshape(rows, K // 16, 12), axis=-1, bitorder="little")
+    bits = bits.reshape(rows, K // 16, 16, 6).astype(np.int64)
+    return (bits << np.arange(6)).sum(-1).reshape(rows, K)
+
+
+def _encode_e2m3(codes):
+    """Host encoder of integer codes in [-7, 7] into the E2M3 layout, from the
+    format definition: |q| = (1 + m / 8) 2^(e - 1), e >= 1 (0 for q = 0)."""
+    codes = np.asarray(codes, np.int64)
+    rows, K = codes.shape
+    mag = np.abs(codes)
+    e = np.where(mag == 0, 0, np.floor(np.log2(np.maximum(mag, 1))).astype(np.int64) + 1)
+    m = np.where(mag == 0, 0, (mag * 8 // (1 << np.maximum(e - 1, 0))) - 8)
+    f = (np.where(codes < 0, 0x20, 0) | (e << 3) | m).astype(np.int64)
+    assert np.array_equal(_decode_e2m3(f), codes.astype(np.float64))
+    bits = ((f.reshape(rows, K // 16, 16, 1) >> np.arange(6)) & 1).astype(np.uint8)
+    return np.packbits(bits.reshape(rows, K // 16, 96), axis=-1,
+                       bitorder="little").reshape(rows, K // 4 * 3)
+
+
 def _codes(Xq, K):
-    """Integer codes of a GPU code array in either layout."""
+    """Integer codes of a GPU code array in any 4-bit layout."""
     Xq = np.asarray(Xq)
+    if 4 * Xq.shape[1] == 3 * K:
+        v = _decode_e2m3(_e2m3_fields(Xq, K))
+        assert np.array_equal(v, np.rint(v)) and np.abs(v).max(initial=0) <= 7
+        return v.astype(np.int8)
     if Xq.shape[1] == K:
         v = _decode_e4m3(Xq)
         assert np.array_equal(v, np.rint(v)) and np.abs(v).max(initial=0) <= 7
@@ -80,6 +120,11 @@ def _check_rq(x_t, x32, perm, b):
     # gives the same rotation too
     assert np.array_equal(_codes(eq, K), _codes(gq, K)) and np.array_equal(es, gs)
     check_rot(erot, orot)
+    if K % 128 == 0:  # the E2M3 layout (same XOR-ordered gather as E4M3)
+        fq, fs, frot = _rq_gpu(x_t, perm, b, clq.CLQ_CODES_E2M3)
+        assert fq.shape == (x32.shape[0], K // 4 * 3)
+        assert np.array_equal(_codes(fq, K), _codes(gq, K)) and np.array_equal(fs, gs)
+        check_rot(frot, orot)
     return gq, gs
 
 
@@ -217,6 +262,53 @@ def test_expand_weights_is_exact_e4m3_of_codes():
     assert np.array_equal(_decode_e4m3(We.cpu().numpy()), codes.astype(np.float64))
 
 
+def test_convert_codes_between_layouts():
+    rng = np.random.default_rng(9)
+    rows, K = 70, 1152
+    codes = rng.integers(-7, 8, (rows, K)).astype(np.int8)
+    codes[0, :15] = np.arange(-7, 8)
+    packed = torch.from_numpy(oracle.pack_int4(codes)).to(DEV)
+    e2 = clq.convert_codes(packed, K, clq.CLQ_CODES_E2M3)
+    e4 = clq.convert_codes(e2, K, clq.CLQ_CODES_E4M3)
+    back = clq.convert_codes(e4, K, clq.CLQ_CODES_INT4_PACKED)
+    again = clq.convert_codes(e2, K, clq.CLQ_CODES_E2M3)
+    torch.cuda.synchronize()
+    assert np.array_equal(e2.cpu().numpy(), _encode_e2m3(codes))
+    assert np.array_equal(_decode_e4m3(e4.cpu().numpy()), codes.astype(np.float64))
+    assert torch.equal(back, packed) and torch.equal(again, e2)
+    assert clq.device_status() == 0
+    # packed -8 has no E2M3 encoding: written as 0 and reported
+    bad = codes.copy()
+    bad[3, 5] = -8
+    e2b = clq.convert_codes(torch.from_numpy(oracle.pack_int4(bad)).to(DEV), K,
+                            clq.CLQ_CODES_E2M3)
+    assert clq.device_status() == 9           # CLQ_ERR_DEVICE_CODE
+    fixed = bad.copy()
+    fixed[3, 5] = 0
+    assert np.array_equal(e2b.cpu().numpy(), _encode_e2m3(fixed))
+
+
+def test_prepared_linear_keeps_one_weight_layout():
+    rng = np.random.default_rng(3)
+    N, K = 96, 1152
+    W = torch.from_numpy((rng.standard_normal((N, K)) * 0.02).astype(np.float32)).half().to(DEV)
+    perm = torch.from_numpy(_perm(K, "random", 2)).to(DEV)
+    layer = clq.PreparedLinear.from_weight(W, perm, 64)
+    # the default execution layout: E4M3, 1 B a weight plus scales and the swap vector
+    assert layer.w_codes == clq.CLQ_CODES_E4M3 and layer.We.shape == (N, K)
+    assert layer.resident_bytes() == N * K + 4 * N + 4 * K
+    # on request E2M3, 0.75 B a weight
+    small = clq.PreparedLinear.from_weight(W, perm, 64, w_codes=clq.CLQ_CODES_E2M3)
+    assert small.We.shape == (N, K // 4 * 3)
+    assert small.resident_bytes() == N * K * 3 // 4 + 4 * N + 4 * K
+    Wq, s_w = clq.prepare_weights(W, perm, 64)
+    X = torch.from_numpy(rng.standard_normal((40, K)).astype(np.float32)).half().to(DEV)
+    torch.cuda.synchronize()
+    assert torch.equal(layer.Wq, Wq) and torch.equal(small.Wq, Wq)
+    assert torch.equal(layer.s_w, s_w) and torch.equal(small.s_w, s_w)
+    assert torch.equal(layer(X), small(X))
+
+
 def _gemm_case(M, N, K, b, dtype, seed, bias=True):
     x_t, x32 = _inputs(M, K, dtype, seed)
     rng = np.random.default_rng(seed + 1)
@@ -231,19 +323,23 @@ def _gemm_case(M, N, K, b, dtype, seed, bias=True):
     Wq = torch.from_numpy(oWq).to(DEV)
     Xq = torch.from_numpy(oXq).to(DEV)
     outs = []
-    # every combination of storage (packed) and execution (E4M3) layouts
-    for Xc in (Xq, clq.expand_weights(Xq)):
-        for W in (Wq, clq.expand_weights(Wq)):
-            Y, gacc = clq.w4a4_linear(Xc, torch.from_numpy(os_x).to(DEV), W,
-                                      torch.from_numpy(os_w).to(DEV), b, K,
-                                      None if bias_t is None else bias_t.to(DEV),
-                                      out_dtype=TD[dtype], with_acc=True)
-            torch.cuda.synchronize()
-            assert np.array_equal(gacc.cpu().numpy(), acc)
-            y = Y.float().cpu().numpy()
-            check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
-            check_output_frobenius(y, y64)
-            outs.append(Y)
+    # every combination of storage (packed) and execution (E4M3) layouts, and
+    # E2M3 with E2M3 (host-encoded from the oracle's codes)
+    pairs = [(Xc, W) for Xc in (Xq, clq.expand_weights(Xq)) for W in (Wq, clq.expand_weights(Wq))]
+    if K % 128 == 0:
+        pairs.append((torch.from_numpy(_encode_e2m3(oracle.unpack_int4(oXq))).to(DEV),
+                      torch.from_numpy(_encode_e2m3(oracle.unpack_int4(oWq))).to(DEV)))
+    for Xc, W in pairs:
+        Y, gacc = clq.w4a4_linear(Xc, torch.from_numpy(os_x).to(DEV), W,
+                                  torch.from_numpy(os_w).to(DEV), b, K,
+                                  None if bias_t is None else bias_t.to(DEV),
+                                  out_dtype=TD[dtype], with_acc=True)
+        torch.cuda.synchronize()
+        assert np.array_equal(gacc.cpu().numpy(), acc)
+        y = Y.float().cpu().numpy()
+        check_output_elementwise(y, y64, acc, os_x, os_w, b, b32, dtype)
+        check_output_frobenius(y, y64)
+        outs.append(Y)
     for Y in outs[1:]:
         assert torch.equal(outs[0], Y)
 
@@ -283,12 +379,14 @@ def test_gemm_carrier_exact_at_extremes(K):
     ones_w = torch.ones(N, dtype=torch.float32, device=DEV)
     Wd = torch.from_numpy(Wq).to(DEV)
     Xd = torch.from_numpy(Xq).to(DEV)
-    for Xc in (Xd, clq.expand_weights(Xd)):
-        for W in (Wd, clq.expand_weights(Wd)):
-            _, gacc = clq.w4a4_linear(Xc, ones_x, W, ones_w, 32, K,
-                                      out_dtype=torch.bfloat16, with_acc=True)
-            torch.cuda.synchronize()
-            assert np.array_equal(gacc.cpu().numpy(), acc)
+    pairs = [(Xc, W) for Xc in (Xd, clq.expand_weights(Xd)) for W in (Wd, clq.expand_weights(Wd))]
+    pairs.append((torch.from_numpy(_encode_e2m3(qx)).to(DEV),
+                  torch.from_numpy(_encode_e2m3(qw)).to(DEV)))
+    for Xc, W in pairs:
+        _, gacc = clq.w4a4_linear(Xc, ones_x, W, ones_w, 32, K,
+                                  out_dtype=torch.bfloat16, with_acc=True)
+        torch.cuda.synchronize()
+        assert np.array_equal(gacc.cpu().numpy(), acc)
 
 
 def test_gemm_random_codes_all_values():
@@ -336,8 +434,13 @@ def _layer_e2e(cfg, li, M, rows=None):
     y64, _ = oracle.w4a4_linear(oXq, os_x, oWq, os_w, b, d["bias32"])
     check_output_frobenius(Y.float().cpu().numpy()[rows], y64)
     Yf = layer(X, fused=True)
+    # the E2M3 execution layout on both sides of the GEMM
+    l6 = clq.PreparedLinear.from_weight(d["W"].to(DEV), permd, b, bias=d["bias"].to(DEV),
+                                        w_codes=clq.CLQ_CODES_E2M3)
+    Y6 = l6(X)
     torch.cuda.synchronize()
     assert torch.equal(Yf, Y)          # fused = separate kernels, bit for bit
+    assert torch.equal(Y6, Y)
     return d, layer, Y
 
 
@@ -399,7 +502,11 @@ def test_fused_matches_separate_and_oracle(M, N, K, b, dtype):
     X = x_t.to(DEV)
     Y_sep = layer(X)
     ws = clq.fused_workspace(M, K, DEV)
-    for W in (layer.We, layer.Wq):
+    # the execution layout (E4M3), packed, and E2M3 where K % 128 == 0
+    Ws = [layer.We, layer.Wq]
+    if K % 128 == 0:
+        Ws.append(clq.convert_codes(layer.We, K, clq.CLQ_CODES_E2M3))
+    for W in Ws:
         Y_f = clq.fused_linear(X, layer.perm, b, W, layer.s_w, layer.bias, workspace=ws)
         torch.cuda.synchronize()
         assert torch.equal(Y_f, Y_sep)

@@ -39,7 +39,7 @@ def _noalloc(X, layer, Y):
     N = layer.We.shape[0]
     st = clq.clq_fused_linear_noalloc(
         X.data_ptr(), clq.CLQ_F16, M, K, X.stride(0), layer.perm.data_ptr(), layer.b,
-        layer.We.data_ptr(), clq.CLQ_CODES_E4M3, layer.s_w.data_ptr(), layer.bias.data_ptr(),
+        layer.We.data_ptr(), layer.w_codes, layer.s_w.data_ptr(), layer.bias.data_ptr(),
         N, Y.data_ptr(), torch.cuda.current_stream().cuda_stream)
     return st
 
