@@ -44,8 +44,10 @@ def parse():
     p.add_argument("--impl", default="clq", choices=["clq", "reference"])
     p.add_argument("--workload", default="pixart_1024")
     p.add_argument("--fused", action="store_true")
-    p.add_argument("--codes", default="auto", choices=["auto", "e4m3", "e2m3"],
-                   help="execution layout of the 4-bit codes (auto: the layer's default)")
+    p.add_argument("--codes", default="auto", choices=list(CODES),
+                   help="layouts of the 4-bit weight and activation codes (auto: the "
+                        "layer's default, E4M3; packed_w: packed-nibble weights with "
+                        "E4M3 activations; packed_a: the reverse; packed: both packed)")
     p.add_argument("--sweep", action="store_true",
                    help="time the 100-cell M x (K, N) x b grid, one JSON line per cell")
     p.add_argument("--bits", action="store_true",
@@ -93,7 +95,10 @@ KERNEL_SOURCES = {
 }
 
 
-CODES = {"auto": None, "e4m3": 1, "e2m3": 3}  # clq.CLQ_CODES_E4M3 / CLQ_CODES_E2M3
+# --codes: (weight layout, activation layout); None = the layer's default.
+# Layout numbers: 0 packed INT4 nibbles, 1 E4M3, 3 E2M3 (clq.CLQ_CODES_*).
+CODES = {"auto": (None, None), "e4m3": (1, None), "e2m3": (3, None),
+         "packed_w": (0, 1), "packed_a": (1, 0), "packed": (0, 0)}
 
 
 def rq_algorithmic_bytes(M, K):
@@ -108,6 +113,23 @@ def rq_layout_bytes(M, K, code_bytes):
     """Bytes the launch actually moves with `code_bytes` bytes a code (1 for
     the E4M3 layout, 0.75 for E2M3, 0.5 packed, 2 for split 8-bit planes)."""
     return M * ((2.0 + code_bytes) * K + 4)
+
+
+LAYOUT_NAMES = {0: "int4 packed nibbles", 1: "e4m3", 2: "e4m3 split planes", 3: "e2m3"}
+
+
+def weight_memory(layers):
+    """Resident device bytes of the prepared layers' weight codes, per weight
+    and against fp16 (2 B a weight), and of the whole packages (codes, fp32
+    scales, swap vectors, biases)."""
+    nw = sum(N * K for (_, K, N, _) in layers)
+    codes = sum(lay.We.numel() for (_, _, _, lay) in layers)
+    total = sum(lay.resident_bytes() for (_, _, _, lay) in layers)
+    return {"weight_layout": LAYOUT_NAMES[layers[0][3].w_codes],
+            "activation_layout": LAYOUT_NAMES[layers[0][3].act_codes],
+            "code_bytes_per_weight": round(codes / nw, 4),
+            "fp16_over_codes": round(2.0 * nw / codes, 3),
+            "package_bytes": total, "fp16_over_package": round(2.0 * nw / total, 3)}
 
 
 def gemm_intake_bound(M, shapes, sms, sm_mhz, bytes_per_clk):
@@ -377,7 +399,8 @@ def config_dict(cfg, args):
             "layers": ["%s %dx%d" % (n, K, N) for (n, K, N) in cfg["layers"]],
             "io_dtype": cfg["dtype"], "path": "fused" if args.fused else "separate",
             "launch": "eager" if getattr(args, "no_graph", False) else "one cuda graph of the K steps",
-            "l2": "inputs rotated over sets totalling > 2x L2 (129 MB)"}
+            "l2": "inputs rotated over sets totalling > 2x L2 (129 MB)",
+            **({} if getattr(args, "codes", "auto") == "auto" else {"codes": args.codes})}
 
 
 # ------------------------------------------------------------------ sweep ---
@@ -735,7 +758,8 @@ def main():
         calib = torch.from_numpy(d["calib"]).to(td).to(dev)
         perm = clq.build_permutation(clq.outlier_scores(calib)).to(dev)
         lay = clq.PreparedLinear.from_weight(d["W"].to(dev), perm, b,
-                                             bias=d["bias"].to(dev), w_codes=CODES[args.codes])
+                                             bias=d["bias"].to(dev), w_codes=CODES[args.codes][0],
+                                             a_codes=CODES[args.codes][1])
         layers.append((d["name"], d["K"], d["N"], lay))
         xs_host.append(d["X"])
         w_dense.append((d["W"].to(dev), d["bias"].to(dev)))  # fp16 cuBLAS comparator
@@ -1085,6 +1109,7 @@ def main():
             "scaling": "weak", "vs_baseline": None,
             "dtype": "int4 codes on %s tcgen05 operands, f32 accumulate" % (
                 "e2m3" if layers[0][3].act_codes == clq.CLQ_CODES_E2M3 else "e4m3"),
+            "weights": weight_memory(layers),
             "data": "synthetic (seeded Philox, DiT-shaped; no model weights)",
             "config": config_dict(cfg, args), "roofline": roofline,
             "roofline_rotate_quant": rq_roof, "per_layer": per_layer,

@@ -600,13 +600,16 @@ class PreparedLinear:
     paper's memory figure counts; the split planes at W8A8), converted from
     ``We`` on demand.  Activation codes are produced in an execution layout
     too (they are transient): the 4-bit layout of the weights, or split
-    planes for 8-bit activations (a_bits).  ``state_dict()`` keeps the
+    planes for 8-bit activations (a_bits); ``a_codes`` picks another 4-bit
+    activation layout (packed nibbles or E4M3 with packed or E4M3 weights,
+    E2M3 with E2M3 weights).  ``state_dict()`` keeps the
     storage codes; ``from_state_dict()`` converts them back.  Calling the
     object runs the separate rotate-quant and GEMM kernels (``fused=False``)
     or, at W4A4, the fused kernel.
     """
 
-    def __init__(self, Wq, s_w, perm, b, bias=None, We=None, a_bits=4, w_codes=None):
+    def __init__(self, Wq, s_w, perm, b, bias=None, We=None, a_bits=4, w_codes=None,
+                 a_codes=None):
         """Wq: weight codes in any layout (packed storage codes, an
         execution layout, or split planes for 8-bit weights); they are
         converted to the execution layout unless ``We`` already holds it."""
@@ -628,6 +631,13 @@ class PreparedLinear:
             self.We = src
         else:
             self.We = convert_codes(src, K, self.w_codes)
+        if a_codes is not None:
+            four = (CLQ_CODES_INT4_PACKED, CLQ_CODES_E4M3, CLQ_CODES_E2M3)
+            if a_bits != 4 or a_codes not in four or self.w_codes not in four or (
+                    (a_codes == CLQ_CODES_E2M3) != (self.w_codes == CLQ_CODES_E2M3)):
+                raise ValueError("4-bit activation codes pair packed or E4M3 with packed "
+                                 "or E4M3 weights, and E2M3 with E2M3")
+        self._a_codes = a_codes
 
     @property
     def Wq(self):
@@ -649,7 +659,7 @@ class PreparedLinear:
 
     @classmethod
     def from_weight(cls, W, perm, b, bias=None, clip=None, a_bits=4, w_bits=4,
-                    w_codes=None):
+                    w_codes=None, a_codes=None):
         perm = perm.to(W.device, torch.int32).contiguous()
         K = W.shape[1]
         if w_bits == 8:
@@ -659,7 +669,8 @@ class PreparedLinear:
         else:
             codes = exec_layout(K) if a_bits == 4 else CLQ_CODES_E4M3
         We, s_w = prepare_weights(W.contiguous(), perm, b, clip, codes=codes)
-        return cls(None, s_w, perm, b, bias, We=We, a_bits=a_bits, w_codes=codes)
+        return cls(None, s_w, perm, b, bias, We=We, a_bits=a_bits, w_codes=codes,
+                   a_codes=a_codes)
 
     @classmethod
     def calibrate(cls, W, calib, b, bias=None, metric="absmax", clip_grid=None,
@@ -694,10 +705,12 @@ class PreparedLinear:
     @property
     def act_codes(self):
         """Layout of the activation codes the separate path writes: split
-        planes for 8-bit activations, else the 4-bit layout of the weights
-        (E2M3 with E2M3, E4M3 otherwise)."""
+        planes for 8-bit activations, else the ``a_codes`` given, else the
+        4-bit layout of the weights (E2M3 with E2M3, E4M3 otherwise)."""
         if self.a_bits == 8:
             return CLQ_CODES_E4M3_SPLIT
+        if self._a_codes is not None:
+            return self._a_codes
         return CLQ_CODES_E2M3 if self.w_codes == CLQ_CODES_E2M3 else CLQ_CODES_E4M3
 
     def state_dict(self):

@@ -306,7 +306,21 @@ def test_prepared_linear_keeps_one_weight_layout():
     torch.cuda.synchronize()
     assert torch.equal(layer.Wq, Wq) and torch.equal(small.Wq, Wq)
     assert torch.equal(layer.s_w, s_w) and torch.equal(small.s_w, s_w)
-    assert torch.equal(layer(X), small(X))
+    Y = layer(X)
+    assert torch.equal(Y, small(X))
+    # packed-nibble weights (0.5 B a weight) with E4M3 or packed activations,
+    # and packed activations with E4M3 weights: the same codes, so the same Y
+    P, E = clq.CLQ_CODES_INT4_PACKED, clq.CLQ_CODES_E4M3
+    for w_codes, a_codes in ((P, E), (P, P), (E, P)):
+        lay = clq.PreparedLinear.from_weight(W, perm, 64, w_codes=w_codes, a_codes=a_codes)
+        assert lay.act_codes == a_codes and lay.w_codes == w_codes
+        if w_codes == P:
+            assert lay.We.shape == (N, K // 2)
+            assert lay.resident_bytes() == N * K // 2 + 4 * N + 4 * K
+        assert torch.equal(lay.Wq, Wq)
+        assert torch.equal(lay(X), Y)
+    with pytest.raises(ValueError):
+        clq.PreparedLinear.from_weight(W, perm, 64, w_codes=P, a_codes=clq.CLQ_CODES_E2M3)
 
 
 def _gemm_case(M, N, K, b, dtype, seed, bias=True):
