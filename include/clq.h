@@ -475,10 +475,7 @@ clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream);
  *   aligned).  mma = 0: each stage is released as soon as it lands, *ops =
  *   the shared-memory bytes filled (the rate an SM takes operands in);
  *   mma = 1: the GEMM's four 128 x 256 x 32 MMAs run on each stage, *ops =
- *   the multiply-accumulates; mma = 2 (E4M3 only): no MMA, CTAs in clusters
- *   of two that share each B tile, each loading one 128-row half of it
- *   multicast to both (every SM still receives 48 KB a step but issues
- *   32 KB), *ops = the shared-memory bytes received.
+ *   the multiply-accumulates.
  */
 clq_status clq_peak_tcgen05_e4m3(int32_t iters, int64_t* ops, void* stream);
 clq_status clq_peak_mma_sync(int32_t kind, int32_t iters, int64_t* ops, void* stream);

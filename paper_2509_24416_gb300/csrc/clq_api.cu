@@ -562,7 +562,7 @@ clq_status clq_peak_operand_stream(const uint8_t* buf, int32_t rows, int32_t K,
                                    clq_codes codes, int32_t mma, int32_t tiles, int64_t* ops,
                                    void* stream) {
   if (ops == nullptr || buf == nullptr || (codes != CLQ_CODES_E4M3 && codes != CLQ_CODES_E2M3) ||
-      mma < 0 || mma > 2 || (mma == 2 && codes != CLQ_CODES_E4M3) || tiles < 1 || tiles > 100000)
+      mma < 0 || mma > 1 || tiles < 1 || tiles > 100000)
     return CLQ_ERR_INVALID_ARG;
   if (rows < 256 || rows % 256 != 0 || K < 128 || K > 16384 || K % 128 != 0)
     return CLQ_ERR_SHAPE;

@@ -205,95 +205,6 @@ __global__ void __launch_bounds__(128, 1)
   }
 }
 
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
-               ::: "memory");
-}
-
-// Arrive once on the barrier at the same shared-memory offset in CTA `rank`
-// of the cluster.
-__device__ __forceinline__ void mbar_arrive_remote(uint64_t* bar, uint32_t rank) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_addr(bar)),
-               "r"(rank));
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote)
-               : "memory");
-}
-
-// TMA load multicast to the CTAs of `mask`: the box lands at the same
-// shared-memory offset in each and completes bytes on each one's barrier at
-// the same offset.
-__device__ __forceinline__ void tma_load_2d_mc(void* smem_dst, const CUtensorMap* map, int32_t x,
-                                               int32_t y, uint64_t* bar, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_addr(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar)), "h"(mask)
-      : "memory");
-}
-
-// The operand stream with two CTAs a cluster sharing the B tile: each CTA
-// loads its own A box and one 128-row half of B multicast to both, so every
-// SM still receives 48 KB a step but issues 32 KB.  A stage is refilled once
-// both CTAs' consumers have released it.
-__global__ void __launch_bounds__(128, 1)
-    peak_stream_mc_kernel(const __grid_constant__ CUtensorMap mapA,
-                          const __grid_constant__ CUtensorMap mapB, int rows, int K, int tiles,
-                          int32_t* status) {
-  extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full[kStreamStages], empty[kStreamStages];
-  __shared__ int32_t abort;
-  uint8_t* smem = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t rank = cluster_rank(), peer = rank ^ 1u;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kStreamStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 2);  // both CTAs' consumers
-    }
-    abort = 0;
-    fence_mbarrier_init();
-  }
-  __syncthreads();
-  cluster_sync();
-  const int nk = K / 128, mt = rows / 128, nt = rows / 256;
-  const int steps = tiles * nk;
-  if (warp == 0 && lane == 0) {
-    prefetch_tensor_map(&mapA);
-    prefetch_tensor_map(&mapB);
-    for (int it = 0; it < steps; ++it) {
-      const int s = it % kStreamStages;
-      const int t = static_cast<int>(blockIdx.x >> 1) + (it / nk) * static_cast<int>(gridDim.x >> 1);
-      const int kb = it % nk;
-      if (!mbar_wait_bounded(&empty[s], ((it / kStreamStages) & 1) ^ 1, &abort, status,
-                             kWaitLimitNs))
-        break;
-      mbar_arrive_expect_tx(&full[s], kStreamA + kStreamB);
-      uint8_t* st = smem + s * (kStreamA + kStreamB);
-      tma_load_2d(st, &mapA, kb * 128, ((2 * t + static_cast<int>(rank)) % mt) * 128, &full[s]);
-      tma_load_2d_mc(st + kStreamA + rank * (kStreamB / 2), &mapB, kb * 128,
-                     (t % nt) * 256 + static_cast<int>(rank) * 128, &full[s], 0x3);
-    }
-  } else if (warp == 1 && lane == 0) {
-    for (int it = 0; it < steps; ++it) {
-      const int s = it % kStreamStages;
-      if (!mbar_wait_bounded(&full[s], (it / kStreamStages) & 1, &abort, status, kWaitLimitNs))
-        break;
-      mbar_arrive(&empty[s]);
-      mbar_arrive_remote(&empty[s], peer);
-    }
-  }
-  __syncthreads();
-  cluster_sync();  // no CTA leaves while its peer may still write into it
-}
-
 template <bool F6, bool MMA>
 cudaError_t launch_stream_t(const CUtensorMap& a, const CUtensorMap& b, int rows, int K,
                             int tiles, int32_t* status, int sms, cudaStream_t st) {
@@ -314,33 +225,12 @@ cudaError_t launch_peak_operand_stream(const uint8_t* buf, int rows, int K, int 
   if (sms <= 0) return cudaErrorInvalidDevice;
   CUtensorMap a, b;
   if (!encode_codes_map(&a, buf, codes, rows, K, 128, 0) ||
-      !encode_codes_map(&b, buf, codes, rows, K, mma == 2 ? 128 : 256, 0))
+      !encode_codes_map(&b, buf, codes, rows, K, 256, 0))
     return cudaErrorInvalidValue;
   const long long steps = static_cast<long long>(sms) * tiles * (K / 128);
   *smem_bytes = steps * (kStreamA + kStreamB);
   *macs = mma ? steps * 128LL * 256 * 128 : 0;
-  if (mma == 2) {  // two-CTA clusters sharing B by multicast, no MMA (E4M3 boxes)
-    *macs = 0;
-    const int grid = sms & ~1;
-    *smem_bytes = static_cast<long long>(grid) * tiles * (K / 128) * (kStreamA + kStreamB);
-    const size_t smem = kStreamStages * (kStreamA + kStreamB) + 1024;
-    cudaError_t e = kernel_setup(reinterpret_cast<const void*>(peak_stream_mc_kernel), smem, 128,
-                                 nullptr);
-    if (e != cudaSuccess) return e;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(grid));
-    cfg.blockDim = dim3(128);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = st;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, peak_stream_mc_kernel, a, b, rows, K, tiles, status);
-  }
+
   const bool f6 = codes == CLQ_CODES_E2M3;
   if (f6)
     return mma ? launch_stream_t<true, true>(a, b, rows, K, tiles, status, sms, st)
