@@ -233,6 +233,16 @@ def test_peak_microbenchmark_host_validation(lib):
     assert clq.clq_peak_hbm_read(P, 100, ctypes.byref(ops), None) == 1     # bytes % 16
     assert clq.clq_peak_hbm_read(P + 4, 64, ctypes.byref(ops), None) == 3  # alignment
     assert clq.clq_peak_hbm_read(None, 64, ctypes.byref(ops), None) == 1
+    E4, E2, PK = clq.CLQ_CODES_E4M3, clq.CLQ_CODES_E2M3, clq.CLQ_CODES_INT4_PACKED
+    ok = (P, 256, 128, E4, 0, 1, ctypes.byref(ops), None)
+    for i, bad, want in ((3, PK, 1), (4, 2, 1), (4, -1, 1), (5, 0, 1), (5, 100001, 1),
+                         (1, 255, 2), (1, 384, 2), (2, 64, 2), (2, 192, 2), (2, 16512, 2),
+                         (0, P + 16, 3), (0, None, 1)):
+        args = list(ok)
+        args[i] = bad
+        assert clq.clq_peak_operand_stream(*args) == want, (i, bad)
+    assert clq.clq_peak_operand_stream(P, 256, 128, E2, 2, 1, ctypes.byref(ops), None) == 1
+    assert clq.clq_peak_operand_stream(P, 256, 128, E4, 0, 1, None, None) == 1
 
 
 @pytest.mark.parametrize("K,seed", [(1, 0), (2, 1), (7, 2), (64, 3),
