@@ -165,7 +165,9 @@ cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
   // than the paired kernel, which wins at b = 128 and 256), the paired-row
   // kernel for 32 <= b <= 256 otherwise.
   const bool hot = a.lo == nullptr && a.clip == nullptr && (a.e4m3 == 1 || a.e4m3 == 3);
-  if (hot && logb == 6 && a.K % 64 == 0) {
+  // Asymmetric 4-bit codes in E4M3 bytes take the wide kernel too (b = 64).
+  const bool hot_asym = a.lo != nullptr && a.clip == nullptr && a.e4m3 == 1;
+  if ((hot || hot_asym) && logb == 6 && a.K % 64 == 0) {
     int stage = 0;
     rotate_quant_wide_config(a.M, a.K, sms, &args.rows_per_tile, &threads, &smem, &stage);
     const bool e2 = a.e4m3 == 3;

@@ -107,10 +107,10 @@ cudaError_t launch_rotate_quant_pair_t(const RotateQuantArgs& a, int logb, int h
 }
 
 // Wide-segment kernel (rq_wide.cuh): a.rows_per_tile = rows of a tile.
-template <typename T, int LOGB, int CODES, int STAGE, bool ROT>
+template <typename T, int LOGB, int CODES, int STAGE, bool ROT, bool ASYM = false>
 cudaError_t launch_wide_geom(const RotateQuantArgs& a, int threads, size_t smem, int sms,
                              cudaStream_t st) {
-  auto kern = rotate_quant_wide_kernel<T, LOGB, CODES, STAGE, kPairStages, ROT>;
+  auto kern = rotate_quant_wide_kernel<T, LOGB, CODES, STAGE, kPairStages, ROT, ASYM>;
   int per_sm = 0;
   cudaError_t e = kernel_setup(reinterpret_cast<const void*>(kern), smem, threads, &per_sm);
   if (e != cudaSuccess) return e;
@@ -124,6 +124,9 @@ template <typename T, int CODES, int STAGE, bool ROT>
 cudaError_t launch_wide_b(const RotateQuantArgs& a, int logb, int threads, size_t smem, int sms,
                           cudaStream_t st) {
   (void)logb;  // b = 64 only
+  if constexpr (CODES == 1)
+    if (a.lo != nullptr)
+      return launch_wide_geom<T, 6, CODES, STAGE, ROT, true>(a, threads, smem, sms, st);
   return launch_wide_geom<T, 6, CODES, STAGE, ROT>(a, threads, smem, sms, st);
 }
 

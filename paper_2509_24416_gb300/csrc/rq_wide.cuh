@@ -1,7 +1,8 @@
 // Wide-segment rotate-quantize: the hot-path variant of the tile loop for
-// symmetric 4-bit activation codes when b >= 64 and K % 64 == 0 (the OBS
-// transform of arxiv 2509.24416 Sec. 3.3 and the per-token symmetric
-// quantization of Sec. 3.1 / Eq. 1, as in rq_device.cuh).
+// 4-bit activation codes when b >= 64 and K % 64 == 0 (the OBS transform of
+// arxiv 2509.24416 Sec. 3.3 and the per-token quantization of Sec. 3.1 /
+// Eq. 1, symmetric, or asymmetric with the row's minimum and maximum, as in
+// rq_device.cuh).
 //
 // Each thread owns 64 consecutive permuted positions of one row, so a block
 // of b = 64 is transformed entirely in its registers (b = 128 / 256 keep one /
@@ -22,9 +23,28 @@ namespace rq {
 constexpr int kWideMaxRegs = 160;
 
 // Shared memory of the wide loop: STAGES stages of STAGE bytes, row maxima
-// [3][RH], STAGES barriers, abort flag.
+// and (asymmetric codes) row minima [3][RH] each, STAGES barriers, abort flag.
 __host__ __device__ inline size_t wide_smem_bytes(int RH, int stage, int stages) {
-  return static_cast<size_t>(stages) * stage + 12u * RH + 8u + 8u * stages + 16u;
+  return static_cast<size_t>(stages) * stage + 24u * RH + 8u + 8u * stages + 16u;
+}
+
+// max_k v[k] and min_k v[k] over the 64 values of a segment.
+__device__ __forceinline__ void wide_minmax(const float2 (&v)[32], float& mx, float& mn) {
+  float a[16], b[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    a[i] = max3(fmaxf(v[2 * i].x, v[2 * i].y), v[2 * i + 1].x, v[2 * i + 1].y);
+    b[i] = fminf(fminf(v[2 * i].x, v[2 * i].y), fminf(v[2 * i + 1].x, v[2 * i + 1].y));
+  }
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      a[i] = fmaxf(a[i], a[i + w]);
+      b[i] = fminf(b[i], b[i + w]);
+    }
+  mx = a[0];
+  mn = b[0];
 }
 
 // max_k |v[k]| over the 64 values of a segment.
@@ -163,14 +183,79 @@ __device__ __forceinline__ void wide_quant_store(const RotateQuantArgs& a, float
   }
 }
 
+// Asymmetric codes of one row's 64-wide segment (Eq. 1 with the row's
+// minimum and maximum as bounds, as in rq_device.cuh): delta = (max - min) /
+// 15 by the same division by a constant, q = rint((v - min) / delta) stored
+// centered as q - 8 in E4M3 bytes; kmax / kmin are the row's order keys of
+// max and -min.  v holds the true transform (signs already restored).
+template <bool ROT>
+__device__ __forceinline__ void wide_quant_store_asym(const RotateQuantArgs& a, float2 (&v)[32],
+                                                      int row, int seg, uint32_t kmax,
+                                                      uint32_t kmin) {
+  const int K = a.K;
+  constexpr float div = 15.0f;
+  constexpr float rdiv = 1.0f / 15.0f;
+  const float row_lo = -order_key_inv(kmin);
+  const float am = __fsub_rn(order_key_inv(kmax), row_lo);
+  const float q1 = am * rdiv;
+  const float s_row = fmaf(fmaf(-div, q1, am), rdiv, q1);
+  if (seg == 0) {
+    a.S[row] = s_row;
+    a.lo[row] = row_lo;
+  }
+  if (ROT) {
+    float4* dst = reinterpret_cast<float4*>(a.rot + static_cast<size_t>(row) * K + seg * 64);
+#pragma unroll
+    for (int q = 0; q < 16; ++q)
+      dst[q] = make_float4(v[2 * q].x, v[2 * q].y, v[2 * q + 1].x, v[2 * q + 1].y);
+  }
+  // v <- rint((v - min) * 15 / span) + 1.5 * 2^23 - 8 (the centered code in
+  // the low mantissa bits); a constant row gets q = 0; a subnormal span takes
+  // exact divisions.
+  const float2 mg = make_float2(12582912.0f - 8.0f, 12582912.0f - 8.0f);
+  const float2 nlo = make_float2(-row_lo, -row_lo);
+  if (am > 0.f && am < 1.17549435e-38f) {
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float2 d = __fadd2_rn(v[k], nlo);
+      v[k] = __fadd2_rn(make_float2(__fmul_rn(__fdiv_rn(d.x, am), div),
+                                    __fmul_rn(__fdiv_rn(d.y, am), div)),
+                        mg);
+    }
+  } else {
+    const float inv = am > 0.f ? div * rcp_approx(am) : 0.f;
+    const float2 inv2 = make_float2(inv, inv);
+#pragma unroll
+    for (int k = 0; k < 32; ++k) v[k] = __ffma2_rn(__fadd2_rn(v[k], nlo), inv2, mg);
+  }
+  const float2 nmagic = make_float2(-12582912.0f, -12582912.0f);
+  uint4* qrow = reinterpret_cast<uint4*>(a.Q + static_cast<size_t>(row) * K + seg * 64);
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {  // 16 codes a store
+    uint32_t w[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int k = 8 * c + 2 * j;
+      uint16_t e0, e1;
+      const float2 q0 = __fadd2_rn(v[k], nmagic), q1v = __fadd2_rn(v[k + 1], nmagic);
+      asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(e0) : "f"(q0.y), "f"(q0.x));
+      asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(e1) : "f"(q1v.y), "f"(q1v.x));
+      w[j] = static_cast<uint32_t>(e0) | (static_cast<uint32_t>(e1) << 16);
+    }
+    qrow[c] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
 // CODES 1 (E4M3) or 3 (E2M3); 64 <= b <= 256 (LOGB 6 .. 8); K % 64 == 0.
+// ASYM: asymmetric codes (a.lo != null), E4M3 only.
 // a.rows_per_tile = RH rows a tile (RH * 2K <= STAGE, RH * K / 64 <=
 // blockDim.x).
-template <typename T, int LOGB, int CODES, int STAGE, int STAGES, bool ROT>
+template <typename T, int LOGB, int CODES, int STAGE, int STAGES, bool ROT, bool ASYM = false>
 __global__ void __maxnreg__(kWideMaxRegs) rotate_quant_wide_kernel(RotateQuantArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   static_assert(LOGB >= 6 && LOGB <= 8, "wide loop: 64 <= b <= 256");
   static_assert(STAGE <= 65536, "gather offsets are 16-bit");
+  static_assert(!ASYM || CODES == 1, "asymmetric codes in E4M3 bytes only");
   const int K = a.K;
   const int segs = K >> 6;
   const int RH = a.rows_per_tile;
@@ -180,8 +265,9 @@ __global__ void __maxnreg__(kWideMaxRegs) rotate_quant_wide_kernel(RotateQuantAr
 
   uint8_t* raw = smem;
   uint32_t* amax = reinterpret_cast<uint32_t*>(smem + STAGES * STAGE);  // [3][RH]
+  uint32_t* amin = amax + 3 * RH;                                          // [3][RH]
   uint64_t* full = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(amax + 3 * RH) + 7) & ~static_cast<uintptr_t>(7));
+      (reinterpret_cast<uintptr_t>(amin + 3 * RH) + 7) & ~static_cast<uintptr_t>(7));
   int32_t* abort = reinterpret_cast<int32_t*>(full + STAGES);
 
   const int ntiles = (a.M + RH - 1) / RH;
@@ -190,7 +276,7 @@ __global__ void __maxnreg__(kWideMaxRegs) rotate_quant_wide_kernel(RotateQuantAr
     *abort = 0;
     fence_mbarrier_init();
   }
-  for (int i = tid; i < 3 * RH; i += blockDim.x) amax[i] = 0u;
+  for (int i = tid; i < 6 * RH; i += blockDim.x) amax[i] = 0u;  // and amin
   __syncthreads();
   // Global inputs are read only from here on.
   pdl_wait();
@@ -284,18 +370,47 @@ __global__ void __maxnreg__(kWideMaxRegs) rotate_quant_wide_kernel(RotateQuantAr
       }
       // ---- 2. remaining stages, row maximum -----------------------------------
       wide_butterflies<LOGB>(v, lane);
-      const unsigned kx = __reduce_max_sync(grp, __float_as_uint(wide_absmax(v)));
-      if (active && lane == leader && r < n) atomicMax(&amax[par * RH + r], kx);
+      if constexpr (ASYM) {
+        // the bounds are signed: restore each 4-code group's sign first
+        if (xor_order) {
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const float sg = ((flip >> q) & 1u) ? -1.f : 1.f;
+            const float2 sg2 = make_float2(sg, sg);
+            v[2 * q] = __fmul2_rn(v[2 * q], sg2);
+            v[2 * q + 1] = __fmul2_rn(v[2 * q + 1], sg2);
+          }
+        }
+        float mx, mn;
+        wide_minmax(v, mx, mn);
+        const unsigned kx = __reduce_max_sync(grp, order_key(mx));
+        const unsigned kn = __reduce_max_sync(grp, order_key(-mn));
+        if (active && lane == leader && r < n) {
+          atomicMax(&amax[par * RH + r], kx);
+          atomicMax(&amin[par * RH + r], kn);
+        }
+      } else {
+        const unsigned kx = __reduce_max_sync(grp, __float_as_uint(wide_absmax(v)));
+        if (active && lane == leader && r < n) atomicMax(&amax[par * RH + r], kx);
+      }
       __syncthreads();  // row maxima complete; stage s fully read
       if (tid == 0) {
         const int t2 = t + STAGES * static_cast<int>(gridDim.x);
         if (t2 < ntiles) pair_issue<STAGE, 1>(a, raw + s * STAGE, &full[s], RH, t2);
       }
       // ---- 3. scale, codes, stores --------------------------------------------
-      if (active && r < n)
-        wide_quant_store<CODES, ROT>(a, v, row0 + r, seg, __uint_as_float(amax[par * RH + r]),
-                                     flip);
-      if (tid < RH) amax[((j + 2) % 3) * RH + tid] = 0u;
+      if (active && r < n) {
+        if constexpr (ASYM)
+          wide_quant_store_asym<ROT>(a, v, row0 + r, seg, amax[par * RH + r],
+                                     amin[par * RH + r]);
+        else
+          wide_quant_store<CODES, ROT>(a, v, row0 + r, seg,
+                                       __uint_as_float(amax[par * RH + r]), flip);
+      }
+      if (tid < RH) {
+        amax[((j + 2) % 3) * RH + tid] = 0u;
+        if (ASYM) amin[((j + 2) % 3) * RH + tid] = 0u;
+      }
     }
   }
   __syncthreads();
