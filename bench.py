@@ -383,7 +383,9 @@ def reference_arm(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * sec / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64/int64",
-        "data": "synthetic", "config": config_dict(cfg, args),
+        "data": "synthetic",
+        "config": dict(config_dict(cfg, args), path="oracle (numpy, one host core)",
+                       launch="host", l2="n/a (host)"),
         "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1,
                          "kind": "oracle",
                          "sample": "%d of %d tokens per layer per step" % (rows, cfg["M"])},
