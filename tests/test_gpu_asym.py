@@ -123,6 +123,34 @@ def test_rotate_quant_asym(layout, bits, M, K, b, dtype):
     assert delta[2].item() == 0.0 and np.all(gq[2] == 0)
 
 
+@pytest.mark.parametrize("layout,bits", [(E4M3, 4), (SPLIT, 8)])
+@pytest.mark.parametrize("with_rot", [False, True])
+def test_rotate_quant_asym_perm_4_byte_aligned(layout, bits, with_rot):
+    # perm 4 bytes past a 16-byte boundary: natural-order gather, no sign
+    # restore; the codes, steps and minima must equal the aligned run's.
+    M, K, b = 300, 1152, 64
+    x_t, x32 = _inputs(M, K, "bf16", seed=5, offset=1.5)
+    perm = np.random.default_rng(23).permutation(K).astype(np.int32)
+    X = x_t.to(DEV)
+    buf = torch.zeros(K + 4, dtype=torch.int32, device=DEV)
+    buf[1:K + 1] = torch.from_numpy(perm).to(DEV)
+    pv = buf[1:K + 1]
+    assert pv.data_ptr() % 16 == 4
+    ra = clq.rotate_quant_act_asym(X, torch.from_numpy(perm).to(DEV), b, codes=layout,
+                                   with_rot=with_rot)
+    rb = clq.rotate_quant_act_asym(X, pv, b, codes=layout, with_rot=with_rot)
+    torch.cuda.synchronize()
+    assert torch.equal(ra[1], rb[1]) and torch.equal(ra[2], rb[2])
+    ga = _from_layout(ra[0].cpu().numpy(), layout, K)
+    gb = _from_layout(rb[0].cpu().numpy(), layout, K)
+    assert np.array_equal(ga, gb)
+    if with_rot:
+        assert torch.equal(ra[3], rb[3])
+    oq, od, olo, orot = oracle.rotate_quant_act_asym(x32, perm, b, bits)
+    _check_asym(gb + 2 ** (bits - 1), rb[1].cpu().numpy(), rb[2].cpu().numpy(), oq, od, olo,
+                orot, bits)
+
+
 @pytest.mark.parametrize("layout,bits", [(PACKED, 4), (E4M3, 4), (SPLIT, 8)])
 def test_weight_code_sums(layout, bits):
     N, K = 300, 1152

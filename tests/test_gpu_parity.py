@@ -146,6 +146,35 @@ def test_rotate_quant_shapes(M, K):
     _check_rq(x_t, x32, _perm(K, "random", K), b)
 
 
+@pytest.mark.parametrize("b,codes", [(64, clq.CLQ_CODES_E4M3), (64, clq.CLQ_CODES_E2M3),
+                                     (128, clq.CLQ_CODES_E4M3), (32, clq.CLQ_CODES_E4M3),
+                                     (64, clq.CLQ_CODES_INT4_PACKED)])
+@pytest.mark.parametrize("with_rot", [False, True])
+def test_rotate_quant_perm_4_byte_aligned(b, codes, with_rot):
+    # The API asks perm for 4-byte alignment only; a perm 4 bytes past a
+    # 16-byte boundary makes the kernels gather in natural order (no XOR
+    # order, no sign restore).  Codes and scales must not change.
+    M, K = 300, 1152
+    x_t, x32 = _inputs(M, K, "f16", seed=b + 3)
+    perm = _perm(K, "random", 19)
+    X = x_t.to(DEV)
+    buf = torch.zeros(K + 4, dtype=torch.int32, device=DEV)
+    buf[1:K + 1] = torch.from_numpy(perm).to(DEV)
+    pv = buf[1:K + 1]
+    assert pv.data_ptr() % 16 == 4
+    pa = torch.from_numpy(perm).to(DEV)
+    ra = clq.rotate_quant_act(X, pa, b, codes, with_rot=with_rot)
+    rb = clq.rotate_quant_act(X, pv, b, codes, with_rot=with_rot)
+    torch.cuda.synchronize()
+    assert torch.equal(ra[1], rb[1])
+    assert np.array_equal(_codes(ra[0].cpu().numpy(), K), _codes(rb[0].cpu().numpy(), K))
+    if with_rot:
+        assert torch.equal(ra[2], rb[2])
+    oq, os_, orot, oc = oracle.rotate_quant_act(x32, perm, b)
+    check_scales(rb[1].cpu().numpy(), os_)
+    check_codes(_codes(rb[0].cpu().numpy(), K), oc, orot, os_)
+
+
 @pytest.mark.parametrize("K,b", [(1184, 32), (1216, 64), (1280, 128),
                                  (2112, 64)])
 def test_rotate_quant_padding_lanes_do_not_leak(K, b):
