@@ -504,7 +504,10 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
             constexpr float half = SPLIT ? 128.0f : 8.0f;
             const float2 mg = make_float2(12582912.0f - half, 12582912.0f - half);
             const float2 nlo = make_float2(-row_lo, -row_lo);
-            if (am > 0.f && am < 1.17549435e-38f) {
+            // exact divisions also where rcp(span) would be subnormal (span
+            // >= 2^126, bf16 inputs near their top), which rcp.approx.ftz
+            // flushes to zero
+            if (am > 0.f && (am < 1.17549435e-38f || am >= 8.50705917e37f)) {
 #pragma unroll
               for (int k = 0; k < 16; ++k) {
                 const float2 d = __fadd2_rn(v[k], nlo);

@@ -123,6 +123,35 @@ def test_rotate_quant_asym(layout, bits, M, K, b, dtype):
     assert delta[2].item() == 0.0 and np.all(gq[2] == 0)
 
 
+def test_rotate_quant_asym_edge_rows():
+    # asymmetric E4M3 codes at b = 64 (the wide loop): a zero row, a
+    # constant row, spikes up to 1e38, and a row whose span is subnormal in
+    # fp32 (exact divisions), against the oracle.
+    K, b = 1152, 64
+    x = np.zeros((7, K), np.float32)     # row 0 rotates to zeros: span 0
+    x[1, :] = 2.5                        # constant row: one nonzero output a block
+    x[2, 5] = 3.0
+    x[3, 7] = -1e38                      # near the top of bf16, span still finite
+    x[4, 3] = 9e-41                      # span subnormal
+    x[5] = np.random.default_rng(4).standard_normal(K).astype(np.float32) + 7.0
+    x[6, ::b] = -2.0
+    x_t = torch.from_numpy(x).to(torch.bfloat16)
+    perm = np.random.default_rng(31).permutation(K).astype(np.int32)
+    Xq, delta, lo, rot = clq.rotate_quant_act_asym(x_t.to(DEV), torch.from_numpy(perm).to(DEV),
+                                                   b, codes=E4M3, with_rot=True)
+    Xq2, delta2, lo2 = clq.rotate_quant_act_asym(x_t.to(DEV), torch.from_numpy(perm).to(DEV),
+                                                 b, codes=E4M3)
+    torch.cuda.synchronize()
+    assert torch.equal(delta, delta2) and torch.equal(lo, lo2)
+    gq = _from_layout(Xq.cpu().numpy(), E4M3, K) + 8
+    assert np.array_equal(gq, _from_layout(Xq2.cpu().numpy(), E4M3, K) + 8)
+    oq, od, olo, orot = oracle.rotate_quant_act_asym(x_t.float().numpy(), perm, b, 4)
+    assert 0 < delta[4].item() < 1.17549435e-38     # the exact-division path ran
+    assert delta[0].item() == 0.0 and np.all(gq[0] == 0)
+    check_rot(rot.cpu().numpy(), orot)
+    _check_asym(gq, delta.cpu().numpy(), lo.cpu().numpy(), oq, od, olo, orot, 4)
+
+
 @pytest.mark.parametrize("layout,bits", [(E4M3, 4), (SPLIT, 8)])
 @pytest.mark.parametrize("with_rot", [False, True])
 def test_rotate_quant_asym_perm_4_byte_aligned(layout, bits, with_rot):

@@ -229,6 +229,38 @@ def test_rotate_quant_zero_rows_and_spikes():
     assert np.array_equal(gq, oq)
 
 
+@pytest.mark.parametrize("b", [64, 128])
+def test_rotate_quant_hot_loops_edge_rows(b):
+    # The E4M3 hot-path loops (wide at b = 64, paired at b = 128) on rows
+    # with a zero row, single spikes, the bf16 maximum and values so small
+    # that the row scale is subnormal in fp32 (scaled by 2^64 before the
+    # reciprocal), against the oracle's codes and scales.
+    K = 1152
+    x = np.zeros((9, K), np.float32)
+    x[1, 5] = 3.0
+    x[3, ::b] = -2.0
+    x[4, 7] = 3.3895314e38               # bf16 maximum
+    x[5, :] = 1e-4
+    x[6, :] = 3e-39                      # tiny rows with normal scales
+    x[6, 11] = -5e-39
+    x[7, 3] = 9e-41                      # one subnormal input: subnormal scale
+    x[8] = np.random.default_rng(2).standard_normal(K).astype(np.float32) * 1e-38
+    x_t = torch.from_numpy(x).to(torch.bfloat16)
+    perm = _perm(K, "random", 29)
+    eq, es, erot = _rq_gpu(x_t, perm, b, clq.CLQ_CODES_E4M3)
+    Xq, s_x = clq.rotate_quant_act(x_t.to(DEV), torch.from_numpy(perm).to(DEV), b,
+                                   clq.CLQ_CODES_E4M3)
+    torch.cuda.synchronize()
+    assert np.array_equal(s_x.cpu().numpy(), es)
+    assert np.array_equal(_codes(Xq.cpu().numpy(), K), _codes(eq, K))
+    oq, os_, orot, oc = oracle.rotate_quant_act(x_t.float().numpy(), perm, b)
+    assert es[0] == 0 and es[2] == 0 and not _codes(eq, K)[0].any()
+    assert 0 < es[7] < 1.17549435e-38    # the subnormal-scale path ran
+    check_rot(erot, orot)
+    check_scales(es, os_)
+    check_codes(_codes(eq, K), oc, orot, os_)
+
+
 def test_rotate_quant_exact_ties_half_even():
     # rotated rows with s = 1 exactly and entries at k + 1/2: X = X~ H / b.
     b, K = 16, 64
