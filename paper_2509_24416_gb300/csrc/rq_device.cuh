@@ -264,6 +264,19 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
     fence_mbarrier_init();
   }
   for (int i = tid; i < 6 * R; i += team.size()) amax[i] = 0u;
+  // Round-robin tiles: this CTA's first tiles into L2 while the previous
+  // kernel drains; the copies after the wait still read every value from L2 /
+  // memory, where the previous kernel's writes land.
+  if (tid == 0 && tile_counter == nullptr && a.ld == a.K)
+    for (int s = 0; s < STAGES; ++s) {
+      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
+      if (t < ntiles) {
+        const int row0 = t * R;
+        const uint32_t row_bytes = static_cast<uint32_t>(a.K) * 2u;
+        bulk_prefetch_l2(static_cast<const char*>(a.X) + static_cast<size_t>(row0) * row_bytes,
+                         row_bytes * static_cast<uint32_t>(min(R, a.M - row0)));
+      }
+    }
   tsync();
   // Global inputs are read only from here on (the previous kernel on the
   // stream may still be finishing when this grid starts).

@@ -252,6 +252,17 @@ __device__ __forceinline__ void pair_issue(const RotateQuantArgs& a, uint8_t* ds
   }
 }
 
+// L2 prefetch of the rows pair_issue(.., t) copies (ld == K: one range).
+template <int NR>
+__device__ __forceinline__ void pair_prefetch(const RotateQuantArgs& a, int RH, int t) {
+  const int row0 = NR * RH * t;
+  const int n = max(0, min(NR * RH, a.M - row0));
+  const size_t row_bytes = static_cast<size_t>(a.K) * 2u;
+  if (a.ld == a.K && n > 0)
+    bulk_prefetch_l2(static_cast<const char*>(a.X) + static_cast<size_t>(row0) * row_bytes,
+                     static_cast<uint32_t>(row_bytes * n));
+}
+
 // CODES: 0 packed nibbles, 1 E4M3, 3 E2M3.  ROT: also write the rotated rows
 // to a.rot (a test aid; the variant without it keeps every value in
 // registers).  NR: rows a thread works on (2: the paired loop; 1: one row, a
@@ -290,6 +301,14 @@ __global__ void __maxnreg__(pair_max_regs<NR>()) rotate_quant_pair_kernel(Rotate
   }
   for (int i = tid; i < 6 * RH; i += blockDim.x) amax[i] = 0u;
   __syncthreads();
+  // This CTA's first tiles into L2 while the previous kernel drains; the
+  // copies after the wait still read every value from L2 / memory, where the
+  // previous kernel's writes land.
+  if (tid == 0)
+    for (int s = 0; s < STAGES; ++s) {
+      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
+      if (t < ntiles) pair_prefetch<NR>(a, RH, t);
+    }
   // Global inputs are read only from here on.
   pdl_wait();
   pdl_launch_dependents();

@@ -280,6 +280,14 @@ __global__ void __maxnreg__(kWideMaxRegs) rotate_quant_wide_kernel(RotateQuantAr
   }
   for (int i = tid; i < 6 * RH; i += blockDim.x) amax[i] = 0u;  // and amin
   __syncthreads();
+  // This CTA's first tiles into L2 while the previous kernel drains; the
+  // copies after the wait still read every value from L2 / memory, where the
+  // previous kernel's writes land.
+  if (tid == 0)
+    for (int s = 0; s < STAGES; ++s) {
+      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
+      if (t < ntiles) pair_prefetch<1>(a, RH, t);
+    }
   // Global inputs are read only from here on.
   pdl_wait();
   pdl_launch_dependents();
