@@ -795,10 +795,10 @@ def main():
     sp = stream.cuda_stream
     nlay = len(layers)
 
-    def step(si, ev=None, fused=None, s_ptr=None):
+    def step(si, ev=None, fused=None, s_ptr=None, sets=None):
         fused = args.fused if fused is None else fused
         sp_ = sp if s_ptr is None else s_ptr
-        xs = xsets[si % nsets]
+        xs = (xsets if sets is None else sets)[si % nsets]
         for i, (_, K, N, lay) in enumerate(layers):
             if ev is not None:
                 ev[4 * i].record(stream)
@@ -954,6 +954,15 @@ def main():
 
     other_ms = time_steps(lambda k, s_ptr: step(k, fused=not args.fused, s_ptr=s_ptr),
                           args.steps)
+    # The video workload's second token set (the same tokens in temporal
+    # order, a pure row permutation): the same layers, the same launch.
+    temporal_ms = None
+    tcfg = cfg.get("temporal")
+    if tcfg is not None and args.layer is None and args.tokens is None:
+        tsets = [[synth.temporal_reorder(x, **tcfg).to(dev) for x in xs_host]
+                 for _ in range(nsets)]
+        temporal_ms = time_steps(lambda k, s_ptr: step(k, s_ptr=s_ptr, sets=tsets), args.steps)
+        del tsets
 
     # Each kernel of the separate path alone, K launches back to back per
     # layer (events around the K launches only): its duration with
@@ -1141,7 +1150,12 @@ def main():
                     round(ops_step * world / (other_ms * 1e-3) / 1e12, 1),
                 "fused_over_separate_time": round(
                     (total_ms / args.steps) / other_ms if args.fused
-                    else other_ms / (total_ms / args.steps), 3)},
+                    else other_ms / (total_ms / args.steps), 3),
+                **({} if temporal_ms is None else {
+                    "temporal_token_set_tops":
+                        round(ops_step * world / (temporal_ms * 1e-3) / 1e12, 1),
+                    "temporal_over_spatial_time":
+                        round(temporal_ms / (total_ms / args.steps), 3)})},
             "measured_peaks": measured,
             "gpu_launches": (1 if args.fused else 2) * nlay * args.steps,
             "clocks": clocks,

@@ -97,7 +97,8 @@ WORKLOADS = {
     "video_16x32x32": dict(M=16384, layers=PIXART_LAYERS, b=128,
                            dtype="bf16", out_frac=0.01, out_count=None,
                            out_lo=20.0, out_hi=60.0, w_std=0.02,
-                           text_rows=0, text_scale=1.0),
+                           text_rows=0, text_scale=1.0,
+                           temporal=dict(frames=16, tokens_per_frame=1024)),
     # MMDiT: 4096 image + 512 text tokens, hidden 3072, b = 128, bf16.
     "mmdit_4608": dict(M=4608, layers=MMDIT_LAYERS, b=128, dtype="bf16",
                        out_frac=0.005, out_count=None, out_lo=50.0,
