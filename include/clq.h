@@ -43,6 +43,13 @@
  *    [0, K), a pipeline wait that exceeds its time limit) are recorded in a
  *    device status word read by clq_get_device_status; the kernel skips the
  *    offending access instead of faulting.
+ *  - Stream order holds as usual: every kernel reads its inputs and writes
+ *    its outputs only after the work enqueued before it on `stream` has
+ *    completed.  The kernels launch with programmatic dependent launch, so a
+ *    kernel of this library may become resident while the previous one on
+ *    the stream drains; in that window it only sets up on-chip state and
+ *    hints L2 prefetches of its first input rows, which change no value it
+ *    later reads.
  *  - The library keeps no per-call state and is safe to call from several
  *    host threads.
  *  - The hot-path calls (rotate-quant, the products, the fused kernel) launch
