@@ -45,11 +45,15 @@
  *    offending access instead of faulting.
  *  - Stream order holds as usual: every kernel reads its inputs and writes
  *    its outputs only after the work enqueued before it on `stream` has
- *    completed.  The kernels launch with programmatic dependent launch, so a
- *    kernel of this library may become resident while the previous one on
- *    the stream drains; in that window it only sets up on-chip state and
- *    hints L2 prefetches of its first input rows, which change no value it
- *    later reads.
+ *    completed, with one exception below.  The kernels launch with
+ *    programmatic dependent launch, so a kernel of this library may become
+ *    resident while the previous one on the stream drains; in that window
+ *    it sets up on-chip state, hints L2 prefetches of its first input rows
+ *    (which change no value it later reads) and, in rotate-quant, reads the
+ *    swap vector `perm`, a layer constant.  So `perm` must not be an output
+ *    of the call of this library enqueued just before on the same stream
+ *    (no call of this library writes a swap vector; clq_build_permutation
+ *    runs on the host).
  *  - The library keeps no per-call state and is safe to call from several
  *    host threads.
  *  - The hot-path calls (rotate-quant, the products, the fused kernel) launch

@@ -309,15 +309,6 @@ __global__ void __maxnreg__(pair_max_regs<NR>()) rotate_quant_pair_kernel(Rotate
       const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
       if (t < ntiles) pair_prefetch<NR>(a, RH, t);
     }
-  // Global inputs are read only from here on.
-  pdl_wait();
-  pdl_launch_dependents();
-  if (tid == 0)
-    for (int s = 0; s < STAGES; ++s) {
-      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
-      if (t < ntiles) pair_issue<HALF, NR>(a, raw + s * STRIDE, &full[s], RH, t);
-    }
-
   const int items = RH * segs;
   const bool active = tid < items;
   const int r = active ? tid / segs : 0;
@@ -366,6 +357,15 @@ __global__ void __maxnreg__(pair_max_regs<NR>()) rotate_quant_pair_kernel(Rotate
   // keep the shuffles convergent and never reach a row maximum.
   const unsigned grp = __match_any_sync(0xffffffffu, active ? r : -1);
   const int leader = __ffs(grp) - 1;
+  // X is read only from here on (the swap vector above is a layer constant,
+  // which no kernel of this library writes).
+  pdl_wait();
+  pdl_launch_dependents();
+  if (tid == 0)
+    for (int s = 0; s < STAGES; ++s) {
+      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
+      if (t < ntiles) pair_issue<HALF, NR>(a, raw + s * STRIDE, &full[s], RH, t);
+    }
 
   bool done = false;
   for (int j0 = 0; !done; j0 += STAGES) {
