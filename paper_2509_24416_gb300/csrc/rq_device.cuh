@@ -278,12 +278,14 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
       }
     }
   tsync();
-  // Global inputs are read only from here on (the previous kernel on the
-  // stream may still be finishing when this grid starts).
-  pdl_wait();
-  pdl_launch_dependents();
+  // Past pdl_wait, the previous kernel on the stream has completed (it may
+  // still be finishing when this grid starts): X, the tile counter and every
+  // output are touched only after it, the swap vector (a layer constant that
+  // no kernel of this library writes) before it.
   if (LOADER && tid >= nthr) {
     // ---- loader warp ---------------------------------------------------------
+    pdl_wait();
+    pdl_launch_dependents();
     if ((tid & 31) == 0) {
       for (int s = 0; s < STAGES; ++s) refill(s);
       if (tile_counter != nullptr) ahead = static_cast<int>(atomicAdd(tile_counter, 1u));
@@ -305,9 +307,6 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
     }
     __syncwarp();
   } else {
-    if (!LOADER && tid == 0)
-      for (int s = 0; s < STAGES; ++s) refill(s);
-
     const int items = R * segs;
     const bool active = tid < items;
     const int r_local = active ? tid / segs : 0;
@@ -369,6 +368,10 @@ __device__ __forceinline__ void run(const RotateQuantArgs& a, uint8_t* smem,
     // not data of any row and must not reach a row maximum.
     const unsigned grp = __match_any_sync(0xffffffffu, active ? r_local : -1);
     const int leader = __ffs(grp) - 1;
+    pdl_wait();
+    pdl_launch_dependents();
+    if (!LOADER && tid == 0)
+      for (int s = 0; s < STAGES; ++s) refill(s);
 
     bool aborted = false, done = false;
     for (int i0 = 0; !done; i0 += STAGES) {
