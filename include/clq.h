@@ -49,14 +49,17 @@
  *    programmatic dependent launch, so a kernel of this library may become
  *    resident while the previous one on the stream drains; in that window
  *    it sets up on-chip state, hints L2 prefetches of its first input rows
- *    (which change no value it later reads) and, in rotate-quant, reads the
- *    swap vector `perm`, a layer constant.  So `perm` must not be written by
- *    the kernel enqueued just before the call on the same stream: the
- *    writes of a kernel are guaranteed visible to the next one only once the
- *    latter has waited for it.  No call of this library writes a swap
- *    vector (clq_build_permutation runs on the host); a copy or another
- *    call of this library enqueued between the writing kernel and the call
- *    restores the usual order.
+ *    (which change no value it later reads) and, in the activation
+ *    rotate-quant calls (clq_rotate_quant_act, clq_rotate_quant_act_asym),
+ *    reads the swap vector `perm`, a layer constant.  So that `perm` must not
+ *    be written by the kernel enqueued just before the call on the same
+ *    stream: the writes of a kernel are guaranteed visible to the next one
+ *    only once the latter has waited for it.  No call of this library writes
+ *    a swap vector (clq_build_permutation runs on the host); a copy or
+ *    another call of this library enqueued between the writing kernel and
+ *    the call restores the usual order.  The weight-preparation calls and
+ *    clq_clip_search launch without the overlap, so a swap vector computed
+ *    on the device just before them is safe.
  *  - The library keeps no per-call state and is safe to call from several
  *    host threads.
  *  - The hot-path calls (rotate-quant, the products, the fused kernel) launch

@@ -120,7 +120,7 @@ clq_status fused_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, in
 clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ld,
                                const int32_t* perm, int32_t b, const float* clip, int codes,
                                uint8_t* Q, float* S, float* rot, void* stream,
-                               float* lo = nullptr) {
+                               float* lo = nullptr, bool weights = false) {
   if (!valid_dtype(dtype) || !valid_any_codes(codes) || M < 0) return CLQ_ERR_INVALID_ARG;
   // centered asymmetric codes reach -8, which E2M3 does not hold
   if (lo != nullptr && codes == CLQ_CODES_E2M3) return CLQ_ERR_UNSUPPORTED;
@@ -152,6 +152,7 @@ clq_status rotate_quant_common(const void* X, clq_dtype dtype, int32_t M, int32_
   a.rot = rot;
   a.lo = lo;
   a.status = status;
+  a.serial = weights ? 1 : 0;
   a.logb = log2i(b);
   a.e4m3 = codes == CLQ_CODES_E4M3         ? 1
            : codes == CLQ_CODES_E4M3_SPLIT ? 2
@@ -328,7 +329,7 @@ clq_status clq_prepare_weights(const void* W, clq_dtype dtype, int32_t N, int32_
                                const int32_t* perm, int32_t b, const float* clip, uint8_t* Wq,
                                float* s_w, float* w_rot_dbg, void* stream) {
   return rotate_quant_common(W, dtype, N, K, ldw, perm, b, clip, CLQ_CODES_INT4_PACKED, Wq, s_w,
-                             w_rot_dbg, stream);
+                             w_rot_dbg, stream, nullptr, true);
 }
 
 clq_status clq_prepare_weights_codes(const void* W, clq_dtype dtype, int32_t N, int32_t K,
@@ -336,7 +337,7 @@ clq_status clq_prepare_weights_codes(const void* W, clq_dtype dtype, int32_t N, 
                                      const float* clip, clq_codes w_codes, uint8_t* Wq,
                                      float* s_w, float* w_rot_dbg, void* stream) {
   return rotate_quant_common(W, dtype, N, K, ldw, perm, b, clip, w_codes, Wq, s_w, w_rot_dbg,
-                             stream);
+                             stream, nullptr, true);
 }
 
 clq_status clq_rotate_quant_act(const void* X, clq_dtype dtype, int32_t M, int32_t K, int32_t ldx,
@@ -640,6 +641,7 @@ clq_status clq_clip_search(const void* W, clq_dtype dtype, int32_t N, int32_t K,
     a.S = S;
     a.rot = rot;
     a.status = status;
+    a.serial = X == W ? 1 : 0;  // the weights: see clq_prepare_weights
     a.logb = log2i(b);
     a.e4m3 = 1;
     return clq::launch_rotate_quant(a, dtype, log2i(b), s);

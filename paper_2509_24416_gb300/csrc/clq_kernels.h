@@ -25,6 +25,9 @@ struct RotateQuantArgs {
   int32_t e4m3;          // codes layout: 0 packed nibbles, 1 one E4M3 byte each,
                          // 2 8-bit codes as two E4M3 planes (16 h, l), 3 E2M3
                          // (16 codes in 12 bytes)
+  int32_t serial;        // 1: launched without programmatic overlap (weight
+                         // preparation, whose swap vector may have just been
+                         // written on the device)
 };
 
 cudaError_t launch_rotate_quant(const RotateQuantArgs& a, int dtype, int logb,
@@ -144,13 +147,14 @@ cudaError_t launch_peak_operand_stream(const uint8_t* buf, int rows, int K, int 
 // cached, so that launches make no per-call attribute queries.
 cudaError_t kernel_setup(const void* func, size_t smem, int threads, int* per_sm);
 
-// Launch with programmatic stream serialization: the kernel may start while
-// the previous kernel on `st` finishes and must call pdl_wait() before it
-// reads global memory.  (Only kernel-to-kernel edges overlap; after a copy or
-// a memset the launch waits as usual.)
+// Launch with programmatic stream serialization (pdl true): the kernel may
+// start while the previous kernel on `st` finishes and must call pdl_wait()
+// before it reads what that kernel may have written.  (Only kernel-to-kernel
+// edges overlap; after a copy or a memset the launch waits as usual.)  With
+// pdl false the launch waits for the previous kernel as usual.
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), int grid, int threads, size_t smem,
-                       cudaStream_t st, Args&&... args) {
+cudaError_t launch_ex(void (*kernel)(KArgs...), int grid, int threads, size_t smem,
+                      cudaStream_t st, bool pdl, Args&&... args) {
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
@@ -160,8 +164,14 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), int grid, int threads, size_t s
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), int grid, int threads, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  return launch_ex(kernel, grid, threads, smem, st, true, std::forward<Args>(args)...);
 }
 
 }  // namespace clq

@@ -54,7 +54,7 @@ cudaError_t launch_geom(const RotateQuantArgs& a, int threads, size_t smem, int 
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
   const int ntiles = (a.M + a.rows_per_tile - 1) / a.rows_per_tile;
   const int g = std::min(ntiles, sms * per_sm);
-  return launch_pdl(kern, g, threads, smem, st, a);
+  return launch_ex(kern, g, threads, smem, st, a.serial == 0, a);
 }
 
 template <typename T, int LOGB, bool CLIP, bool SPLIT = false, bool ASYM = false>
@@ -74,7 +74,7 @@ cudaError_t launch_pair_geom(const RotateQuantArgs& a, int threads, size_t smem,
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
   const int tiles = (a.M + 2 * a.rows_per_tile - 1) / (2 * a.rows_per_tile);
   const int g = std::min(tiles, sms * per_sm);
-  return launch_pdl(kern, g, threads, smem, st, a);
+  return launch_ex(kern, g, threads, smem, st, a.serial == 0, a);
 }
 
 template <typename T, int CODES, int HALF, bool ROT>
@@ -117,7 +117,7 @@ cudaError_t launch_wide_geom(const RotateQuantArgs& a, int threads, size_t smem,
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
   const int tiles = (a.M + a.rows_per_tile - 1) / a.rows_per_tile;
   const int g = std::min(tiles, sms * per_sm);
-  return launch_pdl(kern, g, threads, smem, st, a);
+  return launch_ex(kern, g, threads, smem, st, a.serial == 0, a);
 }
 
 template <typename T, int CODES, int STAGE, bool ROT>

@@ -7,7 +7,8 @@ calls with a device synchronization between layers, bit for bit, with every
 intermediate buffer filled with NaN on the stream first (an input read too
 early would carry the NaN through), for each rotate-quant loop: the wide loop
 (b = 64), the paired loop (b = 128), the general loop (8-bit activations, and
-asymmetric 4-bit codes at b = 32), and the fused kernel."""
+asymmetric 4-bit codes at b = 32), and the fused kernel; and weights
+prepared right after torch kernels computed their swap vector."""
 import pytest
 import torch
 
@@ -85,3 +86,24 @@ def test_chained_asymmetric_layers_equal_synchronized():
         clq.linear_asym(Xq, delta, lo, lay.We, lay.s_w, wsums[i], b, K, bias=lay.bias, Y=y)
 
     _check_chain(run_layer, _x0(14))
+
+
+def test_weights_prepared_right_after_a_device_swap_vector():
+    """Weight preparation launches without programmatic overlap, so a swap
+    vector that torch kernels compute on the device just before it is read
+    complete: the prepared codes and scales equal those from the same swap
+    vector copied in after a synchronization."""
+    K, N, b = 1152, 640, 64
+    g = torch.Generator().manual_seed(21)
+    W = (torch.randn(N, K, generator=g) * 0.02).half().to(DEV)
+    scores = torch.rand(K, generator=g).to(DEV)
+    torch.cuda.synchronize()
+    for _ in range(3):
+        perm_dev = torch.argsort(scores, descending=True).to(torch.int32)  # device kernels
+        lay = clq.PreparedLinear.from_weight(W, perm_dev, b)
+        torch.cuda.synchronize()
+        ref = clq.PreparedLinear.from_weight(W, perm_dev.cpu().to(DEV), b)
+        torch.cuda.synchronize()
+        assert clq.device_status() == 0
+        assert torch.equal(lay.We, ref.We) and torch.equal(lay.s_w, ref.s_w)
+        scores = scores.roll(1)
