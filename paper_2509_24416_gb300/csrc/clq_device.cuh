@@ -128,6 +128,15 @@ __device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint
       : "memory");
 }
 
+// L2 prefetch of the box at (x, y) of a 2-D tensor map; a hint with no effect
+// on any value later read.
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
 // Bulk prefetch of [gsrc, gsrc + bytes) into L2 (16-byte aligned, bytes a
 // multiple of 16); a hint with no effect on any value later read.
 __device__ __forceinline__ void bulk_prefetch_l2(const void* gsrc, uint32_t bytes) {

@@ -49,6 +49,19 @@ __global__ void __launch_bounds__((Cfg<APACK, BPACK, BNT, PA, PB>::THREADS), 1)
     prefetch_tensor_map(&mapA);
     prefetch_tensor_map(&mapB);
     if (use_tma_store) prefetch_tensor_map(&mapY);
+    // The weight boxes of this CTA's first pipeline stages into L2 (a hint:
+    // it changes no value the copies after the wait read).
+    using C = Cfg<APACK, BPACK, BNT, PA, PB, 0, MAX_STAGES, SEP>;
+    const int tiles_n = (g.N + BNT - 1) / BNT;
+    const int tiles = ((g.M + BM - 1) / BM) * tiles_n;
+    if (!BPACK && static_cast<int>(blockIdx.x) < tiles) {
+      const int n0 = (static_cast<int>(blockIdx.x) % tiles_n) * BNT;
+      const int nk = (g.K + BK - 1) / BK;
+      for (int kb = 0; kb < C::S && kb < nk; ++kb) {
+        tma_prefetch_2d(&mapB, kb * BK, n0);
+        if (PB == 2) tma_prefetch_2d(&mapB2, kb * BK, n0);
+      }
+    }
   }
   // Barriers and TMEM are set up; global inputs are read only from here on.
   pdl_wait();
