@@ -13,7 +13,10 @@
 // shared by 64 elements a thread instead of 32, and the two rows' dependency
 // chains interleave.  Tiles are dealt round-robin over the grid (no claim
 // counter), each CTA keeps STAGES tiles in flight, and the row maxima use
-// three-input max instructions.
+// three-input max instructions.  While the previous kernel drains, the CTA
+// sets up its barriers, prefetches its first tiles into L2 and builds its
+// gather addresses from the swap vector (a layer constant); X is read only
+// after the programmatic-launch wait.
 //
 // Per tile, per thread (row r of each half, segment seg of 32 positions):
 //  1. gather both rows' 32 elements from the raw stage at columns

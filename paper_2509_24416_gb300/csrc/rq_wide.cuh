@@ -12,7 +12,10 @@
 // a register, so the thread holds as many address registers as the 32-wide
 // loop while doing twice the work per tile.  The rest follows rq_pair.cuh:
 // round-robin tiles, STAGES stages in flight, three-input maxima, one CTA
-// barrier per tile, the XOR-ordered gather whose sign flips the store undoes.
+// barrier per tile, the XOR-ordered gather whose sign flips the store undoes,
+// and a prologue that runs while the previous kernel drains: barriers, an L2
+// prefetch of the first tiles and the gather offsets from the swap vector (a
+// layer constant), with X read only after the programmatic-launch wait.
 #pragma once
 
 #include "rq_pair.cuh"
