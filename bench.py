@@ -747,6 +747,7 @@ def main():
         return
     import torch
     import torch.distributed as dist
+    import ctypes
     from paper_2509_24416_gb300 import clq, synth
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -968,7 +969,7 @@ def main():
     # layer (events around the K launches only): its duration with
     # programmatic dependent launch overlapping its neighbours, as inside the
     # step, without the event records between kernels of region 2.
-    rq_b2b, gm_b2b = None, None
+    rq_b2b, gm_b2b, rq_floor_b2b = None, None, None
     if not args.fused:
         def rq_only(i):
             _, K, N, lay = layers[i]
@@ -999,6 +1000,29 @@ def main():
 
         rq_b2b = [time_steps(rq_only(i), args.steps) for i in range(nlay)]
         gm_b2b = [time_steps(gm_only(i), args.steps) for i in range(nlay)]
+
+        # The rotate-quant loop's memory side alone on the same inputs and
+        # launch (clq_peak_rq_stream: its tiles, copy ring and stores, no
+        # arithmetic): the floor its back-to-back time is measured against.
+        if all(K % 64 == 0 for (_, K, _, _) in layers):
+            fq = torch.empty((M, max(K for (_, K, _, _) in layers)), dtype=torch.uint8,
+                             device=dev)
+            fs = torch.empty(M, dtype=torch.float32, device=dev)
+
+            def floor_only(i):
+                _, K, _, _ = layers[i]
+                ops = ctypes.c_int64(0)
+
+                def f(k, s_ptr):
+                    x = xsets[k % nsets][i]
+                    st = clq.clq_peak_rq_stream(x.data_ptr(), M, K, fq.data_ptr(), fs.data_ptr(),
+                                                ctypes.byref(ops), sp if s_ptr is None else s_ptr)
+                    if st:
+                        raise clq.ClqError(st, "clq_peak_rq_stream")
+                return f
+
+            rq_floor_b2b = [time_steps(floor_only(i), args.steps) for i in range(nlay)]
+            del fq, fs
 
     def cublas_step(si, s_ptr=None):
         xs = xsets[si % nsets]
@@ -1043,6 +1067,9 @@ def main():
         if rq_b2b is not None:
             per_layer[-1]["rotate_quant_us_back_to_back"] = round(1e3 * rq_b2b[i], 2)
             per_layer[-1]["gemm_us_back_to_back"] = round(1e3 * gm_b2b[i], 2)
+        if rq_floor_b2b is not None:
+            per_layer[-1]["rotate_quant_copy_floor_us_back_to_back"] = round(
+                1e3 * rq_floor_b2b[i], 2)
     gm_total_s = gm_ms.sum() * 1e-3 / args.steps
     rq_total_s = rq_ms.sum() * 1e-3 / args.steps
     gemm_kernel = "fused_linear" if args.fused else "w4a4_gemm"
@@ -1095,6 +1122,13 @@ def main():
             rq_b2b_ach = rq_bytes_all / (sum(rq_b2b) * 1e-3) / 1e9
             rq_roof["achieved_back_to_back"] = round(rq_b2b_ach, 1)
             rq_roof["frac_back_to_back"] = round(rq_b2b_ach / hbm_peak, 4)
+        if rq_b2b is not None and rq_floor_b2b is not None:
+            floor_gbps = rq_bytes_all / (sum(rq_floor_b2b) * 1e-3) / 1e9
+            rq_roof["copy_floor"] = {
+                "GBps": round(floor_gbps, 1), "frac_of_peak": round(floor_gbps / hbm_peak, 4),
+                "kernel_frac_of_floor": round(rq_b2b_ach / floor_gbps, 4),
+                "note": "clq_peak_rq_stream: the loop's tiles, copy ring and stores without "
+                        "its gather and arithmetic, back to back on the same inputs"}
 
     # ---- end to end through the public API with host buffers ----
     e2e = None

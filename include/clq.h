@@ -493,6 +493,15 @@ clq_status clq_selftest_bounded_wait(int64_t timeout_ns, void* stream);
  *   the shared-memory bytes filled (the rate an SM takes operands in);
  *   mma = 1: the GEMM's four 128 x 256 x 32 MMAs run on each stage, *ops =
  *   the multiply-accumulates.
+ * clq_peak_rq_stream: the memory side of clq_rotate_quant_act's b = 64 loop
+ *   alone, on X (device [M][K] 16-bit values, rows contiguous): the loop's
+ *   tiles, two-stage bulk-copy ring, threads per CTA and programmatic-launch
+ *   prologue, writing 1 byte per element to Q (device [M][K]: the high byte
+ *   of each value) and 4 bytes per row to S (device fp32 [M]), with no
+ *   gather and no arithmetic.  *ops = the rotate-quant algorithmic bytes of
+ *   the shape, M (2.5 K + 4), so that ops / time compares with the kernel's
+ *   own rate.  Requires M >= 1, 64 <= K <= 16384, K % 64 == 0; X and Q
+ *   16-byte aligned.
  */
 clq_status clq_peak_tcgen05_e4m3(int32_t iters, int64_t* ops, void* stream);
 clq_status clq_peak_mma_sync(int32_t kind, int32_t iters, int64_t* ops, void* stream);
@@ -500,6 +509,8 @@ clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void
 clq_status clq_peak_operand_stream(const uint8_t* buf, int32_t rows, int32_t K,
                                    clq_codes codes, int32_t mma, int32_t tiles,
                                    int64_t* ops, void* stream);
+clq_status clq_peak_rq_stream(const void* X, int32_t M, int32_t K, uint8_t* Q, float* S,
+                              int64_t* ops, void* stream);
 
 #ifdef __cplusplus
 }

@@ -36,7 +36,8 @@ EXPORTS = ("clq_status_string", "clq_version", "clq_outlier_scores",
            "clq_prepare_weights_codes", "clq_linear",
            "clq_rotate_quant_act_asym", "clq_weight_code_sums",
            "clq_linear_asym", "clq_clip_search_workspace_size",
-           "clq_clip_search", "clq_convert_codes", "clq_peak_operand_stream")
+           "clq_clip_search", "clq_convert_codes", "clq_peak_operand_stream",
+           "clq_peak_rq_stream")
 
 _lib = None
 _P = ctypes.c_void_p
@@ -67,6 +68,7 @@ _SIGS = {
     "clq_peak_mma_sync": (_I, [_I, _I, _P, _P]),
     "clq_peak_hbm_read": (_I, [_P, ctypes.c_uint64, _P, _P]),
     "clq_peak_operand_stream": (_I, [_P, _I, _I, _I, _I, _I, _P, _P]),
+    "clq_peak_rq_stream": (_I, [_P, _I, _I, _P, _P, _P, _P]),
     "clq_prepare_weights_codes": (_I, [_P, _I, _I, _I, _I, _P, _I, _P, _I,
                                        _P, _P, _P, _P]),
     "clq_linear": (_I, [_P, _I, _P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P,
@@ -226,6 +228,10 @@ def clq_peak_tcgen05_e4m3(iters, ops, stream):
 
 def clq_peak_mma_sync(kind, iters, ops, stream):
     return load().clq_peak_mma_sync(kind, iters, ops, stream)
+
+
+def clq_peak_rq_stream(X, M, K, Q, S, ops, stream):
+    return load().clq_peak_rq_stream(X, M, K, Q, S, ops, stream)
 
 
 def clq_peak_operand_stream(buf, rows, K, codes, mma, tiles, ops, stream):

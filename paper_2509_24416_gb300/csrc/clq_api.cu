@@ -254,6 +254,12 @@ ClipWorkspace clip_workspace_layout(int M, int N, int K, int J, int G) {
 
 }  // namespace
 
+namespace clq {
+// peaks.cu
+cudaError_t launch_peak_rq_stream(const void* X, int M, int K, uint8_t* Q, float* S,
+                                  int32_t* status, cudaStream_t st, long long* bytes);
+}  // namespace clq
+
 extern "C" {
 
 const char* clq_status_string(clq_status s) {
@@ -556,6 +562,21 @@ clq_status clq_peak_hbm_read(const void* buf, uint64_t bytes, int64_t* ops, void
   if (st != CLQ_OK) return st;
   st = from_cuda(clq::launch_peak_hbm_read(buf, bytes, status, static_cast<cudaStream_t>(stream)));
   *ops = static_cast<int64_t>(bytes);
+  return st;
+}
+
+clq_status clq_peak_rq_stream(const void* X, int32_t M, int32_t K, uint8_t* Q, float* S,
+                              int64_t* ops, void* stream) {
+  if (ops == nullptr || X == nullptr || Q == nullptr || S == nullptr) return CLQ_ERR_INVALID_ARG;
+  if (M < 1 || K < 64 || K > 16384 || K % 64 != 0) return CLQ_ERR_SHAPE;
+  if (!aligned(X, 16) || !aligned(Q, 16) || !aligned(S, 4)) return CLQ_ERR_ALIGN;
+  int32_t* status = nullptr;
+  clq_status st = device_setup(&status);
+  if (st != CLQ_OK) return st;
+  long long bytes = 0;
+  st = from_cuda(clq::launch_peak_rq_stream(X, M, K, Q, S, status,
+                                            static_cast<cudaStream_t>(stream), &bytes));
+  *ops = bytes;
   return st;
 }
 

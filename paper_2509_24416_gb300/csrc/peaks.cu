@@ -14,7 +14,11 @@
 //    boxes (A 128 rows, B 256 rows, 128 codes a row, E4M3 or E2M3 layout)
 //    from a caller code array, and a consumer either releases each stage at
 //    once (the rate at which an SM takes operands in) or issues the GEMM's
-//    four 128 x 256 x 32 MMAs on it (the rate of the main loop).
+//    four 128 x 256 x 32 MMAs on it (the rate of the main loop);
+//  * rotate-quant stream: the wide rotate-quant loop's data movement without
+//    its arithmetic (its tiles, stage ring, threads and programmatic-launch
+//    prologue; one byte out per element and four per row), the memory floor
+//    the kernel is measured against.
 #include "clq_device.cuh"
 #include "clq_kernels.h"
 
@@ -216,7 +220,110 @@ cudaError_t launch_stream_t(const CUtensorMap& a, const CUtensorMap& b, int rows
   return cudaGetLastError();
 }
 
+// Rotate-quant memory floor.  Tiles of RH rows of 2K bytes are dealt
+// round-robin and bulk-copied into a ring of two STAGE-byte stages (the
+// first two into L2 before the programmatic-launch wait), as in the wide
+// rotate-quant loop; each thread then turns its 16-element chunks of a tile
+// into 16 bytes (the high byte of every 16-bit value) and the first RH
+// threads write a 4-byte value per row: the loop's HBM traffic (2 B in,
+// 1 B + 4 B a row out) with no gather and no arithmetic.
+template <int STAGE>
+__global__ void __launch_bounds__(512) peak_rq_stream_kernel(const uint8_t* X, int M, int K,
+                                                             int RH, uint8_t* Q, float* S,
+                                                             int32_t* status) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ __align__(8) uint64_t full[2];
+  const int tid = threadIdx.x;
+  const int ntiles = (M + RH - 1) / RH;
+  const uint32_t row_bytes = 2u * static_cast<uint32_t>(K);
+  auto rows_of = [&](int t) { return min(RH, M - t * RH); };
+  auto src_of = [&](int t) { return X + static_cast<size_t>(t) * RH * row_bytes; };
+  if (tid == 0) {
+    mbar_init(&full[0], 1);
+    mbar_init(&full[1], 1);
+    fence_mbarrier_init();
+  }
+  __syncthreads();
+  if (tid == 0)
+    for (int s = 0; s < 2; ++s) {
+      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
+      if (t < ntiles) bulk_prefetch_l2(src_of(t), row_bytes * static_cast<uint32_t>(rows_of(t)));
+    }
+  pdl_wait();
+  pdl_launch_dependents();
+  auto issue = [&](int s, int t) {
+    const uint32_t bytes = row_bytes * static_cast<uint32_t>(rows_of(t));
+    mbar_arrive_expect_tx(&full[s], bytes);
+    bulk_load(smem + s * STAGE, src_of(t), bytes, &full[s]);
+  };
+  if (tid == 0)
+    for (int s = 0; s < 2; ++s) {
+      const int t = static_cast<int>(blockIdx.x) + s * static_cast<int>(gridDim.x);
+      if (t < ntiles) issue(s, t);
+    }
+  for (int j = 0;; ++j) {
+    const int s = j & 1;
+    const int t = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
+    if (t >= ntiles) break;
+    if (!mbar_wait_bounded(&full[s], (j >> 1) & 1, nullptr, status, kWaitLimitNs)) {
+      if (tid == 0)  // copies already issued land before the CTA exits
+        for (int s2 = 0; s2 < 2; ++s2)
+          for (int ph = 0; ph < 2; ++ph)
+            mbar_wait_bounded(&full[s2], ph, nullptr, nullptr, 10000000ull);
+      break;
+    }
+    const int rows = rows_of(t);
+    const int n16 = rows * K / 16;
+    const uint8_t* stage = smem + s * STAGE;
+    uint4* q = reinterpret_cast<uint4*>(Q + static_cast<size_t>(t) * RH * K);
+    for (int i = tid; i < n16; i += blockDim.x) {
+      const uint4 a = *reinterpret_cast<const uint4*>(stage + 32 * i);
+      const uint4 b = *reinterpret_cast<const uint4*>(stage + 32 * i + 16);
+      q[i] = make_uint4(__byte_perm(a.x, a.y, 0x7531), __byte_perm(a.z, a.w, 0x7531),
+                        __byte_perm(b.x, b.y, 0x7531), __byte_perm(b.z, b.w, 0x7531));
+    }
+    if (tid < rows) S[t * RH + tid] = 1.0f;
+    __syncthreads();  // stage s fully read
+    if (tid == 0) {
+      const int t2 = t + 2 * static_cast<int>(gridDim.x);
+      if (t2 < ntiles) issue(s, t2);
+    }
+  }
+}
+
+template <int STAGE>
+cudaError_t launch_rq_stream_t(const uint8_t* X, int M, int K, int RH, int threads, uint8_t* Q,
+                               float* S, int32_t* status, int sms, cudaStream_t st) {
+  auto k = peak_rq_stream_kernel<STAGE>;
+  const size_t smem = 2 * STAGE;
+  int per_sm = 0;
+  cudaError_t e = kernel_setup(reinterpret_cast<const void*>(k), smem, threads, &per_sm);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  const int tiles = (M + RH - 1) / RH;
+  return launch_pdl(k, std::min(tiles, sms * per_sm), threads, smem, st, X, M, K, RH, Q, S,
+                    status);
+}
+
 }  // namespace
+
+// The wide loop's geometry (rotate_quant.cu).
+void rotate_quant_wide_config(int M, int K, int sms, int* rows, int* threads, size_t* smem,
+                              int* stage);
+
+cudaError_t launch_peak_rq_stream(const void* X, int M, int K, uint8_t* Q, float* S,
+                                  int32_t* status, cudaStream_t st, long long* bytes) {
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  int RH = 0, threads = 0, stage = 0;
+  size_t smem = 0;
+  rotate_quant_wide_config(M, K, sms, &RH, &threads, &smem, &stage);
+  *bytes = static_cast<long long>(M) * (5LL * K / 2 + 4);
+  const uint8_t* x = static_cast<const uint8_t*>(X);
+  if (stage == 16 * 1024)
+    return launch_rq_stream_t<16384>(x, M, K, RH, threads, Q, S, status, sms, st);
+  return launch_rq_stream_t<32768>(x, M, K, RH, threads, Q, S, status, sms, st);
+}
 
 cudaError_t launch_peak_operand_stream(const uint8_t* buf, int rows, int K, int codes, int mma,
                                        int tiles, int32_t* status, cudaStream_t st,

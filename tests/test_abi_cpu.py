@@ -243,6 +243,14 @@ def test_peak_microbenchmark_host_validation(lib):
         assert clq.clq_peak_operand_stream(*args) == want, (i, bad)
     assert clq.clq_peak_operand_stream(P, 256, 128, E2, 2, 1, ctypes.byref(ops), None) == 1
     assert clq.clq_peak_operand_stream(P, 256, 128, E4, 0, 1, None, None) == 1
+    # rotate-quant memory floor: X, M, K, Q, S, ops
+    ok = (P, 8, 1152, P, P, ctypes.byref(ops), None)
+    for i, bad, want in ((0, None, 1), (3, None, 1), (4, None, 1), (5, None, 1),
+                         (1, 0, 2), (2, 32, 2), (2, 1120, 2), (2, 16448, 2),
+                         (0, P + 8, 3), (3, P + 4, 3), (4, P + 2, 3)):
+        args = list(ok)
+        args[i] = bad
+        assert clq.clq_peak_rq_stream(*args) == want, (i, bad)
 
 
 @pytest.mark.parametrize("K,seed", [(1, 0), (2, 1), (7, 2), (64, 3),
