@@ -23,7 +23,7 @@
 namespace clq {
 namespace rq {
 
-constexpr int kWideMaxRegs = 160;
+constexpr int kWideMaxRegs = 168;
 
 // Shared memory of the wide loop: STAGES stages of STAGE bytes, row maxima
 // and (asymmetric codes) row minima [3][RH] each, STAGES barriers, abort flag.
