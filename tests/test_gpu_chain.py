@@ -20,12 +20,12 @@ M = 4096
 WIDTHS = (1152, 1152, 2304, 1152)  # K of the first layer, then each layer's N
 
 
-def _layers(seed, b, a_bits=4, w_bits=4):
+def _layers(seed, b, a_bits=4, w_bits=4, dtype=torch.float16):
     g = torch.Generator().manual_seed(seed)
     out = []
     for K, N in zip(WIDTHS[:-1], WIDTHS[1:]):
-        W = (torch.randn(N, K, generator=g) * (1.0 / K ** 0.5)).half().to(DEV)
-        bias = (torch.randn(N, generator=g) * 0.01).half().to(DEV)
+        W = (torch.randn(N, K, generator=g) * (1.0 / K ** 0.5)).to(dtype).to(DEV)
+        bias = (torch.randn(N, generator=g) * 0.01).to(dtype).to(DEV)
         perm = torch.randperm(K, generator=g).to(torch.int32).to(DEV)
         out.append(clq.PreparedLinear.from_weight(W, perm, b, bias=bias, a_bits=a_bits,
                                                   w_bits=w_bits))
@@ -36,7 +36,7 @@ def _check_chain(run_layer, x0, reps=3):
     ref = []
     x = x0
     for i in range(len(WIDTHS) - 1):
-        y = torch.empty((M, WIDTHS[i + 1]), dtype=torch.float16, device=DEV)
+        y = torch.empty((M, WIDTHS[i + 1]), dtype=x0.dtype, device=DEV)
         run_layer(i, x, y)
         torch.cuda.synchronize()
         ref.append(y)
@@ -56,21 +56,25 @@ def _check_chain(run_layer, x0, reps=3):
             assert torch.equal(y.view(torch.int16), r.view(torch.int16))
 
 
-def _x0(seed):
+def _x0(seed, dtype=torch.float16):
     g = torch.Generator().manual_seed(seed)
-    return (torch.randn(M, WIDTHS[0], generator=g) * 3).half().to(DEV)
+    return (torch.randn(M, WIDTHS[0], generator=g) * 3).to(dtype).to(DEV)
 
 
-@pytest.mark.parametrize("b,a_bits,fused", [(64, 4, False), (128, 4, False), (64, 8, False),
-                                            (64, 4, True)])
-def test_chained_layers_equal_synchronized(b, a_bits, fused):
-    layers = _layers(11, b, a_bits=a_bits)
+@pytest.mark.parametrize("b,a_bits,fused,dtype", [(64, 4, False, torch.float16),
+                                                  (128, 4, False, torch.float16),
+                                                  (64, 8, False, torch.float16),
+                                                  (64, 4, True, torch.float16),
+                                                  (64, 4, False, torch.bfloat16),
+                                                  (128, 4, False, torch.bfloat16)])
+def test_chained_layers_equal_synchronized(b, a_bits, fused, dtype):
+    layers = _layers(11, b, a_bits=a_bits, dtype=dtype)
     ws = [clq.fused_workspace(M, K, DEV) if fused else None for K in WIDTHS[:-1]]
 
     def run_layer(i, x, y):
         layers[i](x, fused=fused, workspace=ws[i], Y=y)
 
-    _check_chain(run_layer, _x0(12))
+    _check_chain(run_layer, _x0(12, dtype))
 
 
 def test_chained_asymmetric_layers_equal_synchronized():
