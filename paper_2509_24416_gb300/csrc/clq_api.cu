@@ -281,7 +281,7 @@ const char* clq_status_string(clq_status s) {
   }
 }
 
-int32_t clq_version(void) { return 101; }
+int32_t clq_version(void) { return 102; }
 
 clq_status clq_build_permutation(const float* host_scores, int32_t K, int32_t* host_perm) {
   if (host_scores == nullptr || host_perm == nullptr || K < 1) return CLQ_ERR_INVALID_ARG;

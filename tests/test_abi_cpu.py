@@ -39,7 +39,7 @@ def test_all_symbols_exported(lib):
 def test_status_strings(lib):
     for code, name in clq.STATUS.items():
         assert lib.clq_status_string(code).decode().startswith(name)
-    assert lib.clq_version() == 101
+    assert lib.clq_version() == 102
 
 
 P = 1 << 20  # a fake, 16-byte aligned "device" address; never dereferenced
